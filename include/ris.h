@@ -1,0 +1,204 @@
+/*
+ * ris.h -- C ABI of libris, the GB300 (sm_103a) implementation of RIS (Reduced
+ * Interaction Sampling) prefill sparse self-attention, arxiv 2607.21927.
+ *
+ * Conventions shared by every call
+ *   - Tensors are caller-owned, contiguous, token-major DEVICE pointers unless a comment
+ *     says "host". q is [N][heads][head_dim], k and v are [N][kv_heads][head_dim], out is
+ *     [N][heads][head_dim] (per-seed calls: [n_seeds][N][heads][head_dim]).
+ *     Every device pointer must be 16-byte aligned.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). Calls
+ *     are stream-ordered and asynchronous unless their comment says "blocks".
+ *   - Each call returns a ris_status. Arguments are validated before anything is launched;
+ *     an invalid call launches nothing and returns RIS_ERR_INVALID. The text of the last
+ *     error of the calling thread is returned by ris_last_error(). A device fault of an
+ *     earlier launch surfaces as RIS_ERR_CUDA from a later call or at the caller's sync.
+ *   - There is no CPU fallback: without a CUDA device every compute call returns
+ *     RIS_ERR_CUDA.
+ *   - Temporary device memory is taken from the device's stream-ordered pool
+ *     (cudaMallocAsync on `stream`) and released on the same stream.
+ */
+#ifndef RIS_H
+#define RIS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    RIS_OK = 0,
+    RIS_ERR_INVALID = 1,        /* bad argument; nothing was launched */
+    RIS_ERR_OOM = 2,            /* device allocation failed */
+    RIS_ERR_CUDA = 3,           /* a CUDA runtime call failed (or no device) */
+    RIS_ERR_UNSUPPORTED = 4,    /* valid but not built (e.g. head_dim outside {64,128}) */
+    RIS_ERR_DEVICE_TIMEOUT = 5  /* a bounded device-side wait gave up */
+} ris_status;
+
+/* Sampling modes (paper, Methods, "Sampling Modes: Stochastic and Structural"). */
+typedef enum {
+    RIS_MODE_STOCHASTIC = 0, /* the whole density budget drawn uniformly per pivot row */
+    RIS_MODE_STRUCTURAL = 1, /* block cliques of B = min(0.1 N, round(d N)) + global draws */
+    RIS_MODE_DENSE = 2       /* every causal pair (the dense upper bound, Table tab:results_32k) */
+} ris_mode;
+
+typedef enum { RIS_F32 = 0, RIS_BF16 = 1 } ris_dtype;
+
+/* RoPE position extension (Methods, "Dynamic RoPE Scaling"). */
+typedef enum { RIS_ROPE_NONE = 0, RIS_ROPE_PLAIN = 1, RIS_ROPE_LINEAR = 2, RIS_ROPE_YARN = 3 } ris_rope_kind;
+
+typedef struct {
+    int32_t kind;       /* ris_rope_kind */
+    int32_t reserved;   /* must be 0 */
+    double theta;       /* base, e.g. 1e6 (Qwen2) or 1e4 (TinyLlama) */
+    int64_t native_len; /* trained positional limit, e.g. 32768 or 2048 */
+    double factor;      /* extension factor s; <= 0 resolves to max(1, N / native_len) */
+    double yarn_alpha;  /* YaRN ramp start in rotations per native window (default 1) */
+    double yarn_beta;   /* YaRN ramp end (default 32) */
+} ris_rope_cfg;
+
+/* Forced set and keying of a mask; NULL means all defaults. */
+typedef struct {
+    int32_t local_window; /* W >= 1: keys i-W < j <= i always kept (1 = diagonal only, default) */
+    int32_t n_anchor;     /* A >= 0: keys j < A always kept (global anchors, default 0) */
+    int32_t per_head;     /* 0: one mask shared by all heads (default); 1: one mask per KV head */
+    uint32_t layer_key;   /* mixed into every draw; 0 = shared across layers (default) */
+} ris_mask_opts;
+
+/* Derived scalars of one call, resolved on the host. */
+typedef struct {
+    int64_t bmax;            /* K = floor(d N + 0.5), the paper's B_max */
+    int64_t block;           /* Structural block size B = max(1, min(floor(N/10), K)) */
+    int64_t clique_pairs;    /* C, causal clique pairs of all blocks */
+    double d_clique;         /* C / N^2 */
+    double d_global;         /* max(0, d - d_clique): Structural global draw density */
+    uint64_t thr;            /* keep iff Philox word < thr; 2^32 = always */
+    uint32_t stream;         /* Philox counter word 2: 0 Stochastic draws, 1 Structural global */
+    int32_t dense;           /* 1 when every causal pair is kept (dense mode or density 1) */
+    double rope_factor;      /* resolved s */
+    double rope_mscale;      /* 0.1 ln s + 1 for YaRN, else 1 */
+} ris_params;
+
+/* Opaque handle to a mask held in device memory. */
+typedef struct ris_mask_s *ris_mask_t;
+
+/* Device-side layout of a mask, read by ris_mask_info. All pointers are owned by the mask.
+ *   n_masks = (per_seed ? n_seeds : 1) * (per_head ? kv_heads : 1); mask m = s * heads_keyed + h.
+ *   CSR: keys of row i of mask m are col[row_ptr[m*N + i] .. row_ptr[m*N + i + 1]),
+ *        ascending, int64 row_ptr of n_masks*N + 1 entries, col of col_bytes (2 if N <= 65536,
+ *        else 4) each.
+ *   Bitmap: row i of mask m holds words floor(i/32)+1 words at
+ *        bitmap + m * words_per_mask + row_word_offset(i), with
+ *        row_word_offset(32a + b) = 32a + b + 16 a (a - 1) + a b; bit (j mod 32) of word j/32
+ *        is pair (i, j); bits above the diagonal are zero.
+ *   Dense masks (mode DENSE or density 1) store nothing: row_ptr, col and bitmap are NULL
+ *   and row i holds keys 0..i. */
+typedef struct {
+    int64_t N;
+    int32_t n_masks;
+    int32_t heads_keyed;   /* 1, or kv_heads when per_head */
+    int32_t n_seeds;
+    int32_t per_seed;
+    int32_t col_bytes;
+    int32_t dense;
+    int64_t n_pairs;       /* total stored pairs over all masks */
+    int64_t words_per_mask;
+    const int64_t *row_ptr;
+    const void *col;
+    const uint32_t *bitmap;
+    ris_params params;
+} ris_mask_desc;
+
+/* Resolve the scalars of a call on the host (no device work, usable without a GPU).
+ * Structural geometry follows Methods, "Sampling Modes"; B_max = round(d N) matches the
+ * B_max column of the sub-1% sweet-spot table. rope may be NULL (factor 1, mscale 1).
+ * Returns RIS_ERR_INVALID for N < 1, density outside (0, 1], an unknown mode or rope kind. */
+ris_status ris_resolve_params(int64_t N, int32_t mode, double density, const ris_rope_cfg *rope,
+                              ris_params *out);
+
+/* RoPE rotation frequencies f[head_dim/2] (host array, fp64) and the vector scale for a
+ * sequence of N tokens: plain theta^(-2k/D); linear f/s; YaRN ramp between the two
+ * (Methods, "Dynamic RoPE Scaling"; YaRN per Peng et al. 2023). No device work. */
+ris_status ris_rope_freqs(const ris_rope_cfg *rope, int64_t N, int32_t head_dim, double *f_out,
+                          double *mscale_out);
+
+/* Build the RIS mask of N tokens (Methods, "Memory-Bounded Geometry Generation" and
+ * "Sampling Modes"): for every seed, keep causal pair (i, j<i) iff Philox4x32-10 word
+ * (j mod 4) of key (seed, head_key) and counter (j/4, i, stream, layer_key) is below thr;
+ * Structural adds the block cliques; the forced local window and anchors are added; with
+ * per_seed = 0 all seeds are OR-merged into one master mask, with per_seed = 1 each seed
+ * keeps its own mask. Output: bitmap + CSR in device memory owned by *out_mask.
+ * seeds: HOST array of n_seeds values, 1 <= n_seeds <= 256. kv_heads is used only when
+ * opts->per_head = 1. Blocks: the CSR size is read back before the key lists are written.
+ * Errors: RIS_ERR_INVALID (N < 1 or > 2^31, density outside (0,1], bad opts or seeds),
+ * RIS_ERR_OOM, RIS_ERR_CUDA. On error *out_mask is NULL. */
+ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double density,
+                             const uint32_t *seeds, int32_t n_seeds, const ris_mask_opts *opts,
+                             int32_t per_seed, ris_mask_t *out_mask, void *stream);
+
+/* Describe a mask (host struct filled from host-side metadata; no device work). */
+ris_status ris_mask_info(ris_mask_t mask, ris_mask_desc *out);
+
+/* Release a mask's device memory, ordered on the stream it was built on. NULL is a no-op. */
+ris_status ris_mask_free(ris_mask_t mask);
+
+/* Rotate x[N][heads][head_dim] in place with RoPE (rotate-half pairs (c, c + D/2)) at
+ * positions 0..N-1, then scale by mscale (Methods, "Dynamic RoPE Scaling"). Angles are
+ * formed and reduced in fp64; the rotation runs in fp32; bf16 results are rounded to
+ * nearest even. head_dim must be even. Errors: RIS_ERR_INVALID. */
+ris_status ris_rope_apply(void *x, int32_t dtype, int64_t N, int32_t heads, int32_t head_dim,
+                          const ris_rope_cfg *rope, void *stream);
+
+/* RIS sparse attention of one layer (Methods, "Hybrid Anchor and Pre-Fusion Unified Softmax"):
+ *   out[i][h] = sum_{j in M_i} softmax_j(<q~_i,h , k~_j,g> / sqrt(D)) v_j,g,  g = h / (heads/kv_heads)
+ * with one softmax over the whole key set M_i of the master mask (all seeds OR-merged), q~ and
+ * k~ rotated by `rope` (NULL or kind NONE: q and k are used as given). Builds the mask, runs
+ * the attention and frees the mask, all on `stream`; blocks once while the mask is sized.
+ * dtype: q, k, v element type; out_dtype: out element type (F32 or BF16). lse: optional
+ * [heads][N] fp32 natural-log sum of exp of the scaled scores (NULL to skip).
+ * head_dim in {64, 128}; heads a multiple of kv_heads; heads/kv_heads <= 8 (larger groups:
+ * RIS_ERR_UNSUPPORTED).
+ * Errors: RIS_ERR_INVALID, RIS_ERR_UNSUPPORTED, RIS_ERR_OOM, RIS_ERR_CUDA. */
+ris_status ris_sparse_attention_fwd(const void *q, const void *k, const void *v, void *out,
+                                    int64_t N, int32_t heads, int32_t kv_heads, int32_t head_dim,
+                                    int32_t mode, double density, const uint32_t *seeds,
+                                    int32_t n_seeds, int32_t dtype, int32_t out_dtype,
+                                    const ris_rope_cfg *rope, const ris_mask_opts *opts, float *lse,
+                                    void *stream);
+
+/* The attention step alone on a mask built by ris_mask_generate (the mask is built once per
+ * prefill and reused by every layer, Methods, "Memory-Bounded Geometry Generation"). With a
+ * per-seed mask, out is [n_seeds][N][heads][head_dim] and lse [n_seeds][heads][N].
+ * kv_heads must equal the mask's kv_heads when it is keyed per head. Asynchronous.
+ * Errors: as ris_sparse_attention_fwd. */
+ris_status ris_attention_masked(ris_mask_t mask, const void *q, const void *k, const void *v,
+                                void *out, int32_t heads, int32_t kv_heads, int32_t head_dim,
+                                int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
+                                float *lse, void *stream);
+
+/* Ensemble of per-seed sparse views in one launch: seed s attends over F + M_s only and
+ * writes out[s] (the "independent sparse views" read of Results, "Linear Interpolation";
+ * union coverage of Eq. union_coverage is the OR of these views). Same arguments as
+ * ris_sparse_attention_fwd; out is [n_seeds][N][heads][head_dim], lse [n_seeds][heads][N]. */
+ris_status ris_ensemble_batch(const void *q, const void *k, const void *v, void *out, int64_t N,
+                              int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t mode,
+                              double density, const uint32_t *seeds, int32_t n_seeds,
+                              int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
+                              const ris_mask_opts *opts, float *lse, void *stream);
+
+/* Text of the calling thread's last error ("" if none). The string is owned by the library. */
+const char *ris_last_error(void);
+
+/* Number of kernels this library has launched since it was loaded (all threads). */
+int64_t ris_launch_count(void);
+
+/* Library version string. */
+const char *ris_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RIS_H */

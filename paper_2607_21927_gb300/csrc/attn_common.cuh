@@ -1,0 +1,70 @@
+// Device helpers shared by the attention kernels of libris.
+#pragma once
+
+#include <cuda_bf16.h>
+
+#include <cstdint>
+
+#include "ris_internal.h"
+
+namespace ris {
+
+constexpr int kAttnWarps = 4;  // tasks (one per warp) per CTA
+constexpr float kLn2 = 0.69314718055994530942f;
+
+// A task is (output set s, row i, KV head g). Rows are handed out from the last (longest
+// key list) to the first so the short rows fill the tail of the grid.
+struct Task {
+    int64_t i;
+    int g;
+    int s;
+    int mask_id;
+};
+
+__device__ __forceinline__ Task decode_task(const AttnArgs &a, int64_t t)
+{
+    Task k;
+    k.g = (int)(t % a.Hkv);
+    const int64_t r = t / a.Hkv;
+    k.s = (int)(r % a.n_sets);
+    k.i = a.N - 1 - r / a.n_sets;
+    k.mask_id = k.s * a.heads_keyed + (a.heads_keyed > 1 ? k.g : 0);
+    return k;
+}
+
+// Key range of a task: [beg, beg + n) of the CSR, or keys 0..i when dense.
+template <bool DENSE>
+__device__ __forceinline__ void key_range(const AttnArgs &a, const Task &t, int64_t &beg, int64_t &n)
+{
+    if (DENSE) {
+        beg = 0;
+        n = t.i + 1;
+    } else {
+        const int64_t rr = (int64_t)t.mask_id * a.N + t.i;
+        beg = a.row_ptr[rr];
+        n = a.row_ptr[rr + 1] - beg;
+    }
+}
+
+template <bool DENSE, typename TIdx>
+__device__ __forceinline__ int key_at(const TIdx *cols, int64_t pos)
+{
+    if (DENSE) return (int)pos;
+    return (int)cols[pos];
+}
+
+__device__ __forceinline__ float warp_max(float x)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xFFFFFFFFu, x, o));
+    return x;
+}
+
+__device__ __forceinline__ float warp_sum(float x)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+    return x;
+}
+
+}  // namespace ris

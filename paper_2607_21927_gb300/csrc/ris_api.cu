@@ -1,0 +1,573 @@
+// libris C ABI: argument validation, host-side parameter resolution, mask objects and the
+// launch sequence of each call. Every step of the path runs in this library's kernels; this
+// file only decides, allocates (stream-ordered pool) and launches.
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+
+#include "ris_internal.h"
+
+namespace ris {
+
+static std::atomic<int64_t> g_launches{0};
+void note_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+cudaError_t launch_attention_bf16(const AttnArgs &a, int D, int out_dtype, bool q_split, int col_bytes,
+                                  bool dense, cudaStream_t s);
+cudaError_t launch_attention_f32(const AttnArgs &a, int D, int out_dtype, int col_bytes, bool dense,
+                                 cudaStream_t s);
+
+}  // namespace ris
+
+using namespace ris;
+
+struct ris_mask_s {
+    int64_t N = 0;
+    int32_t n_masks = 0, heads_keyed = 1, kv_heads = 1, n_seeds = 0, per_seed = 0;
+    int32_t col_bytes = 2, dense = 0;
+    int64_t n_pairs = 0, words_per_mask = 0;
+    int64_t *row_ptr = nullptr;
+    void *col = nullptr;
+    uint32_t *bitmap = nullptr;
+    ris_params params{};
+    cudaStream_t stream = nullptr;
+};
+
+namespace {
+
+thread_local std::string t_err;
+
+ris_status fail(ris_status st, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    t_err = buf;
+    return st;
+}
+
+ris_status cuda_fail(cudaError_t e, const char *what)
+{
+    cudaGetLastError();  // clear a sticky launch error of this thread
+    return fail(e == cudaErrorMemoryAllocation ? RIS_ERR_OOM : RIS_ERR_CUDA, "%s: %s", what,
+                cudaGetErrorString(e));
+}
+
+#define RIS_CUDA(call)                                        \
+    do {                                                      \
+        cudaError_t e_ = (call);                              \
+        if (e_ != cudaSuccess) return cuda_fail(e_, #call);   \
+    } while (0)
+
+// Keep freed pool memory cached in the process (the default pool would hand it back to the
+// driver at every synchronisation, and re-mapping gigabytes costs milliseconds).
+void prepare_pool_once()
+{
+    static std::mutex mu;
+    static bool done[64] = {false};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return;
+    std::lock_guard<std::mutex> lk(mu);
+    if (done[dev]) return;
+    cudaMemPool_t pool;
+    if (cudaDeviceGetDefaultMemPool(&pool, dev) == cudaSuccess) {
+        uint64_t thr = UINT64_MAX;
+        cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &thr);
+    }
+    done[dev] = true;
+}
+
+// Stream-ordered temporary buffer, released on its stream when it leaves scope.
+struct Scratch {
+    void *p = nullptr;
+    cudaStream_t s = nullptr;
+    cudaError_t alloc(size_t bytes, cudaStream_t st)
+    {
+        s = st;
+        return cudaMallocAsync(&p, bytes < 16 ? 16 : bytes, st);
+    }
+    void *release()
+    {
+        void *q = p;
+        p = nullptr;
+        return q;
+    }
+    ~Scratch()
+    {
+        if (p) cudaFreeAsync(p, s);
+    }
+};
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int64_t row_word_offset(int64_t i)
+{
+    const int64_t a = i >> 5, b = i & 31;
+    return i + 16 * a * (a - 1) + a * b;
+}
+
+ris_status check_N(int64_t N)
+{
+    if (N < 1 || N > 2147483647LL) return fail(RIS_ERR_INVALID, "N=%lld outside [1, 2^31-1]", (long long)N);
+    return RIS_OK;
+}
+
+ris_status check_mode_density(int32_t mode, double density)
+{
+    if (mode < RIS_MODE_STOCHASTIC || mode > RIS_MODE_DENSE) return fail(RIS_ERR_INVALID, "unknown mode %d", mode);
+    if (!(density > 0.0 && density <= 1.0)) return fail(RIS_ERR_INVALID, "density %g outside (0, 1]", density);
+    return RIS_OK;
+}
+
+ris_status check_rope(const ris_rope_cfg *r)
+{
+    if (r == nullptr) return RIS_OK;
+    if (r->kind < RIS_ROPE_NONE || r->kind > RIS_ROPE_YARN) return fail(RIS_ERR_INVALID, "unknown rope kind %d", r->kind);
+    if (r->kind == RIS_ROPE_NONE) return RIS_OK;
+    if (r->reserved != 0) return fail(RIS_ERR_INVALID, "rope.reserved must be 0");
+    if (!(r->theta > 1.0) || !std::isfinite(r->theta)) return fail(RIS_ERR_INVALID, "rope.theta %g must be > 1", r->theta);
+    if (r->native_len < 1) return fail(RIS_ERR_INVALID, "rope.native_len must be >= 1");
+    if (!std::isfinite(r->factor) || (r->factor > 0.0 && r->factor < 1.0))
+        return fail(RIS_ERR_INVALID, "rope.factor %g must be <= 0 (auto) or >= 1", r->factor);
+    if (r->kind == RIS_ROPE_YARN && !(r->yarn_beta > r->yarn_alpha))
+        return fail(RIS_ERR_INVALID, "rope.yarn_beta must exceed rope.yarn_alpha");
+    return RIS_OK;
+}
+
+ris_status check_opts(const ris_mask_opts *o)
+{
+    if (o == nullptr) return RIS_OK;
+    if (o->local_window < 1) return fail(RIS_ERR_INVALID, "local_window %d must be >= 1", o->local_window);
+    if (o->n_anchor < 0) return fail(RIS_ERR_INVALID, "n_anchor %d must be >= 0", o->n_anchor);
+    if (o->per_head != 0 && o->per_head != 1) return fail(RIS_ERR_INVALID, "per_head must be 0 or 1");
+    return RIS_OK;
+}
+
+ris_status check_seeds(const uint32_t *seeds, int32_t n_seeds)
+{
+    if (n_seeds < 1 || n_seeds > kMaxSeeds) return fail(RIS_ERR_INVALID, "n_seeds %d outside [1, %d]", n_seeds, kMaxSeeds);
+    if (seeds == nullptr) return fail(RIS_ERR_INVALID, "seeds is NULL");
+    return RIS_OK;
+}
+
+ris_status check_shape(int32_t heads, int32_t kv_heads, int32_t head_dim)
+{
+    if (heads < 1 || kv_heads < 1) return fail(RIS_ERR_INVALID, "heads and kv_heads must be >= 1");
+    if (heads % kv_heads != 0) return fail(RIS_ERR_INVALID, "heads %d not a multiple of kv_heads %d", heads, kv_heads);
+    if (head_dim != 64 && head_dim != 128) return fail(RIS_ERR_INVALID, "head_dim %d not in {64, 128}", head_dim);
+    if (heads / kv_heads > 8) return fail(RIS_ERR_UNSUPPORTED, "heads/kv_heads = %d > 8 is not built", heads / kv_heads);
+    return RIS_OK;
+}
+
+ris_status check_dtype(int32_t dt, const char *what)
+{
+    if (dt != RIS_F32 && dt != RIS_BF16) return fail(RIS_ERR_INVALID, "%s %d is neither F32 nor BF16", what, dt);
+    return RIS_OK;
+}
+
+ris_status check_ptr(const void *p, const char *what)
+{
+    if (p == nullptr) return fail(RIS_ERR_INVALID, "%s is NULL", what);
+    if (!aligned16(p)) return fail(RIS_ERR_INVALID, "%s is not 16-byte aligned", what);
+    return RIS_OK;
+}
+
+#define RIS_TRY(expr)                    \
+    do {                                 \
+        ris_status st_ = (expr);         \
+        if (st_ != RIS_OK) return st_;   \
+    } while (0)
+
+uint64_t keep_threshold(double p)
+{
+    if (!(p > 0.0)) return 0;
+    const double t = std::floor(p * 4294967296.0 + 0.5);
+    return t >= 4294967296.0 ? (uint64_t(1) << 32) : (uint64_t)t;
+}
+
+double resolve_factor(const ris_rope_cfg *r, int64_t N)
+{
+    if (r == nullptr || r->kind == RIS_ROPE_NONE) return 1.0;
+    if (r->factor > 0.0) return r->factor;
+    const double s = (double)N / (double)r->native_len;
+    return s > 1.0 ? s : 1.0;
+}
+
+ris_status validate_attention(const void *q, const void *k, const void *v, void *out, int32_t heads,
+                              int32_t kv_heads, int32_t head_dim, int32_t dtype, int32_t out_dtype,
+                              const ris_rope_cfg *rope, const float *lse)
+{
+    RIS_TRY(check_ptr(q, "q"));
+    RIS_TRY(check_ptr(k, "k"));
+    RIS_TRY(check_ptr(v, "v"));
+    RIS_TRY(check_ptr(out, "out"));
+    if (lse != nullptr && !aligned16(lse)) return fail(RIS_ERR_INVALID, "lse is not 16-byte aligned");
+    RIS_TRY(check_shape(heads, kv_heads, head_dim));
+    RIS_TRY(check_dtype(dtype, "dtype"));
+    RIS_TRY(check_dtype(out_dtype, "out_dtype"));
+    RIS_TRY(check_rope(rope));
+    return RIS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *ris_last_error(void) { return t_err.c_str(); }
+
+int64_t ris_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+const char *ris_version(void) { return "libris 0.1 (sm_103a)"; }
+
+ris_status ris_resolve_params(int64_t N, int32_t mode, double density, const ris_rope_cfg *rope,
+                              ris_params *out)
+{
+    RIS_TRY(check_N(N));
+    RIS_TRY(check_mode_density(mode, density));
+    RIS_TRY(check_rope(rope));
+    if (out == nullptr) return fail(RIS_ERR_INVALID, "out is NULL");
+    ris_params p{};
+    p.bmax = (int64_t)std::floor(density * (double)N + 0.5);
+    int64_t B = std::min<int64_t>(N / 10, p.bmax);
+    if (B < 1) B = 1;
+    const int64_t nb = N / B, rem = N - nb * B;
+    p.block = B;
+    p.clique_pairs = nb * (B * (B + 1) / 2) + rem * (rem + 1) / 2;
+    p.d_clique = (double)p.clique_pairs / ((double)N * (double)N);
+    p.d_global = std::max(0.0, density - p.d_clique);
+    p.dense = (mode == RIS_MODE_DENSE || density >= 1.0) ? 1 : 0;
+    if (p.dense) {
+        p.thr = uint64_t(1) << 32;
+        p.stream = 0;
+    } else if (mode == RIS_MODE_STRUCTURAL) {
+        p.thr = keep_threshold(p.d_global);
+        p.stream = 1;
+    } else {
+        p.thr = keep_threshold(density);
+        p.stream = 0;
+    }
+    p.rope_factor = resolve_factor(rope, N);
+    p.rope_mscale = (rope != nullptr && rope->kind == RIS_ROPE_YARN) ? 0.1 * std::log(p.rope_factor) + 1.0 : 1.0;
+    *out = p;
+    return RIS_OK;
+}
+
+ris_status ris_rope_freqs(const ris_rope_cfg *rope, int64_t N, int32_t head_dim, double *f_out,
+                          double *mscale_out)
+{
+    RIS_TRY(check_N(N));
+    RIS_TRY(check_rope(rope));
+    if (head_dim < 2 || (head_dim & 1) || head_dim > 2 * kMaxHeadDimHalf)
+        return fail(RIS_ERR_INVALID, "head_dim %d must be even and <= %d", head_dim, 2 * kMaxHeadDimHalf);
+    if (f_out == nullptr || mscale_out == nullptr) return fail(RIS_ERR_INVALID, "output pointer is NULL");
+    const double s = resolve_factor(rope, N);
+    const int kind = rope ? rope->kind : RIS_ROPE_NONE;
+    const double theta = (rope && kind != RIS_ROPE_NONE) ? rope->theta : 10000.0;
+    const double two_pi = 6.283185307179586476925286766559;
+    for (int c = 0; c < head_dim / 2; ++c) {
+        const double base = std::pow(theta, -2.0 * (double)c / (double)head_dim);
+        double f = base;
+        if (kind == RIS_ROPE_LINEAR) {
+            f = base / s;
+        } else if (kind == RIS_ROPE_YARN) {
+            // rotations of this frequency inside the native window, ramped between alpha and beta
+            const double r = (double)rope->native_len * base / two_pi;
+            const double gmm = std::min(1.0, std::max(0.0, (r - rope->yarn_alpha) / (rope->yarn_beta - rope->yarn_alpha)));
+            f = (1.0 - gmm) * (base / s) + gmm * base;
+        }
+        f_out[c] = f;
+    }
+    *mscale_out = (kind == RIS_ROPE_YARN) ? 0.1 * std::log(s) + 1.0 : 1.0;
+    return RIS_OK;
+}
+
+ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double density, const uint32_t *seeds,
+                             int32_t n_seeds, const ris_mask_opts *opts, int32_t per_seed, ris_mask_t *out_mask,
+                             void *stream)
+{
+    if (out_mask == nullptr) return fail(RIS_ERR_INVALID, "out_mask is NULL");
+    *out_mask = nullptr;
+    RIS_TRY(check_N(N));
+    RIS_TRY(check_mode_density(mode, density));
+    RIS_TRY(check_seeds(seeds, n_seeds));
+    RIS_TRY(check_opts(opts));
+    if (per_seed != 0 && per_seed != 1) return fail(RIS_ERR_INVALID, "per_seed must be 0 or 1");
+    const ris_mask_opts o = opts ? *opts : ris_mask_opts{1, 0, 0, 0u};
+    if (o.per_head && kv_heads < 1) return fail(RIS_ERR_INVALID, "kv_heads must be >= 1 with per_head");
+    const int32_t heads_keyed = o.per_head ? kv_heads : 1;
+    const int64_t n_masks = (int64_t)(per_seed ? n_seeds : 1) * heads_keyed;
+    if (n_masks * N > 2147483647LL) return fail(RIS_ERR_INVALID, "n_masks * N exceeds 2^31-1");
+
+    ris_params p{};
+    RIS_TRY(ris_resolve_params(N, mode, density, nullptr, &p));
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
+    ris_mask_s *mk = new (std::nothrow) ris_mask_s();
+    if (mk == nullptr) return fail(RIS_ERR_OOM, "host allocation failed");
+    mk->N = N;
+    mk->n_masks = (int32_t)n_masks;
+    mk->heads_keyed = heads_keyed;
+    mk->kv_heads = kv_heads;
+    mk->n_seeds = n_seeds;
+    mk->per_seed = per_seed;
+    mk->col_bytes = N <= 65536 ? 2 : 4;
+    mk->params = p;
+    mk->stream = s;
+    if (p.dense) {
+        mk->dense = 1;
+        mk->n_pairs = n_masks * (N * (N + 1) / 2);
+        *out_mask = mk;
+        return RIS_OK;
+    }
+    prepare_pool_once();
+    struct Guard {
+        ris_mask_s *m;
+        ~Guard()
+        {
+            if (m) ris_mask_free(m);
+        }
+    } guard{mk};
+
+    mk->words_per_mask = row_word_offset(N);
+    const int64_t n_rows = n_masks * N;
+    RIS_CUDA(cudaMallocAsync((void **)&mk->bitmap, sizeof(uint32_t) * (size_t)(n_masks * mk->words_per_mask), s));
+    RIS_CUDA(cudaMallocAsync((void **)&mk->row_ptr, sizeof(int64_t) * (size_t)(n_rows + 1), s));
+    RIS_CUDA(cudaMemsetAsync(mk->row_ptr, 0, sizeof(int64_t), s));
+
+    MaskBitsArgs a{};
+    a.N = N;
+    a.n_seeds = n_seeds;
+    a.per_seed = per_seed;
+    a.heads_keyed = heads_keyed;
+    a.n_masks = (int32_t)n_masks;
+    a.mode = mode;
+    a.W = o.local_window;
+    a.A = o.n_anchor;
+    a.layer_key = o.layer_key;
+    a.stream = p.stream;
+    a.thr = p.thr;
+    a.B = p.block;
+    a.words_per_mask = mk->words_per_mask;
+    a.bitmap = mk->bitmap;
+    a.counts = mk->row_ptr + 1;
+    for (int k = 0; k < n_seeds; ++k) a.seeds.v[k] = seeds[k];
+    RIS_CUDA(launch_mask_bits(a, s));
+
+    Scratch partials;
+    RIS_CUDA(partials.alloc(sizeof(int64_t) * (size_t)scan_partials_count(n_rows), s));
+    RIS_CUDA(launch_scan_inplace(mk->row_ptr + 1, n_rows, (int64_t *)partials.p, s));
+
+    int64_t total = 0;
+    RIS_CUDA(cudaMemcpyAsync(&total, mk->row_ptr + n_rows, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+    RIS_CUDA(cudaStreamSynchronize(s));
+    mk->n_pairs = total;
+    RIS_CUDA(cudaMallocAsync(&mk->col, (size_t)(total > 0 ? total : 1) * mk->col_bytes, s));
+
+    MaskFillArgs f{};
+    f.N = N;
+    f.n_masks = (int32_t)n_masks;
+    f.col_bytes = mk->col_bytes;
+    f.words_per_mask = mk->words_per_mask;
+    f.bitmap = mk->bitmap;
+    f.row_ptr = mk->row_ptr;
+    f.col = mk->col;
+    RIS_CUDA(launch_mask_fill(f, s));
+
+    guard.m = nullptr;
+    *out_mask = mk;
+    return RIS_OK;
+}
+
+ris_status ris_mask_info(ris_mask_t m, ris_mask_desc *out)
+{
+    if (m == nullptr || out == nullptr) return fail(RIS_ERR_INVALID, "mask or out is NULL");
+    ris_mask_desc d{};
+    d.N = m->N;
+    d.n_masks = m->n_masks;
+    d.heads_keyed = m->heads_keyed;
+    d.n_seeds = m->n_seeds;
+    d.per_seed = m->per_seed;
+    d.col_bytes = m->col_bytes;
+    d.dense = m->dense;
+    d.n_pairs = m->n_pairs;
+    d.words_per_mask = m->words_per_mask;
+    d.row_ptr = m->row_ptr;
+    d.col = m->col;
+    d.bitmap = m->bitmap;
+    d.params = m->params;
+    *out = d;
+    return RIS_OK;
+}
+
+ris_status ris_mask_free(ris_mask_t m)
+{
+    if (m == nullptr) return RIS_OK;
+    cudaError_t e = cudaSuccess;
+    if (m->bitmap) e = cudaFreeAsync(m->bitmap, m->stream);
+    if (m->row_ptr) {
+        cudaError_t e2 = cudaFreeAsync(m->row_ptr, m->stream);
+        if (e == cudaSuccess) e = e2;
+    }
+    if (m->col) {
+        cudaError_t e2 = cudaFreeAsync(m->col, m->stream);
+        if (e == cudaSuccess) e = e2;
+    }
+    delete m;
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFreeAsync");
+    return RIS_OK;
+}
+
+ris_status ris_rope_apply(void *x, int32_t dtype, int64_t N, int32_t heads, int32_t head_dim,
+                          const ris_rope_cfg *rope, void *stream)
+{
+    RIS_TRY(check_ptr(x, "x"));
+    RIS_TRY(check_dtype(dtype, "dtype"));
+    RIS_TRY(check_N(N));
+    if (heads < 1) return fail(RIS_ERR_INVALID, "heads must be >= 1");
+    if (head_dim < 8 || (head_dim % 8) || head_dim > 2 * kMaxHeadDimHalf)
+        return fail(RIS_ERR_INVALID, "head_dim %d must be a multiple of 8 in [8, 128]", head_dim);
+    RIS_TRY(check_rope(rope));
+    if (rope == nullptr || rope->kind == RIS_ROPE_NONE) return RIS_OK;
+    RopeArgs a{};
+    double ms = 1.0;
+    RIS_TRY(ris_rope_freqs(rope, N, head_dim, a.f, &ms));
+    a.x_in = x;
+    a.x_out = x;
+    a.N = N;
+    a.H = heads;
+    a.D = head_dim;
+    a.mscale = (float)ms;
+    RIS_CUDA(launch_rope(a, dtype, dtype, reinterpret_cast<cudaStream_t>(stream)));
+    return RIS_OK;
+}
+
+namespace {
+
+// Attention over an existing mask; arguments already validated.
+ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, const void *v, void *out,
+                         int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t dtype, int32_t out_dtype,
+                         const ris_rope_cfg *rope, float *lse, cudaStream_t s)
+{
+    const int64_t N = m->N;
+    prepare_pool_once();
+    Scratch qt, kt, ktl;
+    const void *qu = q, *ku = k, *kl = nullptr;
+    bool q_split = false;
+    if (rope != nullptr && rope->kind != RIS_ROPE_NONE) {
+        RopeArgs ra{};
+        double ms = 1.0;
+        RIS_TRY(ris_rope_freqs(rope, N, head_dim, ra.f, &ms));
+        ra.N = N;
+        ra.D = head_dim;
+        ra.mscale = (float)ms;
+        const size_t nq = (size_t)N * heads * head_dim, nk = (size_t)N * kv_heads * head_dim;
+        // rotated queries in fp32 (split into bf16 hi + lo by the tensor-core path); rotated
+        // keys in fp32, or for bf16 inputs as a bf16 hi + lo pair
+        RIS_CUDA(qt.alloc(nq * sizeof(float), s));
+        RIS_CUDA(kt.alloc(nk * (dtype == RIS_BF16 ? 2 : 4), s));
+        if (dtype == RIS_BF16) RIS_CUDA(ktl.alloc(nk * 2, s));
+        ra.x_in = q;
+        ra.x_out = qt.p;
+        ra.H = heads;
+        RIS_CUDA(launch_rope(ra, dtype, RIS_F32, s));
+        ra.x_in = k;
+        ra.x_out = kt.p;
+        ra.x_out_lo = ktl.p;
+        ra.H = kv_heads;
+        RIS_CUDA(launch_rope(ra, dtype, dtype, s));
+        qu = qt.p;
+        ku = kt.p;
+        kl = ktl.p;
+        q_split = (dtype == RIS_BF16);
+    }
+    AttnArgs a{};
+    a.q = qu;
+    a.k = ku;
+    a.k_lo = kl;
+    a.v = v;
+    a.out = out;
+    a.lse = lse;
+    a.row_ptr = m->row_ptr;
+    a.col = m->col;
+    a.N = N;
+    a.Hq = heads;
+    a.Hkv = kv_heads;
+    a.G = heads / kv_heads;
+    a.heads_keyed = m->heads_keyed;
+    a.n_sets = m->per_seed ? m->n_seeds : 1;
+    a.scale_log2 = (float)(1.4426950408889634074 / std::sqrt((double)head_dim));
+    a.n_tasks = (int64_t)a.n_sets * N * kv_heads;
+    if (dtype == RIS_BF16)
+        RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
+    else
+        RIS_CUDA(launch_attention_f32(a, head_dim, out_dtype, m->col_bytes, m->dense != 0, s));
+    return RIS_OK;
+}
+
+ris_status fwd_common(const void *q, const void *k, const void *v, void *out, int64_t N, int32_t heads,
+                      int32_t kv_heads, int32_t head_dim, int32_t mode, double density, const uint32_t *seeds,
+                      int32_t n_seeds, int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
+                      const ris_mask_opts *opts, float *lse, void *stream, int32_t per_seed)
+{
+    RIS_TRY(validate_attention(q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse));
+    RIS_TRY(check_N(N));
+    RIS_TRY(check_mode_density(mode, density));
+    RIS_TRY(check_seeds(seeds, n_seeds));
+    RIS_TRY(check_opts(opts));
+    ris_mask_t m = nullptr;
+    RIS_TRY(ris_mask_generate(N, kv_heads, mode, density, seeds, n_seeds, opts, per_seed, &m, stream));
+    const ris_status st = run_attention(m, q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse,
+                                        reinterpret_cast<cudaStream_t>(stream));
+    const std::string keep = t_err;
+    const ris_status st2 = ris_mask_free(m);
+    if (st != RIS_OK) {
+        t_err = keep;
+        return st;
+    }
+    return st2;
+}
+
+}  // namespace
+
+ris_status ris_attention_masked(ris_mask_t mask, const void *q, const void *k, const void *v, void *out,
+                                int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t dtype,
+                                int32_t out_dtype, const ris_rope_cfg *rope, float *lse, void *stream)
+{
+    if (mask == nullptr) return fail(RIS_ERR_INVALID, "mask is NULL");
+    RIS_TRY(validate_attention(q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse));
+    if (mask->heads_keyed > 1 && mask->heads_keyed != kv_heads)
+        return fail(RIS_ERR_INVALID, "mask keyed for %d KV heads, call has %d", mask->heads_keyed, kv_heads);
+    return run_attention(mask, q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse,
+                         reinterpret_cast<cudaStream_t>(stream));
+}
+
+ris_status ris_sparse_attention_fwd(const void *q, const void *k, const void *v, void *out, int64_t N,
+                                    int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t mode,
+                                    double density, const uint32_t *seeds, int32_t n_seeds, int32_t dtype,
+                                    int32_t out_dtype, const ris_rope_cfg *rope, const ris_mask_opts *opts,
+                                    float *lse, void *stream)
+{
+    return fwd_common(q, k, v, out, N, heads, kv_heads, head_dim, mode, density, seeds, n_seeds, dtype,
+                      out_dtype, rope, opts, lse, stream, 0);
+}
+
+ris_status ris_ensemble_batch(const void *q, const void *k, const void *v, void *out, int64_t N, int32_t heads,
+                              int32_t kv_heads, int32_t head_dim, int32_t mode, double density,
+                              const uint32_t *seeds, int32_t n_seeds, int32_t dtype, int32_t out_dtype,
+                              const ris_rope_cfg *rope, const ris_mask_opts *opts, float *lse, void *stream)
+{
+    return fwd_common(q, k, v, out, N, heads, kv_heads, head_dim, mode, density, seeds, n_seeds, dtype,
+                      out_dtype, rope, opts, lse, stream, 1);
+}
+
+}  // extern "C"

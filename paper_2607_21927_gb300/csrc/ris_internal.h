@@ -1,0 +1,103 @@
+// Internal declarations shared by the translation units of libris (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "../../include/ris.h"
+
+namespace ris {
+
+constexpr int kMaxSeeds = 256;
+constexpr int kMaxHeadDimHalf = 64;  // head_dim <= 128
+
+// Seeds travel by value in the kernel parameter block (1 KB), so concurrent calls on
+// different streams never share a device-side seed table.
+struct SeedList {
+    uint32_t v[kMaxSeeds];
+};
+
+// Arguments of the mask bitmap kernel (one CTA per (mask, row)).
+struct MaskBitsArgs {
+    int64_t N;
+    int32_t n_seeds;      // seeds drawn per mask (all of them for the union, 1 per seed)
+    int32_t per_seed;     // 1: mask m draws only seed m / heads_keyed
+    int32_t heads_keyed;  // 1 or kv_heads
+    int32_t n_masks;
+    int32_t mode;         // RIS_MODE_STOCHASTIC or RIS_MODE_STRUCTURAL
+    int32_t W;            // local window
+    int32_t A;            // anchors
+    uint32_t layer_key;
+    uint32_t stream;      // Philox counter word 2
+    uint64_t thr;         // keep iff word < thr
+    int64_t B;            // Structural block size
+    int64_t words_per_mask;
+    uint32_t *bitmap;     // [n_masks][words_per_mask]
+    int64_t *counts;      // counts[m * N + i] (row_ptr + 1)
+    SeedList seeds;
+};
+
+// Arguments of the CSR fill kernel.
+struct MaskFillArgs {
+    int64_t N;
+    int32_t n_masks;
+    int32_t col_bytes;
+    int64_t words_per_mask;
+    const uint32_t *bitmap;
+    const int64_t *row_ptr;
+    void *col;
+};
+
+// Arguments of the RoPE kernels: x_out[p][h][c], x_out[p][h][c + D/2] from x_in.
+struct RopeArgs {
+    const void *x_in;
+    void *x_out;
+    void *x_out_lo;  // bf16 output only: if set, x_out gets bf16(y) and x_out_lo bf16(y - bf16(y))
+    int64_t N;
+    int32_t H;
+    int32_t D;
+    double f[kMaxHeadDimHalf];  // rotation frequencies (fp64)
+    float mscale;
+};
+
+// Arguments of the attention kernels. One warp handles one task = (set s, row i, KV head g).
+struct AttnArgs {
+    const void *q;         // [N][Hq][D]: fp32 rotated queries (split path) or dtype as given
+    const void *k;         // [N][Hkv][D]
+    const void *k_lo;      // bf16 path: low part of the rotated keys (k~ = k + k_lo), or null
+    const void *v;         // [N][Hkv][D]
+    void *out;             // [n_sets][N][Hq][D]
+    float *lse;            // [n_sets][Hq][N] or null
+    const int64_t *row_ptr;  // [n_masks * N + 1] (null when dense)
+    const void *col;       // keys (null when dense)
+    int64_t N;
+    int32_t Hq;
+    int32_t Hkv;
+    int32_t G;             // Hq / Hkv
+    int32_t heads_keyed;   // masks keyed per KV head (1 or Hkv)
+    int32_t n_sets;        // output sets: n_seeds for per-seed masks, else 1
+    int32_t pad_;
+    float scale_log2;      // log2(e) / sqrt(D)
+    int64_t n_tasks;       // n_sets * N * Hkv
+};
+
+// Library-wide kernel launch counter (ris_launch_count).
+void note_launch(int n = 1);
+
+// Launchers: each returns the launch error (cudaGetLastError) of its kernels.
+cudaError_t launch_mask_bits(const MaskBitsArgs &a, cudaStream_t s);
+cudaError_t launch_scan_inplace(int64_t *x, int64_t n, int64_t *partials, cudaStream_t s);
+int64_t scan_partials_count(int64_t n);
+cudaError_t launch_mask_fill(const MaskFillArgs &a, cudaStream_t s);
+
+// dtype_in / dtype_out are ris_dtype values.
+cudaError_t launch_rope(const RopeArgs &a, int dtype_in, int dtype_out, cudaStream_t s);
+
+// q_split: q is fp32 and is split into bf16 hi + lo on the tensor-core path; a.k_lo set:
+// the keys arrive as a bf16 hi + lo pair.
+cudaError_t launch_attention_bf16(const AttnArgs &a, int D, int out_dtype, bool q_split, int col_bytes,
+                                  bool dense, cudaStream_t s);
+cudaError_t launch_attention_f32(const AttnArgs &a, int D, int out_dtype, int col_bytes, bool dense,
+                                 cudaStream_t s);
+
+}  // namespace ris

@@ -1,0 +1,204 @@
+"""GPU RoPE and sparse attention vs the fp64 oracle, through the C ABI.
+
+Tolerances (see helpers.py): bf16 inputs with fp32 accumulation must be within max-abs
+1e-2 and relative L2 5e-3 of the fp64 oracle; fp32 inputs within relative L2 1e-5.
+Small cases compare every output; the full workload sizes compare sampled rows, computed
+one by one by the oracle, in the same launch configuration the benchmark uses.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as ora
+from helpers import (check_bf16_path, check_f32_path, make_inputs, oracle_rope, rel_l2, sample_rows,
+                     to_np)
+from paper_2607_21927_gb300 import ris
+
+pytestmark = pytest.mark.gpu
+
+QWEN = dict(Hq=12, Hkv=2, D=128, theta=1e6, native=32768)
+TINY = dict(Hq=32, Hkv=4, D=64, theta=1e4, native=2048)
+
+
+def run_gpu(q, k, v, mode, d, seeds, rope_kind, theta, native, out_dtype=torch.float32, opts=None,
+            per_seed=False, return_lse=True):
+    rope = ris.rope_cfg(rope_kind, theta, native) if rope_kind else None
+    fn = ris.ris_ensemble_batch if per_seed else ris.ris_sparse_attention_fwd
+    out, lse = fn(q, k, v, mode, d, seeds, rope=rope, opts=opts, out_dtype=out_dtype, return_lse=True)
+    torch.cuda.synchronize()
+    return out, lse
+
+
+def run_oracle(qn, kn, vn, mode, d, seeds, rope_kind, theta, native, rows=None, seed_index=-1, W=1, A=0,
+               head_key=0):
+    N = qn.shape[0]
+    spec = ora.MaskSpec(N=N, mode=mode, density=d, seeds=seeds, seed_index=seed_index, local_window=W,
+                        n_anchor=A, head_key=head_key)
+    out, lse, _, _ = ora.sparse_attention(qn, kn, vn, spec, oracle_rope(rope_kind, theta, native), rows=rows)
+    return out, lse
+
+
+# ----------------------------------------------------------------------------- RoPE
+@pytest.mark.parametrize("kind,N,native", [(1, 300, 4096), (2, 1024, 256), (3, 4096, 1024), (3, 65536, 32768)])
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_rope_apply(kind, N, native, dtype):
+    H, D, theta = 3, 128, 1e6
+    (x, _, _), (xn, _, _) = make_inputs(N, H, 1, D, dtype=dtype, seed=kind)
+    ris.ris_rope_apply(x, ris.rope_cfg(kind, theta, native))
+    torch.cuda.synchronize()
+    ref = ora.rope(xn, np.arange(N, dtype=np.float64), ora.RopeCfg(kind=kind, theta=theta, native_len=native), N)
+    got = to_np(x)
+    if dtype == torch.float32:
+        # fp32 rotation of exactly reduced angles: a few ulps of the largest pair element
+        assert np.abs(got - ref).max() <= 4e-6 * max(1.0, np.abs(ref).max())
+    else:
+        # bf16 result: one bf16 ulp of the exact rotation, plus the fp32 rotation's own error
+        # (a few fp32 ulps of the pair's inputs) for outputs that cancel to almost zero
+        ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(ref), 1e-30))) - 7)
+        pair = np.concatenate([np.maximum(np.abs(xn[..., :D // 2]), np.abs(xn[..., D // 2:]))] * 2, -1)
+        assert np.all(np.abs(got - ref) <= ulp + 4e-7 * pair * 1.07)
+
+
+# ----------------------------------------------------------------------------- small, full outputs
+SMALL = [
+    # N, Hq, Hkv, D, dtype, mode, d, S, rope kind, native
+    (1, 1, 1, 128, torch.float32, 0, 0.05, 1, 1, 4096),
+    (33, 4, 2, 64, torch.bfloat16, 0, 0.3, 2, 0, 4096),
+    (200, 6, 2, 128, torch.bfloat16, 1, 0.05, 3, 2, 64),
+    (517, 8, 1, 64, torch.bfloat16, 0, 0.05, 5, 3, 128),
+    (640, 3, 3, 128, torch.float32, 1, 0.1, 2, 3, 128),
+    (300, 12, 2, 128, torch.bfloat16, 2, 1.0, 1, 1, 4096),
+    (300, 2, 1, 64, torch.float32, 0, 1.0, 1, 0, 4096),
+    (1025, 5, 1, 128, torch.bfloat16, 0, 0.02, 10, 1, 4096),
+]
+
+
+@pytest.mark.parametrize("N,Hq,Hkv,D,dtype,mode,d,S,kind,native", SMALL)
+def test_attention_small_full(N, Hq, Hkv, D, dtype, mode, d, S, kind, native):
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, dtype=dtype, seed=N + S, outliers=(dtype == torch.bfloat16))
+    seeds = list(range(S))
+    out, lse = run_gpu(q, k, v, mode, d, seeds, kind, 1e4, native)
+    ref, ref_lse = run_oracle(qn, kn, vn, mode, d, seeds, kind, 1e4, native)
+    if dtype == torch.float32:
+        check_f32_path(to_np(out), ref)
+        np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=1e-5, atol=1e-5)
+    else:
+        check_bf16_path(to_np(out), ref)
+        np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-2)
+
+
+def test_attention_bf16_output_and_forced_set():
+    N, Hq, Hkv, D = 700, 6, 2, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=7, outliers=True)
+    opts = ris.mask_opts(local_window=16, n_anchor=4)
+    out = ris.ris_sparse_attention_fwd(q, k, v, 0, 0.02, [1, 2], rope=ris.rope_cfg(1, 1e6, 32768), opts=opts)
+    torch.cuda.synchronize()
+    assert out.dtype == torch.bfloat16
+    ref, _ = run_oracle(qn, kn, vn, 0, 0.02, [1, 2], 1, 1e6, 32768, W=16, A=4)
+    check_bf16_path(to_np(out), ref, out_bf16=True)
+
+
+def test_attention_per_head_masks():
+    N, Hq, Hkv, D = 400, 8, 2, 64
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=11)
+    opts = ris.mask_opts(per_head=True)
+    out = ris.ris_sparse_attention_fwd(q, k, v, 0, 0.1, [4], opts=opts, out_dtype=torch.float32)
+    torch.cuda.synchronize()
+    got = to_np(out)
+    G = Hq // Hkv
+    for g in range(Hkv):
+        ref, _ = run_oracle(qn[:, g * G:(g + 1) * G], kn[:, g:g + 1], vn[:, g:g + 1], 0, 0.1, [4], 0, 1e4, 4096,
+                            head_key=g)
+        check_bf16_path(got[:, g * G:(g + 1) * G], ref)
+
+
+def test_ensemble_batch_small_full():
+    N, Hq, Hkv, D, seeds = 600, 6, 2, 128, [3, 4, 5, 6]
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=5, outliers=True)
+    out, lse = run_gpu(q, k, v, 0, 0.05, seeds, 1, 1e6, 32768, per_seed=True)
+    assert out.shape == (4, N, Hq, D)
+    for s in range(len(seeds)):
+        ref, ref_lse = run_oracle(qn, kn, vn, 0, 0.05, seeds, 1, 1e6, 32768, seed_index=s)
+        check_bf16_path(to_np(out[s]), ref)
+        np.testing.assert_allclose(to_np(lse[s]).T, ref_lse, rtol=0, atol=2e-2)
+
+
+def test_attention_masked_reuses_mask_across_layers():
+    N, Hq, Hkv, D = 512, 12, 2, 128
+    m = ris.ris_mask_generate(N, Hkv, 1, 0.05, [1, 2, 3])
+    rope = ris.rope_cfg(3, 1e6, 256)
+    for layer in range(3):
+        (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=100 + layer, outliers=True)
+        out = ris.ris_attention_masked(m, q, k, v, rope=rope, out_dtype=torch.float32)
+        torch.cuda.synchronize()
+        ref, _ = run_oracle(qn, kn, vn, 1, 0.05, [1, 2, 3], 3, 1e6, 256)
+        check_bf16_path(to_np(out), ref)
+    m.free()
+
+
+def test_v_constant_gives_one():
+    N, Hq, Hkv, D = 1000, 6, 2, 128
+    (q, k, _), _ = make_inputs(N, Hq, Hkv, D, seed=2, outliers=True)
+    v = torch.ones(N, Hkv, D, dtype=torch.bfloat16, device="cuda")
+    out = ris.ris_sparse_attention_fwd(q, k, v, 0, 0.05, [0, 1], out_dtype=torch.float32)
+    torch.cuda.synchronize()
+    assert torch.all((out - 1).abs() < 1e-5)
+
+
+# ----------------------------------------------------------------------------- workload configurations
+def _config_case(N, shape, dtype, mode, d, S, kind, outliers, nrows, seed=0, per_seed=False):
+    (q, k, v), (qn, kn, vn) = make_inputs(N, shape["Hq"], shape["Hkv"], shape["D"], dtype=dtype, seed=seed,
+                                          outliers=outliers)
+    seeds = list(range(S))
+    out, lse = run_gpu(q, k, v, mode, d, seeds, kind, shape["theta"], shape["native"], per_seed=per_seed)
+    rows = np.arange(N) if nrows is None else sample_rows(N, nrows, seed=N + S)
+    got = to_np(out[rows] if not per_seed else out[:, rows])
+    return got, (qn, kn, vn), seeds, rows, to_np(lse)
+
+
+def test_c1_single_head_fp32_full():
+    """N=2048, 1 head, D=128, fp32, theta 1e6, Stochastic 5%, 1 seed; every output."""
+    shape = dict(Hq=1, Hkv=1, D=128, theta=1e6, native=32768)
+    got, (qn, kn, vn), seeds, rows, lse = _config_case(2048, shape, torch.float32, 0, 0.05, 1, 1, False, None)
+    ref, ref_lse = run_oracle(qn, kn, vn, 0, 0.05, seeds, 1, 1e6, 32768)
+    check_f32_path(got, ref)
+    np.testing.assert_allclose(lse.T, ref_lse, rtol=1e-6, atol=1e-6)
+
+
+def test_c2_qwen_8k_full():
+    """Qwen2 shape, N=8192, bf16 with outlier channels, Stochastic 1% x 10 seeds; every output."""
+    got, (qn, kn, vn), seeds, rows, _ = _config_case(8192, QWEN, torch.bfloat16, 0, 0.01, 10, 1, True, None)
+    ref, _ = run_oracle(qn, kn, vn, 0, 0.01, seeds, 1, 1e6, 32768)
+    check_bf16_path(got, ref)
+
+
+def test_c3_tinyllama_16k_yarn_structural():
+    """TinyLlama shape, N=16384 (YaRN s=8 beyond the 2048 window), Structural 1% x 10; sampled rows."""
+    got, (qn, kn, vn), seeds, rows, _ = _config_case(16384, TINY, torch.bfloat16, 1, 0.01, 10, 3, False, 384)
+    ref, _ = run_oracle(qn, kn, vn, 1, 0.01, seeds, 3, 1e4, 2048, rows=rows)
+    check_bf16_path(got, ref)
+
+
+@pytest.mark.parametrize("mode,d,S", [(0, 0.01, 70), (0, 0.05, 10), (2, 1.0, 1)], ids=["1pct_x70", "5pct_x10", "dense"])
+def test_c4_qwen_32k(mode, d, S):
+    """Qwen2 shape, N=32768, bf16 with outliers: Stochastic 1% x 70, 5% x 10 and dense causal; sampled rows."""
+    got, (qn, kn, vn), seeds, rows, _ = _config_case(32768, QWEN, torch.bfloat16, mode, d, S, 1, True, 96)
+    ref, _ = run_oracle(qn, kn, vn, mode, d, seeds, 1, 1e6, 32768, rows=rows)
+    check_bf16_path(got, ref)
+
+
+@pytest.mark.parametrize("mode", [0, 1], ids=["stochastic", "structural"])
+def test_c5_qwen_64k_layer(mode):
+    """One layer of the N=65536 stack (YaRN s=2), 1% x 10 seeds; sampled rows."""
+    got, (qn, kn, vn), seeds, rows, _ = _config_case(65536, QWEN, torch.bfloat16, mode, 0.01, 10, 3, True, 96,
+                                                     seed=3)
+    ref, _ = run_oracle(qn, kn, vn, mode, 0.01, seeds, 3, 1e6, 32768, rows=rows)
+    check_bf16_path(got, ref)
+
+
+def test_c2_ensemble_per_seed_sampled():
+    got, (qn, kn, vn), seeds, rows, _ = _config_case(8192, QWEN, torch.bfloat16, 0, 0.01, 10, 1, True, 64,
+                                                     per_seed=True)
+    for s in (0, 9):
+        ref, _ = run_oracle(qn, kn, vn, 0, 0.01, seeds, 1, 1e6, 32768, rows=rows, seed_index=s)
+        check_bf16_path(got[s], ref)

@@ -1,0 +1,108 @@
+"""GPU mask sampler vs the fp64 oracle: bitmap and CSR bit-exact (integer work)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as ora
+from helpers import row_word_offset, sample_rows
+from paper_2607_21927_gb300 import ris
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_mask(N, mode, d, seeds, kv_heads=1, per_seed=False, W=1, A=0, per_head=False, layer_key=0):
+    opts = ris.mask_opts(local_window=W, n_anchor=A, per_head=per_head, layer_key=layer_key)
+    return ris.ris_mask_generate(N, kv_heads, mode, d, seeds, opts=opts, per_seed=per_seed)
+
+
+def oracle_spec(N, mode, d, seeds, seed_index=-1, W=1, A=0, head_key=0, layer_key=0):
+    return ora.MaskSpec(N=N, mode=mode, density=d, seeds=seeds, seed_index=seed_index, local_window=W,
+                        n_anchor=A, head_key=head_key, layer_key=layer_key)
+
+
+def check_rows(m, specs, rows, check_bits=True):
+    """specs[mask_id] is the oracle spec of that mask; compare the given rows."""
+    d = m.info()
+    N = d.N
+    row_ptr = m.row_ptr().cpu().numpy()
+    cols = m.cols().cpu().numpy()
+    bitmap = m.bitmap().cpu().numpy().view(np.uint32) if check_bits else None
+    assert row_ptr[0] == 0 and np.all(np.diff(row_ptr) >= 1)
+    assert row_ptr[-1] == d.n_pairs == cols.shape[0]
+    for mid, spec in enumerate(specs):
+        off, ref = ora.mask_cols(spec, rows)
+        for r, i in enumerate(rows):
+            a, b = row_ptr[mid * N + i], row_ptr[mid * N + i + 1]
+            np.testing.assert_array_equal(cols[a:b], ref[off[r]:off[r + 1]], err_msg=f"mask {mid} row {i}")
+        if check_bits:
+            words = ora.mask_bits(spec, rows)
+            for r, i in enumerate(rows):
+                nw = (i >> 5) + 1
+                start = mid * d.words_per_mask + row_word_offset(int(i))
+                np.testing.assert_array_equal(bitmap[start:start + nw], words[r, :nw],
+                                              err_msg=f"bitmap mask {mid} row {i}")
+
+
+@pytest.mark.parametrize("N,mode,d,S,W,A", [
+    (1, 0, 0.05, 1, 1, 0), (33, 0, 0.3, 2, 1, 0), (100, 1, 0.05, 3, 1, 0), (257, 0, 0.01, 70, 1, 0),
+    (300, 1, 0.2, 1, 4, 3), (513, 0, 1.0, 1, 1, 0), (700, 2, 0.01, 2, 1, 0), (1000, 1, 0.013, 10, 1, 0),
+    (2048, 0, 0.05, 1, 1, 0)])
+def test_mask_full_small(N, mode, d, S, W, A):
+    seeds = list(range(100, 100 + S))
+    m = gpu_mask(N, mode, d, seeds, W=W, A=A)
+    if m.info().dense:
+        assert m.info().n_pairs == N * (N + 1) // 2
+        return
+    check_rows(m, [oracle_spec(N, mode, d, seeds, W=W, A=A)], np.arange(N))
+
+
+def test_mask_per_seed_and_per_head():
+    N, seeds, Hkv = 400, [5, 6, 7], 2
+    m = gpu_mask(N, 0, 0.05, seeds, kv_heads=Hkv, per_seed=True, per_head=True, layer_key=9)
+    d = m.info()
+    assert d.n_masks == 6 and d.heads_keyed == 2
+    specs = [oracle_spec(N, 0, 0.05, seeds, seed_index=s, head_key=h, layer_key=9)
+             for s in range(3) for h in range(Hkv)]
+    check_rows(m, specs, np.arange(N))
+    m2 = gpu_mask(N, 1, 0.05, seeds, per_seed=True)
+    check_rows(m2, [oracle_spec(N, 1, 0.05, seeds, seed_index=s) for s in range(3)], np.arange(N))
+
+
+# The five workload shapes: N, mode, density, seeds.
+CONFIG_MASKS = [
+    ("C1", 2048, 0, 0.05, 1), ("C2", 8192, 0, 0.01, 10), ("C3", 16384, 1, 0.01, 10),
+    ("C4a", 32768, 0, 0.01, 70), ("C4b", 32768, 0, 0.05, 10), ("C5s", 65536, 0, 0.01, 10),
+    ("C5t", 65536, 1, 0.01, 10),
+]
+
+
+@pytest.mark.parametrize("name,N,mode,d,S", CONFIG_MASKS, ids=[c[0] for c in CONFIG_MASKS])
+def test_mask_config_sizes_sampled_rows(name, N, mode, d, S):
+    seeds = list(range(S))
+    m = gpu_mask(N, mode, d, seeds)
+    rows = sample_rows(N, 48, seed=N)
+    check_rows(m, [oracle_spec(N, mode, d, seeds)], rows)
+    # pair count matches its expectation within binomial bounds (property at any size)
+    info = m.info()
+    if mode == 0:
+        U = 1 - (1 - d) ** S
+        T = N * (N - 1) / 2
+        assert abs(info.n_pairs - N - U * T) < 6 * np.sqrt(T * U * (1 - U))
+    m.free()
+    torch.cuda.synchronize()
+
+
+def test_mask_u32_columns_beyond_65536():
+    """N > 65536 switches the key lists to 32-bit indices."""
+    N = 65600
+    m = gpu_mask(N, 0, 0.0005, [1])
+    assert m.info().col_bytes == 4
+    check_rows(m, [oracle_spec(N, 0, 0.0005, [1])], sample_rows(N, 8, seed=3), check_bits=False)
+
+
+def test_mask_deterministic_and_keyed():
+    a = gpu_mask(500, 0, 0.1, [3]).cols().cpu()
+    b = gpu_mask(500, 0, 0.1, [3]).cols().cpu()
+    assert torch.equal(a, b)
+    c = gpu_mask(500, 0, 0.1, [3], layer_key=1).cols().cpu()
+    assert a.shape != c.shape or not torch.equal(a, c)
