@@ -188,6 +188,15 @@ ris_status ris_ensemble_batch(const void *q, const void *k, const void *v, void 
                               int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
                               const ris_mask_opts *opts, float *lse, void *stream);
 
+/* Kernel timer for measurement (off by default). While enabled, every attention kernel launch
+ * (the fused QK^T -> softmax -> PV kernel, not RoPE or mask kernels) is bracketed by CUDA
+ * events recorded on the stream it is launched on. Enabling or disabling clears the record.
+ * ris_kernel_timer_read blocks until the last recorded launch has finished, returns the summed
+ * device milliseconds and the number of launches recorded since the last read, and clears
+ * them. Intended for one thread at a time. Errors: RIS_ERR_INVALID (NULL outputs), RIS_ERR_CUDA. */
+ris_status ris_kernel_timer_enable(int32_t enable);
+ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches);
+
 /* Text of the calling thread's last error ("" if none). The string is owned by the library. */
 const char *ris_last_error(void);
 

@@ -12,6 +12,8 @@
 #include <mutex>
 #include <new>
 #include <string>
+#include <utility>
+#include <vector>
 
 #include "ris_internal.h"
 
@@ -107,6 +109,36 @@ struct Scratch {
         if (p) cudaFreeAsync(p, s);
     }
 };
+
+// Opt-in attention-kernel timer (ris_kernel_timer_*): event pairs recorded around launches.
+struct KernelTimer {
+    std::mutex mu;
+    bool on = false;
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> used, spare;
+};
+KernelTimer g_timer;
+
+void timer_clear_locked()
+{
+    for (auto &e : g_timer.used) g_timer.spare.push_back(e);
+    g_timer.used.clear();
+}
+
+// Returns the event pair to record around one launch, or {nullptr, nullptr} when off.
+std::pair<cudaEvent_t, cudaEvent_t> timer_pair()
+{
+    std::lock_guard<std::mutex> lk(g_timer.mu);
+    if (!g_timer.on) return {nullptr, nullptr};
+    std::pair<cudaEvent_t, cudaEvent_t> e{nullptr, nullptr};
+    if (!g_timer.spare.empty()) {
+        e = g_timer.spare.back();
+        g_timer.spare.pop_back();
+    } else if (cudaEventCreate(&e.first) != cudaSuccess || cudaEventCreate(&e.second) != cudaSuccess) {
+        return {nullptr, nullptr};
+    }
+    g_timer.used.push_back(e);
+    return e;
+}
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -507,10 +539,13 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.n_sets = m->per_seed ? m->n_seeds : 1;
     a.scale_log2 = (float)(1.4426950408889634074 / std::sqrt((double)head_dim));
     a.n_tasks = (int64_t)a.n_sets * N * kv_heads;
+    const auto ev = timer_pair();
+    if (ev.first) RIS_CUDA(cudaEventRecord(ev.first, s));
     if (dtype == RIS_BF16)
         RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
     else
         RIS_CUDA(launch_attention_f32(a, head_dim, out_dtype, m->col_bytes, m->dense != 0, s));
+    if (ev.second) RIS_CUDA(cudaEventRecord(ev.second, s));
     return RIS_OK;
 }
 
@@ -538,6 +573,31 @@ ris_status fwd_common(const void *q, const void *k, const void *v, void *out, in
 }
 
 }  // namespace
+
+ris_status ris_kernel_timer_enable(int32_t enable)
+{
+    std::lock_guard<std::mutex> lk(g_timer.mu);
+    timer_clear_locked();
+    g_timer.on = enable != 0;
+    return RIS_OK;
+}
+
+ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches)
+{
+    if (total_ms == nullptr || launches == nullptr) return fail(RIS_ERR_INVALID, "output pointer is NULL");
+    std::lock_guard<std::mutex> lk(g_timer.mu);
+    double tot = 0.0;
+    for (auto &e : g_timer.used) {
+        RIS_CUDA(cudaEventSynchronize(e.second));
+        float ms = 0.f;
+        RIS_CUDA(cudaEventElapsedTime(&ms, e.first, e.second));
+        tot += ms;
+    }
+    *total_ms = tot;
+    *launches = (int64_t)g_timer.used.size();
+    timer_clear_locked();
+    return RIS_OK;
+}
 
 ris_status ris_attention_masked(ris_mask_t mask, const void *q, const void *k, const void *v, void *out,
                                 int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t dtype,

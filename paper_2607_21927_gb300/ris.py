@@ -82,6 +82,8 @@ _SIGS = {
     "ris_attention_masked": [ctypes.c_void_p] * 5 + [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                              ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p],
     "ris_ensemble_batch": None,  # same as ris_sparse_attention_fwd
+    "ris_kernel_timer_enable": [ctypes.c_int32],
+    "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
 }
 
 
@@ -115,6 +117,17 @@ def ris_launch_count() -> int:
 
 def ris_version() -> str:
     return lib().ris_version().decode()
+
+
+def ris_kernel_timer_enable(enable: bool = True) -> None:
+    _check("ris_kernel_timer_enable", lib().ris_kernel_timer_enable(int(bool(enable))))
+
+
+def ris_kernel_timer_read():
+    """(summed device ms, launches) of the attention kernels recorded since the last read."""
+    ms, n = ctypes.c_double(), ctypes.c_int64()
+    _check("ris_kernel_timer_read", lib().ris_kernel_timer_read(ctypes.byref(ms), ctypes.byref(n)))
+    return ms.value, n.value
 
 
 def _check(name: str, st: int) -> None:
