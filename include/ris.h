@@ -188,6 +188,27 @@ ris_status ris_ensemble_batch(const void *q, const void *k, const void *v, void 
                               int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
                               const ris_mask_opts *opts, float *lse, void *stream);
 
+/* Allocation-free variant of ris_attention_masked (same arguments, results and errors).
+ * The paper has no counterpart: this entry point exists for callers that may not allocate
+ * device memory while a layer runs, such as an inference engine's enqueue callback that may
+ * only launch work, or a server that plans all device memory at load time. They build the
+ * mask once beforehand (ris_mask_generate allocates) and call this per layer.
+ * Instead of the stream-ordered pool, the rotated q (fp32) and k (bf16 hi + lo, or fp32)
+ * live in one library-owned device array of 64 MiB per device, which every GPU that uses
+ * this entry point holds until the process exits. The call needs
+ *   align256(N*heads*head_dim*4) + (bf16 ? 2 : 1) * align256(N*kv_heads*head_dim*(bf16 ? 2 : 4))
+ * bytes when rope is set (none without rope) and returns RIS_ERR_INVALID, launching nothing,
+ * when that exceeds 64 MiB (about N = 9300 tokens at 12 / 2 heads of 128). It calls no
+ * allocation routine. The first call on a device looks up the array's device address (and
+ * may load the library's device code): make that first call before any stream capture.
+ * Every call on a device shares the array and leaves its contents behind; each call writes
+ * all scratch it reads, so nothing needs clearing, but calls whose GPU work overlaps (e.g.
+ * on two streams) race on it and must be ordered by the caller. */
+ris_status ris_attention_masked_noalloc(ris_mask_t mask, const void *q, const void *k, const void *v,
+                                        void *out, int32_t heads, int32_t kv_heads, int32_t head_dim,
+                                        int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
+                                        float *lse, void *stream);
+
 /* Kernel timer for measurement (off by default). While enabled, every attention kernel launch
  * (the fused QK^T -> softmax -> PV kernel, not RoPE or mask kernels) is bracketed by CUDA
  * events recorded on the stream it is launched on. Enabling or disabling clears the record.

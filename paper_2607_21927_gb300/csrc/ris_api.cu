@@ -253,6 +253,10 @@ ris_status validate_attention(const void *q, const void *k, const void *v, void 
 
 }  // namespace
 
+namespace ris {
+void set_error_text(const char *msg) { t_err = msg; }
+}  // namespace ris
+
 extern "C" {
 
 const char *ris_last_error(void) { return t_err.c_str(); }

@@ -84,6 +84,9 @@ struct AttnArgs {
 // Library-wide kernel launch counter (ris_launch_count).
 void note_launch(int n = 1);
 
+// Set the calling thread's error text (returned by ris_last_error).
+void set_error_text(const char *msg);
+
 // Launchers: each returns the launch error (cudaGetLastError) of its kernels.
 cudaError_t launch_mask_bits(const MaskBitsArgs &a, cudaStream_t s);
 cudaError_t launch_scan_inplace(int64_t *x, int64_t n, int64_t *partials, cudaStream_t s);

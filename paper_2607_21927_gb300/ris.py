@@ -82,6 +82,9 @@ _SIGS = {
     "ris_attention_masked": [ctypes.c_void_p] * 5 + [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                              ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p],
     "ris_ensemble_batch": None,  # same as ris_sparse_attention_fwd
+    "ris_attention_masked_noalloc": [ctypes.c_void_p] * 5 + [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                     ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p,
+                                     ctypes.c_void_p],
     "ris_kernel_timer_enable": [ctypes.c_int32],
     "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
 }
@@ -321,3 +324,18 @@ def ris_attention_masked(mask: Mask, q, k, v, rope: Optional[RopeCfg] = None,
         mask.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(out), Hq, Hkv, D, _dtype(q), _dtype(out), _ref(rope),
         _ptr(lse), _stream(stream)))
     return (out, lse) if return_lse else out
+
+
+def ris_attention_masked_noalloc(mask: Mask, q, k, v, out: torch.Tensor, rope: Optional[RopeCfg] = None,
+                                 lse: Optional[torch.Tensor] = None, stream=None):
+    """Allocation-free layer call: the caller passes every output buffer; the library's
+    scratch is a fixed 64 MiB device array (see include/ris.h)."""
+    N, Hq, Hkv, D = _shapes(q, k, v)
+    d = mask.info()
+    if d.N != N:
+        raise ValueError(f"q has {N} tokens, the mask was built for {d.N}")
+    assert out.is_cuda and out.is_contiguous()
+    _check("ris_attention_masked_noalloc", lib().ris_attention_masked_noalloc(
+        mask.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(out), Hq, Hkv, D, _dtype(q), _dtype(out), _ref(rope),
+        _ptr(lse), _stream(stream)))
+    return out
