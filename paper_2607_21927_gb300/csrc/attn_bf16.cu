@@ -10,12 +10,19 @@
 //   online softmax per head in fp32 (exp2 domain, scale log2(e)/sqrt(D) applied in fp32)
 //   O^T[D x 8 heads]     += V^T[D x 16 keys] . P^T           (mma m16n8k16, head dim in M)
 //
-// Gathered rows go straight from L2 into registers, with no shared-memory staging: the head
+// Gathered rows go straight from L2 into registers, with no shared-memory staging. The head
 // dimension is permuted (the same permutation on K~ and Q~, undone when O is stored) so
-// that each lane's share of a K row is one contiguous D/2-byte run and its share of a V row
-// one contiguous D/8-element run, i.e. whole 32-byte sectors with 16-byte loads. P^T moves
-// from the accumulator layout of the first product into the operand layout of the second
-// with movmatrix (an 8x8 transpose in registers).
+// that every 16-byte-per-lane load instruction reads whole, fully used 32-byte sectors in
+// long runs: for K the four lanes that share a key row read 64 contiguous bytes of it, for
+// V the eight lanes that share a row read 128 contiguous bytes. Scattered gathers are
+// bounded by the L1 data pipe's wavefronts per instruction, not by L2 bandwidth, so the
+// fewer sectors and lines an instruction touches the better. P^T moves from the
+// accumulator layout of the first product into the operand layout of the second with
+// movmatrix (an 8x8 transpose in registers).
+//
+// Lane (p = lane/4, q = lane%4). K row: lane q holds elements 32u + 8q + [0, 8), u < D/32;
+// k-step t takes elements 32(t/2) + 8q + 4(t%2) + [0, 4). V row: lane p holds elements
+// 64u + 8p + [0, 8), u < D/64; word j of that run (d, d+1) feeds m-tile j.
 //
 // Precision. With activation outlier channels (|v| up to ~30) a max-abs error of 1e-2 needs
 // ~12+ significant bits in the scores and in P, more than bf16 (8) or fp16 (11) carry. So:
@@ -86,14 +93,17 @@ __device__ __forceinline__ void store_run<__nv_bfloat16>(__nv_bfloat16 *dst, con
 
 // D: head dim (64 or 128). QSPLIT: q is fp32 (split hi + lo); else q is bf16.
 // KSPLIT: keys come as a bf16 hi (a.k) + lo (a.k_lo) pair.
+#ifndef RIS_ATTN_MIN_BLOCKS
+#define RIS_ATTN_MIN_BLOCKS 1
+#endif
+
 template <int D, bool QSPLIT, bool KSPLIT, typename TIdx, bool DENSE, typename TOut>
-__global__ void __launch_bounds__(kAttnWarps * 32) k_attn_bf16(const AttnArgs a)
+__global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
 {
     constexpr int KSTEPS = D / 16;  // k-steps of the score product
     constexpr int KU = D / 32;      // 16-byte loads per K row per lane (D/2 bytes)
     constexpr int VU = D / 64;      // 16-byte loads per V row per lane (D/8 elements)
     constexpr int MT = D / 16;      // m-tiles of the value product (head dim)
-    constexpr int VRUN = D / 8;     // output elements per lane per head
 
     const int lane = threadIdx.x & 31;
     const int64_t tid = (int64_t)blockIdx.x * kAttnWarps + (threadIdx.x >> 5);
@@ -111,7 +121,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_bf16(const AttnArgs a)
         const int64_t qrow = (t.i * a.Hq + (int64_t)t.g * a.G + (hv ? p : 0)) * D;
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
-            const int d0 = (D / 4) * q + 4 * ks;
+            const int d0 = 32 * (ks >> 1) + 8 * q + 4 * (ks & 1);
             if (QSPLIT) {
                 float4 x = hv ? *reinterpret_cast<const float4 *>(reinterpret_cast<const float *>(a.q) + qrow + d0)
                               : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -134,13 +144,10 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_bf16(const AttnArgs a)
     }
 
     const size_t row_bytes = (size_t)a.Hkv * D * sizeof(__nv_bfloat16);
-    const char *kb = reinterpret_cast<const char *>(a.k) + (size_t)t.g * D * sizeof(__nv_bfloat16) +
-                     (size_t)q * (D / 2);
-    const char *kbl = KSPLIT ? reinterpret_cast<const char *>(a.k_lo) + (size_t)t.g * D * sizeof(__nv_bfloat16) +
-                                   (size_t)q * (D / 2)
+    const char *kb = reinterpret_cast<const char *>(a.k) + (size_t)t.g * D * sizeof(__nv_bfloat16) + 16 * q;
+    const char *kbl = KSPLIT ? reinterpret_cast<const char *>(a.k_lo) + (size_t)t.g * D * sizeof(__nv_bfloat16) + 16 * q
                              : nullptr;
-    const char *vb = reinterpret_cast<const char *>(a.v) + (size_t)t.g * D * sizeof(__nv_bfloat16) +
-                     (size_t)p * (D / 8) * sizeof(__nv_bfloat16);
+    const char *vb = reinterpret_cast<const char *>(a.v) + (size_t)t.g * D * sizeof(__nv_bfloat16) + 16 * p;
 
     float o[MT][4];
 #pragma unroll
@@ -148,39 +155,69 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_bf16(const AttnArgs a)
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
     const float sc = a.scale_log2;
 
-    for (int64_t base = 0; base < n; base += 16) {
-        // ---- key indices of this group of 16 (invalid slots read the row itself)
-        int idx = (int)t.i;
-        if (lane < 16 && base + lane < n) idx = key_at<DENSE, TIdx>(cols, base + lane);
-        const int ik0 = __shfl_sync(0xFFFFFFFFu, idx, p);
-        const int ik1 = __shfl_sync(0xFFFFFFFFu, idx, p + 8);
-        const int iv0 = __shfl_sync(0xFFFFFFFFu, idx, 2 * q);
-        const int iv1 = __shfl_sync(0xFFFFFFFFu, idx, 2 * q + 1);
-        const int iv2 = __shfl_sync(0xFFFFFFFFu, idx, 2 * q + 8);
-        const int iv3 = __shfl_sync(0xFFFFFFFFu, idx, 2 * q + 9);
-        const bool val0 = base + p < n, val1 = base + p + 8 < n;
+    // ---- key indices, prefetched 64 keys (4 groups) ahead: lane holds positions
+    //      64c + lane and 64c + 32 + lane of chunk c; slots past the row read the row itself
+    int cur[2], nxt[2];
+    auto load_chunk = [&](int64_t cbase, int (&dst)[2]) {
+#pragma unroll
+        for (int w = 0; w < 2; ++w) {
+            const int64_t pos = cbase + 32 * w + lane;
+            dst[w] = pos < n ? key_at<DENSE, TIdx>(cols, pos) : (int)t.i;
+        }
+    };
+    load_chunk(0, cur);
+    load_chunk(64, nxt);
+    // index of slot r (0..15) of group slot gs (0..3) of a chunk held in (c0, c1)
+    auto slot = [&](int c0, int c1, int gs, int r) -> int {
+        return __shfl_sync(0xFFFFFFFFu, (gs >> 1) ? c1 : c0, (16 * gs + r) & 31);
+    };
 
-        // ---- gather: K rows p and p+8 (D/2 bytes each), V rows 2q, 2q+1, 2q+8, 2q+9 (D/8 elems)
-        uint4 k0[KU], k1[KU], kl0[KSPLIT ? KU : 1], kl1[KSPLIT ? KU : 1], v0[VU], v1[VU], v2[VU], v3[VU];
+    // ---- gathered rows of one group: K rows p and p+8 (D/2 bytes each of hi and lo),
+    //      V rows 2q, 2q+1, 2q+8, 2q+9 (D/8 elements each)
+    uint4 k0[KU], k1[KU], kl0[KSPLIT ? KU : 1], kl1[KSPLIT ? KU : 1], v0[VU], v1[VU], v2[VU], v3[VU];
+    auto issue_k = [&](int c0, int c1, int gs) {
+        const int ik0 = slot(c0, c1, gs, p), ik1 = slot(c0, c1, gs, p + 8);
 #pragma unroll
         for (int u = 0; u < KU; ++u) {
-            k0[u] = ldg16(kb + (size_t)ik0 * row_bytes + 16 * u);
-            k1[u] = ldg16(kb + (size_t)ik1 * row_bytes + 16 * u);
+            k0[u] = ldg16(kb + (size_t)ik0 * row_bytes + 64 * u);
+            k1[u] = ldg16(kb + (size_t)ik1 * row_bytes + 64 * u);
             if (KSPLIT) {
-                kl0[u] = ldg16(kbl + (size_t)ik0 * row_bytes + 16 * u);
-                kl1[u] = ldg16(kbl + (size_t)ik1 * row_bytes + 16 * u);
+                kl0[u % (KSPLIT ? KU : 1)] = ldg16(kbl + (size_t)ik0 * row_bytes + 64 * u);
+                kl1[u % (KSPLIT ? KU : 1)] = ldg16(kbl + (size_t)ik1 * row_bytes + 64 * u);
             }
         }
+    };
+    auto issue_v = [&](int c0, int c1, int gs) {
+        const int iv0 = slot(c0, c1, gs, 2 * q), iv1 = slot(c0, c1, gs, 2 * q + 1);
+        const int iv2 = slot(c0, c1, gs, 2 * q + 8), iv3 = slot(c0, c1, gs, 2 * q + 9);
 #pragma unroll
         for (int u = 0; u < VU; ++u) {
-            v0[u] = ldg16(vb + (size_t)iv0 * row_bytes + 16 * u);
-            v1[u] = ldg16(vb + (size_t)iv1 * row_bytes + 16 * u);
-            v2[u] = ldg16(vb + (size_t)iv2 * row_bytes + 16 * u);
-            v3[u] = ldg16(vb + (size_t)iv3 * row_bytes + 16 * u);
+            v0[u] = ldg16(vb + (size_t)iv0 * row_bytes + 128 * u);
+            v1[u] = ldg16(vb + (size_t)iv1 * row_bytes + 128 * u);
+            v2[u] = ldg16(vb + (size_t)iv2 * row_bytes + 128 * u);
+            v3[u] = ldg16(vb + (size_t)iv3 * row_bytes + 128 * u);
         }
+    };
 
-        // ---- S^T = K~ Q~^T
-        float s[4] = {0.f, 0.f, 0.f, 0.f};
+    // Phase-shifted pipeline: the next group's K rows are requested as soon as this group's
+    // scores are formed, its V rows as soon as this group's values are accumulated.
+    issue_k(cur[0], cur[1], 0);
+    issue_v(cur[0], cur[1], 0);
+    const int64_t ngroups = (n + 15) / 16;
+    for (int64_t g = 0; g < ngroups; ++g) {
+        const int64_t base = 16 * g;
+        const int gs = (int)(g & 3), gs1 = (gs + 1) & 3;
+        const bool more = g + 1 < ngroups;
+        const int n0 = gs1 == 0 ? nxt[0] : cur[0], n1 = gs1 == 0 ? nxt[1] : cur[1];
+        const bool val0 = base + p < n, val1 = base + p + 8 < n;
+
+        // ---- S^T = K~ Q~^T: independent accumulator chains (hi*hi, hi*lo, lo*hi, and even/odd
+        //      k-steps) so the tensor-core latencies overlap instead of forming one serial chain
+        float sa[2][4], sb[2][4], sl[2][4];
+#pragma unroll
+        for (int c = 0; c < 2; ++c)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) sa[c][e] = sb[c][e] = sl[c][e] = 0.f;
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
             const uint4 &x0 = k0[ks >> 1], &x1 = k1[ks >> 1];
@@ -188,14 +225,18 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_bf16(const AttnArgs a)
             const uint32_t a1 = (ks & 1) ? x1.z : x1.x;
             const uint32_t a2 = (ks & 1) ? x0.w : x0.y;
             const uint32_t a3 = (ks & 1) ? x1.w : x1.y;
-            mma16816(s, a0, a1, a2, a3, qh[ks][0], qh[ks][1]);
-            if (QSPLIT) mma16816(s, a0, a1, a2, a3, ql[ks][0], ql[ks][1]);
+            mma16816(sa[ks & 1], a0, a1, a2, a3, qh[ks][0], qh[ks][1]);
+            if (QSPLIT) mma16816(sb[ks & 1], a0, a1, a2, a3, ql[ks][0], ql[ks][1]);
             if (KSPLIT) {
                 const uint4 &y0 = kl0[(ks >> 1) % (KSPLIT ? KU : 1)], &y1 = kl1[(ks >> 1) % (KSPLIT ? KU : 1)];
-                mma16816(s, (ks & 1) ? y0.z : y0.x, (ks & 1) ? y1.z : y1.x, (ks & 1) ? y0.w : y0.y,
+                mma16816(sl[ks & 1], (ks & 1) ? y0.z : y0.x, (ks & 1) ? y1.z : y1.x, (ks & 1) ? y0.w : y0.y,
                          (ks & 1) ? y1.w : y1.y, qh[ks][0], qh[ks][1]);
             }
         }
+        float s[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) s[e] = ((sa[0][e] + sa[1][e]) + (sb[0][e] + sb[1][e])) + (sl[0][e] + sl[1][e]);
+        if (more) issue_k(n0, n1, gs1);
 
         // ---- online softmax; lane holds keys p, p+8 x heads 2q, 2q+1
         float s0 = val0 ? s[0] * sc : -INFINITY, s1 = val0 ? s[1] * sc : -INFINITY;
@@ -244,6 +285,12 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_bf16(const AttnArgs a)
             mma16816(o[mt], a0, a1, a2, a3, pb0, pb1);
             mma16816(o[mt], a0, a1, a2, a3, pl0, pl1);
         }
+        if (more) issue_v(n0, n1, gs1);
+        if (gs == 3) {  // the next group starts the prefetched chunk; fetch the one after it
+            cur[0] = nxt[0];
+            cur[1] = nxt[1];
+            load_chunk(base + 16 + 64, nxt);
+        }
     }
 
     // ---- epilogue: full row sums, normalise, undo the head-dim permutation
@@ -254,24 +301,26 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_bf16(const AttnArgs a)
     }
     const float inv0 = 1.f / l0, inv1 = 1.f / l1;
     const int h0 = 2 * q, h1 = 2 * q + 1;
-    TOut *out = reinterpret_cast<TOut *>(a.out) +
-                (((int64_t)t.s * a.N + t.i) * a.Hq + (int64_t)t.g * a.G) * D + p * VRUN;
-    float run[VRUN];
-    if (h0 < a.G) {
+    TOut *out = reinterpret_cast<TOut *>(a.out) + (((int64_t)t.s * a.N + t.i) * a.Hq + (int64_t)t.g * a.G) * D + 8 * p;
+    float run[8];
 #pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            run[2 * mt] = o[mt][0] * inv0;
-            run[2 * mt + 1] = o[mt][2] * inv0;
-        }
-        store_run<TOut>(out + (int64_t)h0 * D, run, VRUN);
-    }
-    if (h1 < a.G) {
+    for (int u = 0; u < VU; ++u) {
+        if (h0 < a.G) {
 #pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            run[2 * mt] = o[mt][1] * inv1;
-            run[2 * mt + 1] = o[mt][3] * inv1;
+            for (int j = 0; j < 4; ++j) {
+                run[2 * j] = o[4 * u + j][0] * inv0;
+                run[2 * j + 1] = o[4 * u + j][2] * inv0;
+            }
+            store_run<TOut>(out + (int64_t)h0 * D + 64 * u, run, 8);
         }
-        store_run<TOut>(out + (int64_t)h1 * D, run, VRUN);
+        if (h1 < a.G) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                run[2 * j] = o[4 * u + j][1] * inv1;
+                run[2 * j + 1] = o[4 * u + j][3] * inv1;
+            }
+            store_run<TOut>(out + (int64_t)h1 * D + 64 * u, run, 8);
+        }
     }
     if (a.lse != nullptr && p == 0) {
         float *lse = a.lse + ((int64_t)t.s * a.Hq + (int64_t)t.g * a.G) * a.N + t.i;
