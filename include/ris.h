@@ -218,6 +218,12 @@ ris_status ris_attention_masked_noalloc(ris_mask_t mask, const void *q, const vo
 ris_status ris_kernel_timer_enable(int32_t enable);
 ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches);
 
+/* Synchronise `stream` and report (then clear) the device error word set by kernels whose
+ * bounded waits gave up: RIS_ERR_DEVICE_TIMEOUT if any did since the last call, else RIS_OK.
+ * A kernel that sets the word skips the rest of its work, so outputs of that launch are
+ * undefined. Blocks. Errors: RIS_ERR_CUDA. */
+ris_status ris_device_status(void *stream);
+
 /* Text of the calling thread's last error ("" if none). The string is owned by the library. */
 const char *ris_last_error(void);
 

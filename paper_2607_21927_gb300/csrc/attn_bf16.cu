@@ -91,19 +91,57 @@ __device__ __forceinline__ void store_run<__nv_bfloat16>(__nv_bfloat16 *dst, con
     }
 }
 
-// D: head dim (64 or 128). QSPLIT: q is fp32 (split hi + lo); else q is bf16.
-// KSPLIT: keys come as a bf16 hi (a.k) + lo (a.k_lo) pair.
+__device__ __forceinline__ void ldg32(const void *p, uint32_t *w)
+{
+    asm volatile("ld.global.nc.v8.u32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
+                 : "l"(p));
+}
+
+__device__ __forceinline__ void ldg16w(const void *p, uint32_t *w)
+{
+    const uint4 x = ldg16(p);
+    w[0] = x.x;
+    w[1] = x.y;
+    w[2] = x.z;
+    w[3] = x.w;
+}
+
+// Head-dim layout of one lane's share of a gathered row (lane p = lane/4, q = lane%4).
+//   K row, WIDE (32-byte loads): lane q holds elements 64u + 16q + [0, 16), u < D/64, and the
+//     four lanes of a row read 128 contiguous bytes per load; narrow (16-byte loads): lane q
+//     holds 32u + 8q + [0, 8), u < D/32 (64 contiguous bytes per row per load).
+//   Either way word 2t / 2t+1 of the lane's K words is the A operand of k-step t, and the
+//   query takes the same elements (kelem below).
+//   V row, WIDE and D = 128: lane p holds 16p + [0, 16) (eight lanes read the whole 256-byte
+//     row); otherwise 64u + 8p + [0, 8), u < D/64. Word j (elements d, d+1) feeds m-tile j.
+template <int D, bool WIDE>
+__device__ __forceinline__ int kelem(int t, int q)
+{
+    return WIDE ? 64 * (t >> 2) + 16 * q + 4 * (t & 3) : 32 * (t >> 1) + 8 * q + 4 * (t & 1);
+}
+
+template <int D, bool WIDE>
+__device__ __forceinline__ int velem(int j, int p)
+{
+    return (WIDE && D == 128) ? 16 * p + 2 * j : 64 * (j >> 2) + 8 * p + 2 * (j & 3);
+}
+
 #ifndef RIS_ATTN_MIN_BLOCKS
 #define RIS_ATTN_MIN_BLOCKS 1
 #endif
 
-template <int D, bool QSPLIT, bool KSPLIT, typename TIdx, bool DENSE, typename TOut>
+// D: head dim (64 or 128). QSPLIT: q is fp32 (split hi + lo); else q is bf16.
+// KSPLIT: keys come as a bf16 hi (a.k) + lo (a.k_lo) pair. WIDE: 32-byte loads (K, K lo and
+// V pointers 32-byte aligned).
+template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut>
 __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
 {
     constexpr int KSTEPS = D / 16;  // k-steps of the score product
-    constexpr int KU = D / 32;      // 16-byte loads per K row per lane (D/2 bytes)
-    constexpr int VU = D / 64;      // 16-byte loads per V row per lane (D/8 elements)
+    constexpr int KW = D / 8;       // 32-bit words of one K row per lane (D/4 elements)
+    constexpr int VW = D / 16;      // 32-bit words of one V row per lane (D/8 elements)
     constexpr int MT = D / 16;      // m-tiles of the value product (head dim)
+    constexpr bool VWIDE = WIDE && D == 128;
 
     const int lane = threadIdx.x & 31;
     const int64_t tid = (int64_t)blockIdx.x * kAttnWarps + (threadIdx.x >> 5);
@@ -121,7 +159,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         const int64_t qrow = (t.i * a.Hq + (int64_t)t.g * a.G + (hv ? p : 0)) * D;
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
-            const int d0 = 32 * (ks >> 1) + 8 * q + 4 * (ks & 1);
+            const int d0 = kelem<D, WIDE>(ks, q);
             if (QSPLIT) {
                 float4 x = hv ? *reinterpret_cast<const float4 *>(reinterpret_cast<const float *>(a.q) + qrow + d0)
                               : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -144,10 +182,10 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     }
 
     const size_t row_bytes = (size_t)a.Hkv * D * sizeof(__nv_bfloat16);
-    const char *kb = reinterpret_cast<const char *>(a.k) + (size_t)t.g * D * sizeof(__nv_bfloat16) + 16 * q;
-    const char *kbl = KSPLIT ? reinterpret_cast<const char *>(a.k_lo) + (size_t)t.g * D * sizeof(__nv_bfloat16) + 16 * q
-                             : nullptr;
-    const char *vb = reinterpret_cast<const char *>(a.v) + (size_t)t.g * D * sizeof(__nv_bfloat16) + 16 * p;
+    const size_t head_off = (size_t)t.g * D * sizeof(__nv_bfloat16);
+    const char *kb = reinterpret_cast<const char *>(a.k) + head_off + 2 * kelem<D, WIDE>(0, q);
+    const char *kbl = KSPLIT ? reinterpret_cast<const char *>(a.k_lo) + head_off + 2 * kelem<D, WIDE>(0, q) : nullptr;
+    const char *vb = reinterpret_cast<const char *>(a.v) + head_off + 2 * velem<D, WIDE>(0, p);
 
     float o[MT][4];
 #pragma unroll
@@ -172,31 +210,33 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         return __shfl_sync(0xFFFFFFFFu, (gs >> 1) ? c1 : c0, (16 * gs + r) & 31);
     };
 
-    // ---- gathered rows of one group: K rows p and p+8 (D/2 bytes each of hi and lo),
-    //      V rows 2q, 2q+1, 2q+8, 2q+9 (D/8 elements each)
-    uint4 k0[KU], k1[KU], kl0[KSPLIT ? KU : 1], kl1[KSPLIT ? KU : 1], v0[VU], v1[VU], v2[VU], v3[VU];
+    // ---- gathered rows of one group: K rows p and p+8, V rows 2q, 2q+1, 2q+8, 2q+9
+    uint32_t k0[KW], k1[KW], kl0[KSPLIT ? KW : 1], kl1[KSPLIT ? KW : 1], v0[VW], v1[VW], v2[VW], v3[VW];
+    auto load_row = [&](const char *rowp, uint32_t *w, int nwords, int stride, bool wide) {
+        if (wide) {
+#pragma unroll
+            for (int u = 0; u < nwords / 8; ++u) ldg32(rowp + stride * u, w + 8 * u);
+        } else {
+#pragma unroll
+            for (int u = 0; u < nwords / 4; ++u) ldg16w(rowp + stride * u, w + 4 * u);
+        }
+    };
     auto issue_k = [&](int c0, int c1, int gs) {
         const int ik0 = slot(c0, c1, gs, p), ik1 = slot(c0, c1, gs, p + 8);
-#pragma unroll
-        for (int u = 0; u < KU; ++u) {
-            k0[u] = ldg16(kb + (size_t)ik0 * row_bytes + 64 * u);
-            k1[u] = ldg16(kb + (size_t)ik1 * row_bytes + 64 * u);
-            if (KSPLIT) {
-                kl0[u % (KSPLIT ? KU : 1)] = ldg16(kbl + (size_t)ik0 * row_bytes + 64 * u);
-                kl1[u % (KSPLIT ? KU : 1)] = ldg16(kbl + (size_t)ik1 * row_bytes + 64 * u);
-            }
+        load_row(kb + (size_t)ik0 * row_bytes, k0, KW, WIDE ? 128 : 64, WIDE);
+        load_row(kb + (size_t)ik1 * row_bytes, k1, KW, WIDE ? 128 : 64, WIDE);
+        if (KSPLIT) {
+            load_row(kbl + (size_t)ik0 * row_bytes, kl0, KW, WIDE ? 128 : 64, WIDE);
+            load_row(kbl + (size_t)ik1 * row_bytes, kl1, KW, WIDE ? 128 : 64, WIDE);
         }
     };
     auto issue_v = [&](int c0, int c1, int gs) {
         const int iv0 = slot(c0, c1, gs, 2 * q), iv1 = slot(c0, c1, gs, 2 * q + 1);
         const int iv2 = slot(c0, c1, gs, 2 * q + 8), iv3 = slot(c0, c1, gs, 2 * q + 9);
-#pragma unroll
-        for (int u = 0; u < VU; ++u) {
-            v0[u] = ldg16(vb + (size_t)iv0 * row_bytes + 128 * u);
-            v1[u] = ldg16(vb + (size_t)iv1 * row_bytes + 128 * u);
-            v2[u] = ldg16(vb + (size_t)iv2 * row_bytes + 128 * u);
-            v3[u] = ldg16(vb + (size_t)iv3 * row_bytes + 128 * u);
-        }
+        load_row(vb + (size_t)iv0 * row_bytes, v0, VW, 128, VWIDE);
+        load_row(vb + (size_t)iv1 * row_bytes, v1, VW, 128, VWIDE);
+        load_row(vb + (size_t)iv2 * row_bytes, v2, VW, 128, VWIDE);
+        load_row(vb + (size_t)iv3 * row_bytes, v3, VW, 128, VWIDE);
     };
 
     // Phase-shifted pipeline: the next group's K rows are requested as soon as this group's
@@ -220,17 +260,13 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
             for (int e = 0; e < 4; ++e) sa[c][e] = sb[c][e] = sl[c][e] = 0.f;
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
-            const uint4 &x0 = k0[ks >> 1], &x1 = k1[ks >> 1];
-            const uint32_t a0 = (ks & 1) ? x0.z : x0.x;
-            const uint32_t a1 = (ks & 1) ? x1.z : x1.x;
-            const uint32_t a2 = (ks & 1) ? x0.w : x0.y;
-            const uint32_t a3 = (ks & 1) ? x1.w : x1.y;
-            mma16816(sa[ks & 1], a0, a1, a2, a3, qh[ks][0], qh[ks][1]);
-            if (QSPLIT) mma16816(sb[ks & 1], a0, a1, a2, a3, ql[ks][0], ql[ks][1]);
+            mma16816(sa[ks & 1], k0[2 * ks], k1[2 * ks], k0[2 * ks + 1], k1[2 * ks + 1], qh[ks][0], qh[ks][1]);
+            if (QSPLIT)
+                mma16816(sb[ks & 1], k0[2 * ks], k1[2 * ks], k0[2 * ks + 1], k1[2 * ks + 1], ql[ks][0], ql[ks][1]);
             if (KSPLIT) {
-                const uint4 &y0 = kl0[(ks >> 1) % (KSPLIT ? KU : 1)], &y1 = kl1[(ks >> 1) % (KSPLIT ? KU : 1)];
-                mma16816(sl[ks & 1], (ks & 1) ? y0.z : y0.x, (ks & 1) ? y1.z : y1.x, (ks & 1) ? y0.w : y0.y,
-                         (ks & 1) ? y1.w : y1.y, qh[ks][0], qh[ks][1]);
+                constexpr int LW = KSPLIT ? KW : 1;
+                mma16816(sl[ks & 1], kl0[(2 * ks) % LW], kl1[(2 * ks) % LW], kl0[(2 * ks + 1) % LW],
+                         kl1[(2 * ks + 1) % LW], qh[ks][0], qh[ks][1]);
             }
         }
         float s[4];
@@ -272,16 +308,12 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         const uint32_t pl1 = transpose8x8(pack_bf16(p2 - h2, p3 - h3));
 
         // ---- O^T += V^T P^T
-        const uint32_t *w0 = reinterpret_cast<const uint32_t *>(v0);
-        const uint32_t *w1 = reinterpret_cast<const uint32_t *>(v1);
-        const uint32_t *w2 = reinterpret_cast<const uint32_t *>(v2);
-        const uint32_t *w3 = reinterpret_cast<const uint32_t *>(v3);
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
-            const uint32_t a0 = __byte_perm(w0[mt], w1[mt], 0x5410);
-            const uint32_t a1 = __byte_perm(w0[mt], w1[mt], 0x7632);
-            const uint32_t a2 = __byte_perm(w2[mt], w3[mt], 0x5410);
-            const uint32_t a3 = __byte_perm(w2[mt], w3[mt], 0x7632);
+            const uint32_t a0 = __byte_perm(v0[mt], v1[mt], 0x5410);
+            const uint32_t a1 = __byte_perm(v0[mt], v1[mt], 0x7632);
+            const uint32_t a2 = __byte_perm(v2[mt], v3[mt], 0x5410);
+            const uint32_t a3 = __byte_perm(v2[mt], v3[mt], 0x7632);
             mma16816(o[mt], a0, a1, a2, a3, pb0, pb1);
             mma16816(o[mt], a0, a1, a2, a3, pl0, pl1);
         }
@@ -301,25 +333,28 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     }
     const float inv0 = 1.f / l0, inv1 = 1.f / l1;
     const int h0 = 2 * q, h1 = 2 * q + 1;
-    TOut *out = reinterpret_cast<TOut *>(a.out) + (((int64_t)t.s * a.N + t.i) * a.Hq + (int64_t)t.g * a.G) * D + 8 * p;
-    float run[8];
+    TOut *out = reinterpret_cast<TOut *>(a.out) + (((int64_t)t.s * a.N + t.i) * a.Hq + (int64_t)t.g * a.G) * D;
+    // runs of 8 consecutive head-dim elements: words 4r .. 4r+3 of the lane's V layout
+    constexpr int RUNS = MT / 4;
 #pragma unroll
-    for (int u = 0; u < VU; ++u) {
+    for (int r = 0; r < RUNS; ++r) {
+        float run[8];
+        const int d = velem<D, WIDE>(4 * r, p);
         if (h0 < a.G) {
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                run[2 * j] = o[4 * u + j][0] * inv0;
-                run[2 * j + 1] = o[4 * u + j][2] * inv0;
+                run[2 * j] = o[4 * r + j][0] * inv0;
+                run[2 * j + 1] = o[4 * r + j][2] * inv0;
             }
-            store_run<TOut>(out + (int64_t)h0 * D + 64 * u, run, 8);
+            store_run<TOut>(out + (int64_t)h0 * D + d, run, 8);
         }
         if (h1 < a.G) {
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                run[2 * j] = o[4 * u + j][1] * inv1;
-                run[2 * j + 1] = o[4 * u + j][3] * inv1;
+                run[2 * j] = o[4 * r + j][1] * inv1;
+                run[2 * j + 1] = o[4 * r + j][3] * inv1;
             }
-            store_run<TOut>(out + (int64_t)h1 * D + 64 * u, run, 8);
+            store_run<TOut>(out + (int64_t)h1 * D + d, run, 8);
         }
     }
     if (a.lse != nullptr && p == 0) {
@@ -329,21 +364,32 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     }
 }
 
-template <int D, bool QSPLIT, typename TOut>
-cudaError_t launch_d(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t s)
+template <int D, bool QSPLIT, bool WIDE, typename TOut>
+cudaError_t launch_w(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t s)
 {
     // rotated inputs: fp32 queries and hi + lo keys; as given: bf16 queries and keys
     constexpr bool KSPLIT = QSPLIT;
     const unsigned grid = (unsigned)((a.n_tasks + kAttnWarps - 1) / kAttnWarps);
     const dim3 block(kAttnWarps * 32);
     if (dense)
-        k_attn_bf16<D, QSPLIT, KSPLIT, uint32_t, true, TOut><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, true, TOut><<<grid, block, 0, s>>>(a);
     else if (col_bytes == 2)
-        k_attn_bf16<D, QSPLIT, KSPLIT, uint16_t, false, TOut><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut><<<grid, block, 0, s>>>(a);
     else
-        k_attn_bf16<D, QSPLIT, KSPLIT, uint32_t, false, TOut><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut><<<grid, block, 0, s>>>(a);
     note_launch();
     return cudaGetLastError();
+}
+
+bool aligned32(const void *p) { return p == nullptr || (reinterpret_cast<uintptr_t>(p) & 31u) == 0; }
+
+template <int D, bool QSPLIT, typename TOut>
+cudaError_t launch_d(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t s)
+{
+    // 32-byte loads need 32-byte aligned K, K lo and V (the ABI promises 16)
+    if (aligned32(a.k) && aligned32(a.k_lo) && aligned32(a.v))
+        return launch_w<D, QSPLIT, true, TOut>(a, col_bytes, dense, s);
+    return launch_w<D, QSPLIT, false, TOut>(a, col_bytes, dense, s);
 }
 
 template <bool QSPLIT, typename TOut>

@@ -8,6 +8,7 @@
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <new>
@@ -138,6 +139,17 @@ std::pair<cudaEvent_t, cudaEvent_t> timer_pair()
     }
     g_timer.used.push_back(e);
     return e;
+}
+
+// bf16 kernel design: register gather (default) or TMA gather (RIS_FORCE_DESIGN=tma, for
+// benchmarking the two designs against each other).
+bool use_tma_gather()
+{
+    static const bool tma = [] {
+        const char *e = std::getenv("RIS_FORCE_DESIGN");
+        return e != nullptr && std::string(e) == "tma" && tma_gather_available();
+    }();
+    return tma;
 }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -545,7 +557,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.n_tasks = (int64_t)a.n_sets * N * kv_heads;
     const auto ev = timer_pair();
     if (ev.first) RIS_CUDA(cudaEventRecord(ev.first, s));
-    if (dtype == RIS_BF16)
+    if (dtype == RIS_BF16 && use_tma_gather())
+        RIS_CUDA(launch_attention_tma(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
+    else if (dtype == RIS_BF16)
         RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
     else
         RIS_CUDA(launch_attention_f32(a, head_dim, out_dtype, m->col_bytes, m->dense != 0, s));
@@ -600,6 +614,14 @@ ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches)
     *total_ms = tot;
     *launches = (int64_t)g_timer.used.size();
     timer_clear_locked();
+    return RIS_OK;
+}
+
+ris_status ris_device_status(void *stream)
+{
+    unsigned int word = 0;
+    RIS_CUDA(read_device_error(&word, reinterpret_cast<cudaStream_t>(stream)));
+    if (word != 0u) return fail(RIS_ERR_DEVICE_TIMEOUT, "a device-side wait gave up (error word 0x%x)", word);
     return RIS_OK;
 }
 

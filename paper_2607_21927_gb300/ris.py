@@ -86,6 +86,7 @@ _SIGS = {
                                      ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p,
                                      ctypes.c_void_p],
     "ris_kernel_timer_enable": [ctypes.c_int32],
+    "ris_device_status": [ctypes.c_void_p],
     "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
 }
 
@@ -120,6 +121,11 @@ def ris_launch_count() -> int:
 
 def ris_version() -> str:
     return lib().ris_version().decode()
+
+
+def ris_device_status(stream=None) -> None:
+    """Synchronise and raise RisError(RIS_ERR_DEVICE_TIMEOUT) if a device-side wait gave up."""
+    _check("ris_device_status", lib().ris_device_status(_stream(stream)))
 
 
 def ris_kernel_timer_enable(enable: bool = True) -> None:
