@@ -99,12 +99,6 @@ struct Scratch {
         s = st;
         return cudaMallocAsync(&p, bytes < 16 ? 16 : bytes, st);
     }
-    void *release()
-    {
-        void *q = p;
-        p = nullptr;
-        return q;
-    }
     ~Scratch()
     {
         if (p) cudaFreeAsync(p, s);
@@ -141,15 +135,31 @@ std::pair<cudaEvent_t, cudaEvent_t> timer_pair()
     return e;
 }
 
-// bf16 kernel design: register gather (default) or TMA gather (RIS_FORCE_DESIGN=tma, for
-// benchmarking the two designs against each other).
-bool use_tma_gather()
+// Kernel design override for benchmarking the designs against each other:
+// RIS_FORCE_DESIGN = gather (register gather), tma (TMA gather) or tile (masked dense tiles).
+const char *forced_design()
 {
-    static const bool tma = [] {
+    static const std::string d = [] {
         const char *e = std::getenv("RIS_FORCE_DESIGN");
-        return e != nullptr && std::string(e) == "tma" && tma_gather_available();
+        return std::string(e ? e : "");
     }();
-    return tma;
+    return d.c_str();
+}
+
+bool use_tma_gather() { return std::string(forced_design()) == "tma" && tma_gather_available(); }
+
+// Union density at and above which masked dense tiles beat gathering pair by pair (bf16,
+// head dim 128): a tile costs the dense causal products (x2.5 for the precision splits)
+// whatever the mask, a gathered pair 1.5 KB of K/V rows.
+constexpr double kTileDensity = 0.2;
+
+bool use_tile_design(const ris_mask_s *m)
+{
+    const std::string f = forced_design();
+    if (!tile_design_available() || f == "gather" || f == "tma") return false;
+    if (f == "tile" || m->dense) return true;
+    const double causal = (double)m->n_masks * ((double)m->N * (double)(m->N + 1) / 2.0);
+    return (double)m->n_pairs >= kTileDensity * causal;
 }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -508,8 +518,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
 {
     const int64_t N = m->N;
     prepare_pool_once();
-    Scratch qt, kt, ktl;
-    const void *qu = q, *ku = k, *kl = nullptr;
+    const bool tile = dtype == RIS_BF16 && head_dim == 128 && use_tile_design(m);
+    Scratch qt, qtl, kt, ktl;
+    const void *qu = q, *ku = k, *kl = nullptr, *q_lo = nullptr;
     bool q_split = false;
     if (rope != nullptr && rope->kind != RIS_ROPE_NONE) {
         RopeArgs ra{};
@@ -519,21 +530,29 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         ra.D = head_dim;
         ra.mscale = (float)ms;
         const size_t nq = (size_t)N * heads * head_dim, nk = (size_t)N * kv_heads * head_dim;
-        // rotated queries in fp32 (split into bf16 hi + lo by the tensor-core path); rotated
-        // keys in fp32, or for bf16 inputs as a bf16 hi + lo pair
-        RIS_CUDA(qt.alloc(nq * sizeof(float), s));
+        // rotated queries: fp32 (split into bf16 hi + lo by the gather kernels) or, for the
+        // tile kernel, a bf16 hi + lo pair; rotated keys in fp32, or for bf16 inputs a bf16
+        // hi + lo pair
+        if (tile) {
+            RIS_CUDA(qt.alloc(nq * 2, s));
+            RIS_CUDA(qtl.alloc(nq * 2, s));
+        } else {
+            RIS_CUDA(qt.alloc(nq * sizeof(float), s));
+        }
         RIS_CUDA(kt.alloc(nk * (dtype == RIS_BF16 ? 2 : 4), s));
         if (dtype == RIS_BF16) RIS_CUDA(ktl.alloc(nk * 2, s));
         ra.x_in = q;
         ra.x_out = qt.p;
+        ra.x_out_lo = tile ? qtl.p : nullptr;
         ra.H = heads;
-        RIS_CUDA(launch_rope(ra, dtype, RIS_F32, s));
+        RIS_CUDA(launch_rope(ra, dtype, tile ? RIS_BF16 : RIS_F32, s));
         ra.x_in = k;
         ra.x_out = kt.p;
         ra.x_out_lo = ktl.p;
         ra.H = kv_heads;
         RIS_CUDA(launch_rope(ra, dtype, dtype, s));
         qu = qt.p;
+        q_lo = qtl.p;
         ku = kt.p;
         kl = ktl.p;
         q_split = (dtype == RIS_BF16);
@@ -547,6 +566,8 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.lse = lse;
     a.row_ptr = m->row_ptr;
     a.col = m->col;
+    a.bitmap = m->bitmap;
+    a.words_per_mask = m->words_per_mask;
     a.N = N;
     a.Hq = heads;
     a.Hkv = kv_heads;
@@ -557,7 +578,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.n_tasks = (int64_t)a.n_sets * N * kv_heads;
     const auto ev = timer_pair();
     if (ev.first) RIS_CUDA(cudaEventRecord(ev.first, s));
-    if (dtype == RIS_BF16 && use_tma_gather())
+    if (tile)
+        RIS_CUDA(launch_attention_tile(a, qu, q_lo, out_dtype, m->dense != 0, s));
+    else if (dtype == RIS_BF16 && use_tma_gather())
         RIS_CUDA(launch_attention_tma(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
     else if (dtype == RIS_BF16)
         RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
@@ -619,8 +642,10 @@ ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches)
 
 ris_status ris_device_status(void *stream)
 {
-    unsigned int word = 0;
+    unsigned int word = 0, tile_word = 0;
     RIS_CUDA(read_device_error(&word, reinterpret_cast<cudaStream_t>(stream)));
+    RIS_CUDA(read_tile_error(&tile_word));
+    word |= tile_word;
     if (word != 0u) return fail(RIS_ERR_DEVICE_TIMEOUT, "a device-side wait gave up (error word 0x%x)", word);
     return RIS_OK;
 }

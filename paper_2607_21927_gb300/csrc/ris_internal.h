@@ -70,6 +70,8 @@ struct AttnArgs {
     float *lse;            // [n_sets][Hq][N] or null
     const int64_t *row_ptr;  // [n_masks * N + 1] (null when dense)
     const void *col;       // keys (null when dense)
+    const uint32_t *bitmap;  // causal bitmap rows (null when dense)
+    int64_t words_per_mask;
     int64_t N;
     int32_t Hq;
     int32_t Hkv;
@@ -108,5 +110,12 @@ bool tma_gather_available();
 cudaError_t launch_attention_tma(const AttnArgs &a, int D, int out_dtype, bool split, int col_bytes, bool dense,
                                  cudaStream_t s);
 cudaError_t read_device_error(unsigned int *out, cudaStream_t s);
+
+// Masked dense-tile design (tcgen05, head dim 128): q_hi / q_lo bf16 query pair (q_lo null
+// for exact bf16 inputs).
+bool tile_design_available();
+cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const void *q_lo, int out_dtype, bool dense,
+                                  cudaStream_t s);
+cudaError_t read_tile_error(unsigned int *out);
 
 }  // namespace ris
