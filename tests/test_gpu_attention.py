@@ -202,3 +202,28 @@ def test_c2_ensemble_per_seed_sampled():
     for s in (0, 9):
         ref, _ = run_oracle(qn, kn, vn, 0, 0.01, seeds, 1, 1e6, 32768, rows=rows, seed_index=s)
         check_bf16_path(got[s], ref)
+
+
+def test_attention_u32_keys_beyond_65536():
+    """N > 65536 stores 32-bit key indices; sampled rows against the oracle."""
+    N, Hq, Hkv, D = 65600, 2, 1, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=17, outliers=True)
+    out = ris.ris_sparse_attention_fwd(q, k, v, 0, 0.0005, [2], rope=ris.rope_cfg(3, 1e6, 32768),
+                                       out_dtype=torch.float32)
+    torch.cuda.synchronize()
+    rows = sample_rows(N, 24, seed=5)
+    ref, _ = run_oracle(qn, kn, vn, 0, 0.0005, [2], 3, 1e6, 32768, rows=rows)
+    check_bf16_path(to_np(out[rows]), ref)
+
+
+def test_dense_tiles_bf16_output_and_lse():
+    """High union density goes to the masked-tile kernel; bf16 output and lse against the oracle."""
+    N, Hq, Hkv, D = 600, 12, 2, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=23, outliers=True)
+    out, lse = ris.ris_sparse_attention_fwd(q, k, v, 0, 0.5, [1, 2], rope=ris.rope_cfg(3, 1e6, 256),
+                                            return_lse=True)
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    ref, ref_lse = run_oracle(qn, kn, vn, 0, 0.5, [1, 2], 3, 1e6, 256)
+    check_bf16_path(to_np(out), ref, out_bf16=True)
+    np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-2)
