@@ -91,9 +91,11 @@ __device__ __forceinline__ void store_run<__nv_bfloat16>(__nv_bfloat16 *dst, con
     }
 }
 
+// 32-byte load that does not allocate in L1: each gathered sector is consumed whole by the
+// one instruction that loads it, so caching it in L1 only costs data-pipe bandwidth.
 __device__ __forceinline__ void ldg32(const void *p, uint32_t *w)
 {
-    asm volatile("ld.global.nc.v8.u32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+    asm volatile("ld.global.nc.L1::no_allocate.v8.u32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
                  : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
                  : "l"(p));
 }
