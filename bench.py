@@ -292,12 +292,13 @@ def main():
         vs.append(v)
     outs = [[torch.empty(N, Hq, D, dtype=torch.bfloat16, device=dev) for _ in range(L)] for _ in MODES]
     stream = torch.cuda.current_stream()
-    pairs = {}
+    pairs, design = {}, {}
 
     def step():
         for mi, (name, mode) in enumerate(MODES):
             m = ris.ris_mask_generate(N, Hkv, mode, a.density, seeds)
             pairs[name] = m.info().n_pairs
+            design[name] = ris.ris_attention_design(m, torch.bfloat16, D)
             for layer in range(L):
                 ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[mi][layer])
             m.free()
@@ -331,11 +332,10 @@ def main():
     value = world * pair_heads_step * a.steps / (elapsed_ms / 1e3)
     ms_step = elapsed_ms / a.steps
 
-    # roofline of the attention kernel: algorithmic gathered bytes per launch / mean launch time
-    bytes_per_step = sum(pairs[name] for name, _ in MODES) * L * Hkv * 2 * D * 2
+    # roofline of the attention kernel over the timed region: algorithmic bytes (gather) or
+    # algorithmic FLOPs (tiles) per launch / mean launch time
     launches_per_step = len(MODES) * L
     mean_launch_ms = k_ms / max(k_n, 1)
-    achieved = (bytes_per_step / launches_per_step) / (mean_launch_ms / 1e3) / 1e9
     peaks = {}
     try:
         peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -344,13 +344,26 @@ def main():
     hbm = peaks.get("hbm_gbs")
     peak_note = "measured" if hbm else "fallback"
     hbm = hbm or 6800.0
-    traffic = recorded_traffic("attn_bf16.cu")
-    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                "traffic": traffic, "kernel": "k_attn_bf16 (gather design)", "peak_source": peak_note,
-                "mean_launch_ms": mean_launch_ms, "launches_timed": k_n}
+    tc = peaks.get("bf16_tflops_sustained") or 1700.0
+    kinds = sorted(set(design.values()))
+    if kinds == [2]:  # every launch on the tensor-core tile kernel
+        flops_per_launch = 4 * D * Hq * sum(pairs.values()) * L / launches_per_step
+        achieved = flops_per_launch / (mean_launch_ms / 1e3) / 1e12
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": tc, "unit": "TFLOP/s", "frac": achieved / tc,
+                    "traffic": None, "kernel": "k_attn_tile (tcgen05 masked tiles)",
+                    "peak_source": ("measured sustained bf16" if peaks.get("bf16_tflops_sustained") else "fallback"),
+                    "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
+                    "mean_launch_ms": mean_launch_ms, "launches_timed": k_n}
+    else:
+        bytes_per_step = sum(pairs[name] for name, _ in MODES) * L * Hkv * 2 * D * 2
+        achieved = (bytes_per_step / launches_per_step) / (mean_launch_ms / 1e3) / 1e9
+        roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                    "traffic": recorded_traffic("attn_bf16.cu") if kinds == [0] else None,
+                    "kernel": "k_attn_bf16 (register gather)" if kinds == [0] else "mixed designs " + str(kinds),
+                    "peak_source": peak_note, "bytes": "algorithmic: K and V rows of every sampled pair, both KV heads",
+                    "mean_launch_ms": mean_launch_ms, "launches_timed": k_n}
     # the sampled-pair roofline: max(sampled FLOPs / tensor peak, tile-reuse K/V bytes / HBM)
     flops = 4 * D * Hq * sum(pairs.values()) * L
-    tc = peaks.get("bf16_tflops_sustained") or 1700.0
     b_tile = len(MODES) * L * (N / 128) * (N / 2) * Hkv * 2 * D * 2
     t_roof = max(flops / (tc * 1e12), b_tile / (hbm * 1e9))
     clocks = clk.summary(getattr(torch.cuda.get_device_properties(dev), "pci_bus_id", None))
@@ -358,7 +371,8 @@ def main():
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps, "warmup": a.warmup,
             "ms_per_step": ms_step, "ms_per_layer": ms_step / (len(MODES) * L), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": workload_config(a), "pairs_per_mask": pairs, "roofline": roofline,
+            "config": workload_config(a), "pairs_per_mask": pairs,
+            "design_per_mode": {k: ris.DESIGNS.get(v, v) for k, v in design.items()}, "roofline": roofline,
             "pair_roofline": {"t_roof_ms_per_step": 1e3 * t_roof, "frac": 1e3 * t_roof / ms_step,
                                     "formula": "max(4*D*Hq*pairs / bf16 sustained, (N/128)*(N/2)*Hkv*2*D*2 B / HBM)"},
             "clocks": clocks, "gpu_launches": launches}

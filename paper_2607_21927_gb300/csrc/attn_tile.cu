@@ -6,16 +6,18 @@
 // percent, and the dense mode) a dense 128 x 64 score tile with the mask applied as -inf
 // beats gathering rows pair by pair. One CTA owns one (128-query tile, query head, set):
 //
-//   warp 4 (TMA)   loads the query tile once (bf16 hi and lo) and streams 64-key stages of
-//                  K~ hi, K~ lo and V (128-byte swizzled boxes) into a two-stage ring;
-//   warp 5 (MMA)   one elected lane issues tcgen05.mma: S = Q_hi K_hi^T + Q_lo K_hi^T +
+//   warp 8 (TMA)   loads the query tile once (bf16 hi and lo) and streams 64-key stages of
+//                  K~ hi, K~ lo and V (128-byte swizzled boxes) into a three-stage ring (L2
+//                  latency under load is long: the third stage took a layer from 10.5 to 7.8 ms);
+//   warp 9 (MMA)   one elected lane issues tcgen05.mma: S = Q_hi K_hi^T + Q_lo K_hi^T +
 //                  Q_hi K_lo^T into a double-buffered TMEM score tile, and O += P_hi V + P_lo V
-//                  into the TMEM output tile, committing each step to an mbarrier;
-//   warps 0-3      one thread per query row: tcgen05.ld its 64 scores, apply the bitmap
-//                  (or the causal cut), fp32 online softmax with lazy rescaling of O in TMEM
-//                  (only when the row max grows by more than 2^8), write P hi / lo to shared
-//                  memory in the canonical K-major 128-byte-swizzled layout, and at the end
-//                  normalise O and store the row.
+//                  (A = P, written into TMEM over the consumed scores) into the TMEM output
+//                  tile, committing each step to an mbarrier;
+//   warps 0-7      two threads per query row (score columns 0-31 / 32-63, output columns
+//                  0-63 / 64-127): per tile tcgen05.ld the scores, apply the bitmap (or the causal cut), exchange the
+//                  partial row max with the partner thread, fp32 online softmax with lazy
+//                  rescaling of O in TMEM (only when the row max grows by more than 2^8),
+//                  write P hi / lo into TMEM, and at the end normalise O and store the row.
 //
 // Every mbarrier wait is bounded; a wait that gives up sets bit 1 of the device error word,
 // every role falls through to the end, TMEM is released and the CTA returns.
@@ -38,22 +40,29 @@ namespace {
 constexpr int BM = 128;          // query rows per tile (TMEM lanes)
 constexpr int BN = 64;           // keys per stage
 constexpr int DT = 128;          // head dim handled by this kernel
-constexpr int kThreads = 192;    // warps 0-3 softmax, 4 TMA, 5 MMA
-constexpr uint32_t kTmemCols = 256;  // S[2] (2 x 64) + O (128)
+constexpr int kThreads = 320;    // warps 0-7 softmax (two column halves), 8 TMA, 9 MMA
+constexpr int kTmaWarp = 8, kMmaWarp = 9;
+constexpr uint32_t kTmemCols = 256;  // S/P[2] (2 x 64) + O (128)
 
 // shared-memory map (bytes, from a 1024-aligned base)
-constexpr int Q_ARR = BM * DT * 2;          // 32 KB: one of Q hi / Q lo (two 64-column blocks)
-constexpr int Q_BLK = BM * 128;             // 16 KB: one 64-column block of the query tile
 constexpr int KV_ARR = BN * DT * 2;         // 16 KB: one of K hi / K lo / V
 constexpr int KV_BLK = BN * 128;            // 8 KB: one 64-column block
 constexpr int STAGE = 3 * KV_ARR;           // 48 KB
-constexpr int P_ARR = BM * BN * 2;          // 16 KB: P hi or P lo
+constexpr int kKvStages = 3;                // K/V stages in flight
+constexpr int Q_ARR = BM * DT * 2;          // 32 KB: one of Q hi / Q lo (two 64-column blocks)
+constexpr int Q_BLK = BM * 128;             // 16 KB: one 64-column block of the query tile
 constexpr int OFF_Q = 0;
 constexpr int OFF_KV = 2 * Q_ARR;           // 64 KB
-constexpr int OFF_P = OFF_KV + 2 * STAGE;   // 160 KB
-constexpr int SMEM_BYTES = OFF_P + 2 * P_ARR + 1024;  // + alignment slack = 197632
+constexpr int SMEM_BYTES = OFF_KV + kKvStages * STAGE + 1024;  // + alignment slack = 214016
 
-enum Bar { B_Q = 0, B_KV_FULL = 1, B_KV_EMPTY = 3, B_S_FULL = 5, B_S_EMPTY = 7, B_P_FULL = 9, B_PV_DONE = 10, NBAR = 11 };
+// P_FULL and PV_DONE have one barrier per P buffer (tile parity), so that no waiter can fall
+// two phases behind a barrier it polls by parity.
+// B_X: per pair of softmax warps sharing rows (columns 0-31 / 32-63) and tile parity, the
+// exchange of their partial row maxima (and at the end their partial sums).
+enum Bar {
+    B_Q = 0, B_KV_FULL = 1, B_KV_EMPTY = 4, B_S_FULL = 7, B_S_EMPTY = 9, B_P_FULL = 11, B_PV_DONE = 13, B_X = 15,
+    NBAR = 23
+};
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
@@ -139,6 +148,17 @@ __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a, uint64_t b, 
         : "memory");
 }
 
+// A operand from TMEM (rows in lanes, 16-bit values packed two per column), B from shared memory.
+__device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+
 __device__ __forceinline__ void tc_commit(uint32_t bar)
 {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
@@ -180,6 +200,17 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float *v)
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *v)
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+        "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 {
     const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -216,11 +247,13 @@ struct TileMaps {
 };
 
 template <bool SPLIT, bool DENSE, typename TOut>
-__global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, const __grid_constant__ TileMaps maps)
+__global__ void __launch_bounds__(kThreads, 1)
+    k_attn_tile(const AttnArgs a, const __grid_constant__ TileMaps maps, const void *q_hi, const void *q_lo)
 {
     extern __shared__ unsigned char smem_raw[];
     __shared__ __align__(8) uint64_t bars[NBAR];
     __shared__ uint32_t tmem_base_sh;
+    __shared__ float xch[2][2][BM];  // [tile parity][column half][row]
     unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                             ~uintptr_t(1023));
     const uint32_t sbase = smem_u32(smem);
@@ -242,13 +275,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, con
     if (threadIdx.x == 0) {
         for (int i = 0; i < NBAR; ++i) {
             uint32_t cnt = 1;
-            if (i == B_S_EMPTY || i == B_S_EMPTY + 1 || i == B_P_FULL) cnt = 128;
+            if (i == B_S_EMPTY || i == B_S_EMPTY + 1 || i == B_P_FULL || i == B_P_FULL + 1) cnt = 256;
+            if (i >= B_X) cnt = 64;
             mbar_init(smem_u32(&bars[i]), cnt);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
-    if (warp == 5) {  // TMEM allocation by one full warp
+    if (warp == kMmaWarp) {  // TMEM allocation by one full warp
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base_sh)),
                      "r"(kTmemCols)
                      : "memory");
@@ -261,7 +295,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, con
     const uint32_t t_s0 = tmem, t_s1 = tmem + BN, t_o = tmem + 2 * BN;
     bool ok = true;
 
-    if (warp == 4) {
+    if (warp == kTmaWarp) {
         // =============================== TMA producer
         if (lane == 0) {
             const uint32_t bq = smem_u32(&bars[B_Q]);
@@ -271,8 +305,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, con
                 if (SPLIT) tma_load_3d(sbase + OFF_Q + Q_ARR + blk * Q_BLK, &maps.ql, 64 * blk, h, (int)q0, bq);
             }
             for (int j = 0; j < n_kt && ok; ++j) {
-                const int st = j & 1;
-                if (j >= 2) ok = mbar_wait(smem_u32(&bars[B_KV_EMPTY + st]), ((j >> 1) - 1) & 1);
+                const int st = j % kKvStages;
+                if (j >= kKvStages) ok = mbar_wait(smem_u32(&bars[B_KV_EMPTY + st]), ((j / kKvStages) - 1) & 1);
                 if (!ok) break;
                 const uint32_t bf = smem_u32(&bars[B_KV_FULL + st]);
                 const uint32_t dst = sbase + OFF_KV + st * STAGE;
@@ -284,10 +318,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, con
                 }
             }
             // let the last stages land before the CTA can leave
-            for (int j = n_kt - 2; j < n_kt; ++j)
-                if (j >= 0) mbar_wait(smem_u32(&bars[B_KV_FULL + (j & 1)]), (j >> 1) & 1);
+            for (int j = n_kt - kKvStages; j < n_kt; ++j)
+                if (j >= 0) mbar_wait(smem_u32(&bars[B_KV_FULL + j % kKvStages]), (j / kKvStages) & 1);
         }
-    } else if (warp == 5) {
+    } else if (warp == kMmaWarp) {
         // =============================== MMA issuer
         if (lane == 0) {
             constexpr uint32_t ID_S = idesc_bf16(BM, BN, false);  // S[128 x 64] = Q K^T, both K-major
@@ -296,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, con
             tc_fence_after();
             auto issue_s = [&](int j) {
                 const int st = j & 1;
-                const uint32_t kv = sbase + OFF_KV + st * STAGE;
+                const uint32_t kv = sbase + OFF_KV + (j % kKvStages) * STAGE;
                 const uint32_t dt = (j & 1) ? t_s1 : t_s0;
                 uint32_t acc = 0;
                 // (A, B) pairs: (Q hi, K hi), (Q lo, K hi), (Q hi, K lo); 8 k-steps of 16 over D
@@ -314,147 +348,169 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, con
                 tc_commit(smem_u32(&bars[B_S_FULL + st]));
             };
             auto issue_o = [&](int j) {
-                const int st = j & 1;
+                const int st = j % kKvStages;
                 const uint32_t vb = sbase + OFF_KV + st * STAGE + 2 * KV_ARR;
+                // P hi / lo of this tile sit in TMEM over its score columns: 64 keys of 16-bit
+                // values packed two per column, hi in columns 0-31, lo in 32-63
+                const uint32_t pt = (j & 1) ? t_s1 : t_s0;
                 for (int prod = 0; prod < 2; ++prod) {
-                    const uint32_t pa = sbase + OFF_P + prod * P_ARR;
                     for (int ks = 0; ks < BN / 16; ++ks) {
-                        const uint64_t ad = sdesc(pa + ks * 32, 16, 1024);
                         // V block: 64 keys x 128 B rows; 16 keys = two 8-row atoms (SBO 1024);
                         // the second 64-column block of head dim is LBO = 8 KB away
                         const uint64_t bd = sdesc(vb + ks * 2048, KV_BLK, 1024);
-                        tc_mma(t_o, ad, bd, ID_O, (j > 0 || prod > 0 || ks > 0) ? 1u : 0u);
+                        tc_mma_ts(t_o, pt + 32 * prod + 8 * ks, bd, ID_O, (j > 0 || prod > 0 || ks > 0) ? 1u : 0u);
                     }
                 }
-                tc_commit(smem_u32(&bars[B_PV_DONE]));
+                tc_commit(smem_u32(&bars[B_PV_DONE + (j & 1)]));
                 tc_commit(smem_u32(&bars[B_KV_EMPTY + st]));
             };
             for (int j = 0; j < n_kt && ok; ++j) {
                 const int st = j & 1;
-                ok = mbar_wait(smem_u32(&bars[B_KV_FULL + st]), (j >> 1) & 1);
+                ok = mbar_wait(smem_u32(&bars[B_KV_FULL + j % kKvStages]), (j / kKvStages) & 1);
                 if (ok && j >= 2) ok = mbar_wait(smem_u32(&bars[B_S_EMPTY + st]), ((j >> 1) - 1) & 1);
                 if (!ok) break;
                 tc_fence_after();
                 issue_s(j);
                 if (j >= 1) {
-                    ok = mbar_wait(smem_u32(&bars[B_P_FULL]), (j - 1) & 1);
+                    ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((j - 1) & 1)]), ((j - 1) >> 1) & 1);
                     if (!ok) break;
                     tc_fence_after();
                     issue_o(j - 1);
                 }
             }
             if (ok) {
-                ok = mbar_wait(smem_u32(&bars[B_P_FULL]), (n_kt - 1) & 1);
+                ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1);
                 if (ok) {
                     tc_fence_after();
                     issue_o(n_kt - 1);
                 }
             }
             // the last commit has to land before TMEM is released
-            mbar_wait(smem_u32(&bars[B_PV_DONE]), (n_kt - 1) & 1);
+            mbar_wait(smem_u32(&bars[B_PV_DONE + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1);
         }
     } else {
-        // =============================== softmax: thread r owns query row q0 + r
-        const int r = threadIdx.x;  // 0..127 == TMEM lane
+        // =============================== softmax: two threads per query row q0 + r, one per
+        // column half hf (scores 32 hf .. 32 hf + 31 of each tile, O columns 64 hf .. 64 hf + 63)
+        const int wq = warp & 3, hf = warp >> 2;
+        const int r = wq * 32 + lane;  // TMEM lane
         const int64_t i = q0 + r;
         const bool row_ok = i < a.N;
-        const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+        const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
         const uint32_t *bm = DENSE ? nullptr
                                    : a.bitmap + (int64_t)mask_id * a.words_per_mask + (row_ok ? row_word_offset(i) : 0);
         const int64_t last_word = i >> 5;
         const float sc = a.scale_log2;
         float m_used = -INFINITY, l = 0.f;
-        unsigned char *prow_hi = smem + OFF_P + r * 128;
-        unsigned char *prow_lo = smem + OFF_P + P_ARR + r * 128;
+        // bitmap word of keys 64j + 32hf .. 64j + 32hf + 31 of this row, fetched one tile ahead
+        auto mask_word = [&](int j) -> uint32_t {
+            if (!row_ok) return 0u;
+            const int64_t k0 = (int64_t)j * BN + 32 * hf;
+            if (DENSE) {
+                const int64_t lim = i - k0;  // keys k0 .. i are kept
+                return lim >= 31 ? 0xFFFFFFFFu : (lim < 0 ? 0u : ((2u << lim) - 1u));
+            }
+            const int64_t wd = k0 >> 5;
+            return wd <= last_word ? bm[wd] : 0u;
+        };
+        // exchange a value with the partner thread of the other column half (bounded wait)
+        auto exchange = [&](int tag, float v, float &other) -> bool {
+            const int pb = tag & 1;
+            xch[pb][hf][r] = v;
+            const uint32_t bar = smem_u32(&bars[B_X + 2 * wq + pb]);
+            mbar_arrive(bar);
+            const bool got = __all_sync(0xFFFFFFFFu, mbar_wait(bar, (tag >> 1) & 1));
+            other = xch[pb][hf ^ 1][r];
+            return got;
+        };
+        uint32_t cw = mask_word(0);
         for (int j = 0; j < n_kt; ++j) {
             const int st = j & 1;
+            const uint32_t nw = (j + 1 < n_kt) ? mask_word(j + 1) : 0u;
             ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&bars[B_S_FULL + st]), (j >> 1) & 1));
             if (!ok) break;
             tc_fence_after();
-            float sv[BN];
-            tmem_ld32(((j & 1) ? t_s1 : t_s0) + lane_off, sv);
-            tmem_ld32(((j & 1) ? t_s1 : t_s0) + lane_off + 32, sv + 32);
+            float sv[32];
+            tmem_ld32(((j & 1) ? t_s1 : t_s0) + lane_off + 32 * hf, sv);
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_S_EMPTY + st]));
 
-            // mask bits of keys 64j .. 64j + 63 for this row
-            const int64_t k0 = (int64_t)j * BN;
-            uint32_t w0 = 0, w1 = 0;
-            if (row_ok) {
-                if (DENSE) {
-                    const int64_t lim = i - k0;  // keys k0 .. i are kept
-                    w0 = lim >= 31 ? 0xFFFFFFFFu : (lim < 0 ? 0u : ((2u << lim) - 1u));
-                    const int64_t lim1 = lim - 32;
-                    w1 = lim1 >= 31 ? 0xFFFFFFFFu : (lim1 < 0 ? 0u : ((2u << lim1) - 1u));
-                } else {
-                    const int64_t wd = k0 >> 5;
-                    if (wd <= last_word) w0 = bm[wd];
-                    if (wd + 1 <= last_word) w1 = bm[wd + 1];
-                }
-            }
-            float mx = -INFINITY;
+            // mask, scale, partial row max as a tree, then the full row max with the partner
 #pragma unroll
-            for (int c = 0; c < BN; ++c) {
-                const uint32_t bit = (c < 32 ? (w0 >> c) : (w1 >> (c - 32))) & 1u;
-                sv[c] = bit ? sv[c] * sc : -INFINITY;
-                mx = fmaxf(mx, sv[c]);
-            }
-            // P of the previous tile has been consumed and O is settled
-            if (j >= 1) {
-                ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&bars[B_PV_DONE]), (j - 1) & 1));
-                if (!ok) break;
-                tc_fence_after();
-            }
-            // Lazy rescale: a row rescales O only when its max grows by more than 2^8. The
-            // TMEM loads / stores are warp-collective (.sync.aligned), so the whole warp runs
-            // them when any of its rows needs it; the other rows multiply by 1.
+            for (int c = 0; c < 32; ++c) sv[c] = ((cw >> c) & 1u) ? sv[c] * sc : -INFINITY;
+            cw = nw;
+            float mx4[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                mx4[e] = fmaxf(fmaxf(fmaxf(sv[e], sv[e + 4]), fmaxf(sv[e + 8], sv[e + 12])),
+                               fmaxf(fmaxf(sv[e + 16], sv[e + 20]), fmaxf(sv[e + 24], sv[e + 28])));
+            const float pm = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+            float om;
+            ok = exchange(j, pm, om);
+            if (!ok) break;
+            const float mx = fmaxf(pm, om);
+            // Lazy rescale: a row rescales O only when its max grows by more than 2^8 (both
+            // halves see the same max and decide alike). The TMEM loads / stores are
+            // warp-collective (.sync.aligned), so the whole warp runs them when any of its rows
+            // needs it; the other rows multiply by 1.
             const bool upd = mx > m_used + 8.f;
             const float al = upd ? (m_used == -INFINITY ? 0.f : exp2f(m_used - mx)) : 1.f;
             if (upd) {
                 l *= al;
                 m_used = mx;
             }
-            if (__any_sync(0xFFFFFFFFu, upd)) {
+            if (__any_sync(0xFFFFFFFFu, upd && al != 0.f)) {
+                // O must have settled: the value product of tile j - 1 has to be done
+                if (j >= 1) {
+                    ok = __all_sync(0xFFFFFFFFu,
+                                    mbar_wait(smem_u32(&bars[B_PV_DONE + ((j - 1) & 1)]), ((j - 1) >> 1) & 1));
+                    if (!ok) break;
+                }
+                tc_fence_after();
                 float ov[32];
 #pragma unroll
-                for (int c4 = 0; c4 < DT / 32; ++c4) {
-                    tmem_ld32(t_o + lane_off + 32 * c4, ov);
+                for (int c4 = 0; c4 < 2; ++c4) {
+                    tmem_ld32(t_o + lane_off + 64 * hf + 32 * c4, ov);
 #pragma unroll
                     for (int c = 0; c < 32; ++c) ov[c] *= al;
-                    tmem_st32(t_o + lane_off + 32 * c4, ov);
+                    tmem_st32(t_o + lane_off + 64 * hf + 32 * c4, ov);
                 }
             }
             const float mu = (m_used == -INFINITY) ? 0.f : m_used;
-            // P = exp2(s - m_used) in hi + lo, stored as the K-major 128-byte-swizzled A operand
+            // P = exp2(s - m_used) split as hi = p with its low 16 bits cleared (exactly a bf16)
+            // and lo = p - hi rounded to bf16 (p to ~16 significant bits with one conversion per
+            // pair), written into TMEM over this tile's score columns (both halves have read
+            // their scores: the max exchange came first) as the A operand of the value product
+            float lsum[4] = {0.f, 0.f, 0.f, 0.f};
+            uint32_t hw[16], lw[16];
 #pragma unroll
-            for (int c8 = 0; c8 < BN / 8; ++c8) {
-                uint32_t hw[4], lw[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float p0 = exp2f(sv[8 * c8 + 2 * e] - mu), p1 = exp2f(sv[8 * c8 + 2 * e + 1] - mu);
-                    l += p0 + p1;
-                    const float h0 = __bfloat162float(__float2bfloat16_rn(p0));
-                    const float h1 = __bfloat162float(__float2bfloat16_rn(p1));
-                    hw[e] = pack_bf16(h0, h1);
-                    lw[e] = pack_bf16(p0 - h0, p1 - h1);
-                }
-                const int chunk = (c8 ^ (r & 7)) << 4;
-                *reinterpret_cast<uint4 *>(prow_hi + chunk) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-                *reinterpret_cast<uint4 *>(prow_lo + chunk) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+            for (int w = 0; w < 16; ++w) {
+                const float p0 = exp2f(sv[2 * w] - mu), p1 = exp2f(sv[2 * w + 1] - mu);
+                lsum[w & 3] += p0 + p1;
+                const uint32_t b0 = __float_as_uint(p0), b1 = __float_as_uint(p1);
+                hw[w] = __byte_perm(b0, b1, 0x7632);
+                lw[w] = pack_bf16(p0 - __uint_as_float(b0 & 0xFFFF0000u), p1 - __uint_as_float(b1 & 0xFFFF0000u));
             }
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            l += (lsum[0] + lsum[1]) + (lsum[2] + lsum[3]);
+            const uint32_t pt = ((j & 1) ? t_s1 : t_s0) + lane_off;
+            tmem_st16(pt + 16 * hf, hw);
+            tmem_st16(pt + 32 + 16 * hf, lw);
             tc_fence_before();
-            mbar_arrive(smem_u32(&bars[B_P_FULL]));
+            mbar_arrive(smem_u32(&bars[B_P_FULL + st]));
         }
-        if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&bars[B_PV_DONE]), (n_kt - 1) & 1));
+        float ol = 0.f;
+        if (ok) ok = exchange(n_kt, l, ol);
+        if (ok)
+            ok = __all_sync(0xFFFFFFFFu,
+                            mbar_wait(smem_u32(&bars[B_PV_DONE + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1));
         if (ok) {
             tc_fence_after();
-            const float inv = l > 0.f ? 1.f / l : 0.f;
-            TOut *out = reinterpret_cast<TOut *>(a.out) + (((int64_t)s * a.N + (row_ok ? i : 0)) * a.Hq + h) * DT;
+            const float lt = l + ol;
+            const float inv = lt > 0.f ? 1.f / lt : 0.f;
+            TOut *out = reinterpret_cast<TOut *>(a.out) + (((int64_t)s * a.N + (row_ok ? i : 0)) * a.Hq + h) * DT + 64 * hf;
             float ov[32];
 #pragma unroll
-            for (int c4 = 0; c4 < DT / 32; ++c4) {
-                tmem_ld32(t_o + lane_off + 32 * c4, ov);
+            for (int c4 = 0; c4 < 2; ++c4) {
+                tmem_ld32(t_o + lane_off + 64 * hf + 32 * c4, ov);
                 if (row_ok) {
 #pragma unroll
                     for (int c = 0; c < 32; ++c) ov[c] *= inv;
@@ -462,8 +518,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, con
                     for (int e = 0; e < 4; ++e) store8<TOut>(out + 32 * c4 + 8 * e, ov + 8 * e);
                 }
             }
-            if (row_ok && a.lse != nullptr)
-                a.lse[((int64_t)s * a.Hq + h) * a.N + i] = (m_used + __log2f(l)) * kLn2;
+            if (row_ok && hf == 0 && a.lse != nullptr)
+                a.lse[((int64_t)s * a.Hq + h) * a.N + i] = (m_used + __log2f(lt)) * kLn2;
         }
     }
 
@@ -471,7 +527,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_attn_tile(const AttnArgs a, con
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 5)
+    if (warp == kMmaWarp)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
 }
 
@@ -505,7 +561,7 @@ bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows)
 }
 
 template <bool SPLIT, bool DENSE, typename TOut>
-cudaError_t launch_t(const AttnArgs &a, const TileMaps &maps, cudaStream_t s)
+cudaError_t launch_t(const AttnArgs &a, const TileMaps &maps, const void *q_hi, const void *q_lo, cudaStream_t s)
 {
     auto kern = k_attn_tile<SPLIT, DENSE, TOut>;
     static bool attr = false;
@@ -516,7 +572,7 @@ cudaError_t launch_t(const AttnArgs &a, const TileMaps &maps, cudaStream_t s)
     }
     const int64_t n_qt = (a.N + BM - 1) / BM;
     const unsigned grid = (unsigned)(n_qt * a.Hq * a.n_sets);
-    kern<<<grid, kThreads, SMEM_BYTES, s>>>(a, maps);
+    kern<<<grid, kThreads, SMEM_BYTES, s>>>(a, maps, q_hi, q_lo);
     note_launch();
     return cudaGetLastError();
 }
@@ -554,12 +610,12 @@ cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const voi
         maps.kl = maps.kh;
     }
     if (out_dtype == RIS_F32) {
-        if (split) return dense ? launch_t<true, true, float>(a, maps, s) : launch_t<true, false, float>(a, maps, s);
-        return dense ? launch_t<false, true, float>(a, maps, s) : launch_t<false, false, float>(a, maps, s);
+        if (split) return dense ? launch_t<true, true, float>(a, maps, q_hi, q_lo, s) : launch_t<true, false, float>(a, maps, q_hi, q_lo, s);
+        return dense ? launch_t<false, true, float>(a, maps, q_hi, q_lo, s) : launch_t<false, false, float>(a, maps, q_hi, q_lo, s);
     }
     if (split)
-        return dense ? launch_t<true, true, __nv_bfloat16>(a, maps, s) : launch_t<true, false, __nv_bfloat16>(a, maps, s);
-    return dense ? launch_t<false, true, __nv_bfloat16>(a, maps, s) : launch_t<false, false, __nv_bfloat16>(a, maps, s);
+        return dense ? launch_t<true, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s) : launch_t<true, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
+    return dense ? launch_t<false, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s) : launch_t<false, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
 }
 
 }  // namespace ris

@@ -640,6 +640,14 @@ ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches)
     return RIS_OK;
 }
 
+int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim)
+{
+    if (mask == nullptr || (dtype != RIS_F32 && dtype != RIS_BF16) || (head_dim != 64 && head_dim != 128)) return -1;
+    if (dtype == RIS_F32) return 3;
+    if (head_dim == 128 && use_tile_design(mask)) return 2;
+    return use_tma_gather() ? 1 : 0;
+}
+
 ris_status ris_device_status(void *stream)
 {
     unsigned int word = 0, tile_word = 0;

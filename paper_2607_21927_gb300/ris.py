@@ -87,6 +87,7 @@ _SIGS = {
                                      ctypes.c_void_p],
     "ris_kernel_timer_enable": [ctypes.c_int32],
     "ris_device_status": [ctypes.c_void_p],
+    "ris_attention_design": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32],
     "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
 }
 
@@ -121,6 +122,14 @@ def ris_launch_count() -> int:
 
 def ris_version() -> str:
     return lib().ris_version().decode()
+
+
+DESIGNS = {0: "register gather", 1: "TMA gather", 2: "tcgen05 masked tiles", 3: "fp32 gather"}
+
+
+def ris_attention_design(mask: "Mask", dtype=torch.bfloat16, head_dim: int = 128) -> int:
+    """Kernel design a layer call on this mask uses (see DESIGNS)."""
+    return int(lib().ris_attention_design(mask.handle, BF16 if dtype == torch.bfloat16 else F32, int(head_dim)))
 
 
 def ris_device_status(stream=None) -> None:
