@@ -1,22 +1,30 @@
 #!/usr/bin/env python3
 """Benchmark of RIS prefill sparse attention on GB300; prints one JSON line on rank 0.
 
-Workload (one step = one pass of the whole hot path over one batch of synthetic input):
-a Qwen2-1.5B-shaped prefill attention stack at N = 65536 tokens, 28 layers of (12 query
-heads, 2 KV heads, head_dim 128), bf16 Q/K/V ~ N(0, 1) with 1% outlier channels scaled x8
-(layer L drawn from seed L), RoPE theta 1e6 with YaRN extension (s = 65536 / 32768 = 2),
-run once in Stochastic Mode and once in Structural Mode, each at density 1% with 10
-ensemble seeds. Each mode builds its master mask once (all seeds OR-merged) and runs the
-28 layers on it: RoPE of q and k, masked QK^T, one softmax per row, PV.
+Default workload (C5; one step = one pass of the whole hot path over one batch of synthetic
+input): a Qwen2-1.5B-shaped prefill attention stack at N = 65536 tokens, 28 layers of (12
+query heads, 2 KV heads, head_dim 128), bf16 Q/K/V ~ N(0, 1) with 1% outlier channels scaled
+x8 (layer L drawn from seed L), RoPE theta 1e6 with YaRN extension (s = 65536 / 32768 = 2),
+run once in Stochastic Mode and once in Structural Mode, each at density 1% with 10 ensemble
+seeds. Each run builds its master mask once (all seeds OR-merged) and runs the layers on it:
+RoPE of q and k, masked QK^T, one softmax per row, PV. --workload selects the other
+evaluation shapes (C1 .. C4c, one layer shape each, with enough distinct layers per step that
+the inputs of a step exceed L2).
 
-value      = sampled pair-heads per second over the whole job (all ranks): for each mode
-             28 * (pairs of the master mask) * 12 query heads, per step.
-e2e        = the same metric through the C ABI with host buffers: per step the 28 layers'
-             q/k/v are copied from pinned host memory and all outputs copied back, the copies
+value      = sampled pair-heads per second over the whole job (all ranks): for each run
+             layers * (pairs of the master mask) * query heads, per step.
+e2e        = the same metric through the C ABI with host buffers: per step every layer's
+             q/k/v is copied from pinned host memory and all outputs copied back, the copies
              overlapped with the compute on two copy streams.
-roofline   = the attention kernel's algorithmic gathered bytes (K and V rows of every sampled
-             pair, both KV heads: pairs * 2 * 2 * 128 * 2 B) per launch over its CUDA-event
-             duration, against the measured HBM copy bandwidth.
+mask_ms_per_step / attn_ms_per_layer
+           = the mask builds of a step (CUDA events around each build inside the timed region)
+             and the rest of the step per layer (RoPE + attention), so that the per-layer cost
+             is reported with the mask build amortised separately.
+roofline   = the dominant attention kernel: for the gathering designs its algorithmic bytes
+             (K and V rows of every sampled pair, all KV heads) per launch over the mean
+             CUDA-event launch time against the measured HBM copy bandwidth, and against this
+             library's L2 row-gather probe; for the tcgen05 tile design its algorithmic FLOPs
+             (4 * head_dim per sampled pair-head) against the measured sustained bf16 peak.
 
 --impl reference times the fp64 CPU oracle on the host cores on a bounded sample of the
 same workload (its own sample of rows per step) and prints the same line.
@@ -38,7 +46,29 @@ if ROOT not in sys.path:
 
 METRIC = "sampled attention pairs/s and ms/layer at N=32k/64k, 1% density; % of roofline"
 UNIT = "pair-heads/s"
-MODES = (("stochastic", 0), ("structural", 1))
+L2_FLUSH_BYTES = 256 << 20  # distinct per-layer inputs of at least this size, so each layer starts cold in L2
+
+# Workloads (names follow the configuration table of the method's evaluation shapes). Each run
+# is (name, mode, density, n_seeds): one master mask built per run, every layer attended on it.
+# Qwen2-1.5B shape: 12 query heads, 2 KV heads, head_dim 128, theta 1e6, native 32768 tokens;
+# TinyLlama shape: 32 / 4 / 64, theta 1e4, native 2048 tokens.
+WORKLOADS = {
+    "C1": dict(N=2048, layers=0, Hq=1, Hkv=1, D=128, dtype="f32", outliers=False, rope=("plain", 1e6, 32768),
+               runs=[("stochastic", 0, 0.05, 1)], title="single-head fp32 attention, N=2048"),
+    "C2": dict(N=8192, layers=0, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+               runs=[("stochastic", 0, 0.01, 10)], title="Qwen2-1.5B-shaped attention layer, N=8192"),
+    "C3": dict(N=16384, layers=0, Hq=32, Hkv=4, D=64, dtype="bf16", outliers=False, rope=("yarn", 1e4, 2048),
+               runs=[("structural", 1, 0.01, 10)], title="TinyLlama-shaped attention layer, N=16384, YaRN s=8"),
+    "C4a": dict(N=32768, layers=0, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+                runs=[("stochastic", 0, 0.01, 70)], title="Qwen2-1.5B-shaped attention layer, N=32768"),
+    "C4b": dict(N=32768, layers=0, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+                runs=[("stochastic", 0, 0.05, 10)], title="Qwen2-1.5B-shaped attention layer, N=32768"),
+    "C4c": dict(N=32768, layers=0, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+                runs=[("dense", 2, 1.0, 1)], title="Qwen2-1.5B-shaped attention layer, N=32768, dense causal"),
+    "C5": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+               runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)],
+               title="Qwen2-1.5B-shaped prefill attention stack, N=65536, 28 layers, YaRN s=2"),
+}
 
 
 def parse_args():
@@ -47,25 +77,53 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--N", type=int, default=65536)
-    ap.add_argument("--layers", type=int, default=28)
-    ap.add_argument("--seeds", type=int, default=10)
-    ap.add_argument("--density", type=float, default=0.01)
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="C5")
+    ap.add_argument("--N", type=int, default=None, help="override the workload's token count")
+    ap.add_argument("--layers", type=int, default=None, help="override the number of layers per step")
+    ap.add_argument("--seeds", type=int, default=None, help="override the ensemble size of every run")
+    ap.add_argument("--density", type=float, default=None, help="override the density of every sparse run")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end measurement")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle CPU baseline")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle seconds per mode")
-    return ap.parse_args()
+    ap.add_argument("--no-probes", action="store_true", help="skip the L2 / FFMA ceiling probes")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle seconds per step")
+    a = ap.parse_args()
+    w = dict(WORKLOADS[a.workload])
+    w["name"] = a.workload
+    if a.N is not None:
+        w["N"] = a.N
+    runs = []
+    for name, mode, dens, ns in w["runs"]:
+        if mode != 2:
+            dens = a.density if a.density is not None else dens
+            ns = a.seeds if a.seeds is not None else ns
+        runs.append((name, mode, dens, ns))
+    w["runs"] = runs
+    e = 4 if w["dtype"] == "f32" else 2
+    per_layer = w["N"] * (w["Hq"] + 2 * w["Hkv"]) * w["D"] * e
+    if a.layers is not None:
+        w["layers"] = a.layers
+    elif w["layers"] == 0:
+        w["layers"] = max(1, -(-L2_FLUSH_BYTES // per_layer))
+    a.w = w
+    return a
 
 
 def workload_config(a):
+    w = a.w
+    e = 4 if w["dtype"] == "f32" else 2
+    per_layer = w["N"] * (w["Hq"] + 2 * w["Hkv"]) * w["D"] * e
+    kind, theta, native = w["rope"]
+    runs = ", ".join(f"{n}" + ("" if m == 2 else f" {d:g} x {s} seeds") for n, m, d, s in w["runs"])
     return {
-        "workload": f"Qwen2-1.5B-shaped prefill attention stack, N={a.N}, {a.layers} layers x (12 q heads, "
-                    f"2 KV heads, head_dim 128), YaRN RoPE theta 1e6 (native 32768), Stochastic and Structural "
-                    f"modes at {a.density:g} density x {a.seeds} seeds",
-        "N": a.N, "layers": a.layers, "heads": 12, "kv_heads": 2, "head_dim": 128,
-        "rope": "yarn", "rope_theta": 1e6, "native_len": 32768, "modes": [m for m, _ in MODES],
-        "density": a.density, "seeds": a.seeds, "input_dtype": "bf16", "outlier_channels": "1% x8",
-        "l2": "inputs larger than L2 (each layer's q/k/v is 268 MB; layers use distinct buffers)",
+        "workload": f"{w['name']}: {w['title']} ({w['Hq']} q heads, {w['Hkv']} KV heads, head_dim {w['D']}, "
+                    f"{w['dtype']}{' with 1% x8 outlier channels' if w['outliers'] else ''}), {kind} RoPE "
+                    f"theta {theta:g} native {native}; runs: {runs}; {w['layers']} layer(s) per run per step",
+        "name": w["name"], "N": w["N"], "layers": w["layers"], "heads": w["Hq"], "kv_heads": w["Hkv"],
+        "head_dim": w["D"], "rope": kind, "rope_theta": theta, "native_len": native,
+        "runs": [{"name": n, "mode": m, "density": d, "seeds": s} for n, m, d, s in w["runs"]],
+        "input_dtype": w["dtype"], "outlier_channels": "1% x8" if w["outliers"] else None,
+        "l2": (f"inputs larger than L2: each layer has its own q/k/v ({per_layer / 2**20:.0f} MiB), "
+               f"{w['layers']} layers = {w['layers'] * per_layer / 2**20:.0f} MiB per run"),
     }
 
 
@@ -170,14 +228,26 @@ class ClockSampler:
 
 
 # ----------------------------------------------------------------------------- CPU oracle sample
-def oracle_sample(q_host, k_host, v_host, N, mode, density, seeds, target_s, rng_seed):
+ROPE_KINDS = {"none": 0, "plain": 1, "linear": 2, "yarn": 3}
+
+
+def oracle_rope(w):
+    import oracle
+
+    kind, theta, native = w["rope"]
+    return oracle.RopeCfg(kind=ROPE_KINDS[kind], theta=theta, native_len=native)
+
+
+def oracle_sample(q_host, k_host, v_host, w, run, target_s, rng_seed):
     """Time the fp64 oracle on a random sample of rows of one layer; returns (pair-heads, seconds, rows)."""
     import numpy as np
 
     import oracle
 
-    spec = oracle.MaskSpec(N=N, mode=mode, density=density, seeds=seeds)
-    cfg = oracle.RopeCfg(kind=oracle.ROPE_YARN, theta=1e6, native_len=32768)
+    N = w["N"]
+    name, mode, density, n_seeds = run
+    spec = oracle.MaskSpec(N=N, mode=mode, density=density, seeds=list(range(n_seeds)))
+    cfg = oracle_rope(w)
     rng = np.random.default_rng(rng_seed)
     nrows, total_ph, total_t, used = 8, 0, 0.0, 0
     while total_t < target_s and nrows <= N:
@@ -195,28 +265,32 @@ def oracle_sample(q_host, k_host, v_host, N, mode, density, seeds, target_s, rng
     return total_ph, total_t, used
 
 
-def host_qkv(N, layer, device):
+def host_qkv(w, layer, device):
     import torch
 
     from paper_2607_21927_gb300 import inputs
 
-    q, k, v = inputs.make_qkv(N, 12, 2, 128, dtype=torch.bfloat16, seed=layer, outliers=True, device=device)
+    dt = torch.float32 if w["dtype"] == "f32" else torch.bfloat16
+    q, k, v = inputs.make_qkv(w["N"], w["Hq"], w["Hkv"], w["D"], dtype=dt, seed=layer, outliers=w["outliers"],
+                              device=device)
     return [t.float().cpu().numpy().astype("float64") for t in (q, k, v)]
 
 
 def cpu_baseline(a, device):
     import oracle
 
+    w = a.w
     threads = os.cpu_count() or 1
     oracle.set_threads(threads)
-    qn, kn, vn = host_qkv(a.N, 0, device)
+    qn, kn, vn = host_qkv(w, 0, device)
     ph, secs, rows = 0, 0.0, 0
-    for name, mode in MODES:
-        p, t, r = oracle_sample(qn, kn, vn, a.N, mode, a.density, list(range(a.seeds)), a.cpu_seconds, 1234 + mode)
+    for ri, run in enumerate(w["runs"]):
+        p, t, r = oracle_sample(qn, kn, vn, w, run, a.cpu_seconds / len(w["runs"]), 1234 + ri)
         ph, secs, rows = ph + p, secs + t, rows + r
     return {"value": ph / secs, "unit": UNIT, "cores": oracle.get_threads(), "kind": "oracle",
-            "sample": f"layer 0, {rows} random query rows (both modes), whole path per row: mask row, RoPE, "
-                      f"masked softmax attention over all 12 heads; {ph} pair-heads in {secs:.1f} s"}
+            "sample": f"layer 0, {rows} random query rows (over {len(w['runs'])} run(s)), whole path per row: "
+                      f"mask row, RoPE, masked softmax attention over all {w['Hq']} heads; {ph} pair-heads in "
+                      f"{secs:.1f} s"}
 
 
 # ----------------------------------------------------------------------------- reference arm
@@ -225,20 +299,21 @@ def run_reference(a, rank):
         return
     import oracle
 
+    w = a.w
     threads = os.cpu_count() or 1
     oracle.set_threads(threads)
-    qn, kn, vn = host_qkv(a.N, 0, "cpu")
+    qn, kn, vn = host_qkv(w, 0, "cpu")
     per_step = max(2.0, a.cpu_seconds / 2)
-    for w in range(a.warmup):
-        for name, mode in MODES:
-            oracle_sample(qn, kn, vn, a.N, mode, a.density, list(range(a.seeds)), 0.5, 99 + w)
+    for s in range(a.warmup):
+        for ri, run in enumerate(w["runs"]):
+            oracle_sample(qn, kn, vn, w, run, 0.5, 99 + s)
     ph, secs, rows = 0, 0.0, 0
     for s in range(a.steps):
-        for name, mode in MODES:
-            p, t, r = oracle_sample(qn, kn, vn, a.N, mode, a.density, list(range(a.seeds)), per_step / 2, 7 * s + mode)
+        for ri, run in enumerate(w["runs"]):
+            p, t, r = oracle_sample(qn, kn, vn, w, run, per_step / len(w["runs"]), 7 * s + ri)
             ph, secs, rows = ph + p, secs + t, rows + r
     value = ph / secs
-    sample = (f"per step: random query rows of layer 0 in both modes, whole path per row; {rows} rows, "
+    sample = (f"per step: random query rows of layer 0 in every run, whole path per row; {rows} rows, "
               f"{ph} pair-heads in {secs:.1f} s over {a.steps} steps")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": a.gpus,
             "steps": a.steps, "warmup": a.warmup, "ms_per_step": 1e3 * secs / a.steps, "higher_is_better": True,
@@ -267,6 +342,29 @@ def recorded_traffic(kernel_file: str):
 
 
 # ----------------------------------------------------------------------------- our arm
+def ceilings(ris, w, no_probes):
+    """Peaks: MEASURED_PEAKS.json (HBM copy, bf16 GEMM) plus this library's L2 and FFMA probes."""
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        pass
+    c = {"hbm_gbs": peaks.get("hbm_gbs") or 6800.0, "hbm_source": "measured" if peaks.get("hbm_gbs") else "fallback",
+         "tc_tflops": peaks.get("bf16_tflops_sustained") or 1700.0,
+         "tc_source": "measured sustained bf16" if peaks.get("bf16_tflops_sustained") else "fallback",
+         "tc_burst_tflops": peaks.get("bf16_tflops") or 1900.0}
+    c["l2_bytes"] = ris.ris_probe_l2_bytes()
+    if not no_probes:
+        e = 4 if w["dtype"] == "f32" else 2
+        # the gather kernels' working set: rotated K (hi and lo for bf16) and V of one layer
+        kv_set = w["N"] * w["Hkv"] * w["D"] * e * (3 if e == 2 else 2)
+        c["l2_stream_gbs"] = ris.ris_probe_l2_read(64 << 20, 0)
+        c["l2_rows_gbs"] = ris.ris_probe_l2_read(max(1 << 20, min(kv_set, c["l2_bytes"] * 3 // 4)), 1)
+        c["l2_rows_set_bytes"] = max(1 << 20, min(kv_set, c["l2_bytes"] * 3 // 4))
+        c["ffma_tflops"] = ris.ris_probe_ffma()
+    return c
+
+
 def main():
     a = parse_args()
     rank, world, dist = dist_init()
@@ -278,33 +376,46 @@ def main():
 
     from paper_2607_21927_gb300 import inputs, ris
 
+    w = a.w
     dev = torch.device("cuda", torch.cuda.current_device())
-    N, L, Hq, Hkv, D = a.N, a.layers, 12, 2, 128
-    seeds = list(range(a.seeds))
-    rope = ris.rope_cfg(ris.ROPE_YARN, 1e6, 32768)
+    N, L, Hq, Hkv, D = w["N"], w["layers"], w["Hq"], w["Hkv"], w["D"]
+    tdt = torch.float32 if w["dtype"] == "f32" else torch.bfloat16
+    e = 4 if w["dtype"] == "f32" else 2
+    runs = w["runs"]
+    kind, theta, native = w["rope"]
+    rope = ris.rope_cfg(ROPE_KINDS[kind], theta, native)
 
     # inputs resident in HBM: one (q, k, v) per layer, layer L drawn from seed L
     qs, ks, vs = [], [], []
     for layer in range(L):
-        q, k, v = inputs.make_qkv(N, Hq, Hkv, D, dtype=torch.bfloat16, seed=layer, outliers=True, device=dev)
+        q, k, v = inputs.make_qkv(N, Hq, Hkv, D, dtype=tdt, seed=layer, outliers=w["outliers"], device=dev)
         qs.append(q)
         ks.append(k)
         vs.append(v)
-    outs = [[torch.empty(N, Hq, D, dtype=torch.bfloat16, device=dev) for _ in range(L)] for _ in MODES]
+    outs = [[torch.empty(N, Hq, D, dtype=tdt, device=dev) for _ in range(L)] for _ in runs]
     stream = torch.cuda.current_stream()
     pairs, design = {}, {}
+    mask_events = []  # (start, end) around each mask build while `timing` is set
+    timing = [False]
 
     def step():
-        for mi, (name, mode) in enumerate(MODES):
-            m = ris.ris_mask_generate(N, Hkv, mode, a.density, seeds)
+        for ri, (name, mode, dens, ns) in enumerate(runs):
+            if timing[0]:
+                mask_events.append((torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)))
+                mask_events[-1][0].record(stream)
+            m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)))
+            if timing[0]:
+                mask_events[-1][1].record(stream)
             pairs[name] = m.info().n_pairs
-            design[name] = ris.ris_attention_design(m, torch.bfloat16, D)
+            design[name] = ris.ris_attention_design(m, tdt, D)
             for layer in range(L):
-                ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[mi][layer])
+                ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[ri][layer])
             m.free()
 
     for _ in range(a.warmup):
         step()
+    torch.cuda.synchronize()
+    ceil = ceilings(ris, w, a.no_probes)
     torch.cuda.synchronize()
 
     # ---- device-timed region
@@ -312,77 +423,100 @@ def main():
 
     clocks_path = os.path.join(tempfile.gettempdir(), f"ris_bench_clocks_{os.getpid()}.csv")
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.reset_peak_memory_stats(dev)
+    ris.ris_memory_stats(reset_high_water=True)
     barrier(dist)
     torch.cuda.synchronize()
     ris.ris_kernel_timer_enable(True)
     n0 = ris.ris_launch_count()
     with ClockSampler(clocks_path) as clk:
+        timing[0] = True
         ev0.record(stream)
         for _ in range(a.steps):
             step()
         ev1.record(stream)
         torch.cuda.synchronize()
+        timing[0] = False
     launches = ris.ris_launch_count() - n0
     k_ms, k_n = ris.ris_kernel_timer_read()
     ris.ris_kernel_timer_enable(False)
     barrier(dist)
     elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1), dist)
+    lib_cur, lib_high = ris.ris_memory_stats()
+    torch_high = torch.cuda.max_memory_allocated(dev)
 
-    pair_heads_step = sum(pairs[name] for name, _ in MODES) * L * Hq
+    mask_ms = max_over_ranks(sum(e0.elapsed_time(e1) for e0, e1 in mask_events) / a.steps, dist)
+    total_pairs = sum(pairs.values())
+    pair_heads_step = total_pairs * L * Hq
     value = world * pair_heads_step * a.steps / (elapsed_ms / 1e3)
     ms_step = elapsed_ms / a.steps
 
     # roofline of the attention kernel over the timed region: algorithmic bytes (gather) or
     # algorithmic FLOPs (tiles) per launch / mean launch time
-    launches_per_step = len(MODES) * L
+    launches_per_step = len(runs) * L
     mean_launch_ms = k_ms / max(k_n, 1)
-    peaks = {}
-    try:
-        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
-    except Exception:
-        pass
-    hbm = peaks.get("hbm_gbs")
-    peak_note = "measured" if hbm else "fallback"
-    hbm = hbm or 6800.0
-    tc = peaks.get("bf16_tflops_sustained") or 1700.0
     kinds = sorted(set(design.values()))
+    hbm, tc = ceil["hbm_gbs"], ceil["tc_tflops"]
+    kv_row_bytes = Hkv * 2 * D * e  # K and V rows of one key, all KV heads
     if kinds == [2]:  # every launch on the tensor-core tile kernel
-        flops_per_launch = 4 * D * Hq * sum(pairs.values()) * L / launches_per_step
+        flops_per_launch = 4 * D * Hq * total_pairs * L / launches_per_step
         achieved = flops_per_launch / (mean_launch_ms / 1e3) / 1e12
+        dense_flops = sum((4 * D * Hq * N * (N + 1) / 2) for _ in runs) * L / launches_per_step
         roofline = {"bound": "tensor", "achieved": achieved, "peak": tc, "unit": "TFLOP/s", "frac": achieved / tc,
-                    "traffic": None, "kernel": "k_attn_tile (tcgen05 masked tiles)",
-                    "peak_source": ("measured sustained bf16" if peaks.get("bf16_tflops_sustained") else "fallback"),
+                    "traffic": None, "kernel": "k_attn_tile (tcgen05 masked tiles)", "peak_source": ceil["tc_source"],
                     "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
-                    "mean_launch_ms": mean_launch_ms, "launches_timed": k_n}
+                    "mean_launch_ms": mean_launch_ms, "launches_timed": k_n,
+                    "design_frac": (dense_flops / (tc * 1e12)) / (mean_launch_ms / 1e3),
+                    "design_note": "dense-causal tile FLOPs / sustained bf16 peak over the launch time (the "
+                                   "kernel issues 2.5x that in hi/lo split products)"}
     else:
-        bytes_per_step = sum(pairs[name] for name, _ in MODES) * L * Hkv * 2 * D * 2
-        achieved = (bytes_per_step / launches_per_step) / (mean_launch_ms / 1e3) / 1e9
+        bytes_per_launch = total_pairs * L * kv_row_bytes / launches_per_step
+        achieved = bytes_per_launch / (mean_launch_ms / 1e3) / 1e9
+        gather = {0: "k_attn_bf16 (register gather)", 1: "k_attn_tma (TMA gather4)", 3: "k_attn_f32 (fp32 gather)"}
         roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                    "traffic": recorded_traffic("attn_bf16.cu") if kinds == [0] else None,
-                    "kernel": "k_attn_bf16 (register gather)" if kinds == [0] else "mixed designs " + str(kinds),
-                    "peak_source": peak_note, "bytes": "algorithmic: K and V rows of every sampled pair, both KV heads",
+                    "traffic": recorded_traffic("attn_bf16.cu") if kinds == [0] and a.workload == "C5" else None,
+                    "kernel": gather.get(kinds[0], "?") if len(kinds) == 1 else "mixed designs " + str(kinds),
+                    "peak_source": ceil["hbm_source"],
+                    "bytes": "algorithmic: K and V rows of every sampled pair, all KV heads",
                     "mean_launch_ms": mean_launch_ms, "launches_timed": k_n}
-    # the sampled-pair roofline: max(sampled FLOPs / tensor peak, tile-reuse K/V bytes / HBM)
-    flops = 4 * D * Hq * sum(pairs.values()) * L
-    b_tile = len(MODES) * L * (N / 128) * (N / 2) * Hkv * 2 * D * 2
-    t_roof = max(flops / (tc * 1e12), b_tile / (hbm * 1e9))
+        if "l2_rows_gbs" in ceil:
+            roofline["l2_rows_peak"] = ceil["l2_rows_gbs"]
+            roofline["frac_of_l2_rows"] = achieved / ceil["l2_rows_gbs"]
+            roofline["l2_note"] = ("the K/V working set is L2-resident, so the gather is served from L2: "
+                                   "peak = this library's probe reading whole 256-byte rows at random indices "
+                                   f"over {ceil['l2_rows_set_bytes'] / 2**20:.0f} MiB")
+    # the sampled-pair roofline: max(sampled FLOPs / tensor peak, min(row, tile) K/V bytes / bandwidth)
+    flops = 4 * D * Hq * total_pairs * L
+    b_row = total_pairs * L * kv_row_bytes
+    b_tile = len(runs) * L * (N / 128) * (N / 2) * kv_row_bytes
+    in_l2 = N * kv_row_bytes < ceil["l2_bytes"]
+    bw = ceil.get("l2_stream_gbs", hbm) if in_l2 else hbm
+    t_roof = max(flops / (tc * 1e12), min(b_row, b_tile) / (bw * 1e9))
     clocks = clk.summary(getattr(torch.cuda.get_device_properties(dev), "pci_bus_id", None))
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps, "warmup": a.warmup,
-            "ms_per_step": ms_step, "ms_per_layer": ms_step / (len(MODES) * L), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "ms_per_step": ms_step, "ms_per_layer": ms_step / (len(runs) * L), "higher_is_better": True,
+            "mask_ms_per_step": mask_ms,
+            "attn_ms_per_layer": (ms_step - mask_ms) / (len(runs) * L),
+            "attn_pair_heads_per_s": world * pair_heads_step / ((ms_step - mask_ms) / 1e3),
+            "scaling": "weak", "vs_baseline": None, "dtype": w["dtype"], "data": "synthetic",
             "config": workload_config(a), "pairs_per_mask": pairs,
-            "design_per_mode": {k: ris.DESIGNS.get(v, v) for k, v in design.items()}, "roofline": roofline,
+            "design_per_run": {k: ris.DESIGNS.get(v, v) for k, v in design.items()}, "roofline": roofline,
             "pair_roofline": {"t_roof_ms_per_step": 1e3 * t_roof, "frac": 1e3 * t_roof / ms_step,
-                                    "formula": "max(4*D*Hq*pairs / bf16 sustained, (N/128)*(N/2)*Hkv*2*D*2 B / HBM)"},
-            "clocks": clocks, "gpu_launches": launches}
+                              "bandwidth": ("L2 stream probe" if in_l2 and "l2_stream_gbs" in ceil else "HBM"),
+                              "formula": "max(4*D*Hq*pairs / bf16 sustained, min(pairs, (N/128)*(N/2)) * "
+                                         "Hkv*2*D*e / bandwidth)"},
+            "ceilings": ceil, "clocks": clocks, "gpu_launches": launches,
+            "memory": {"library_pool_high_water_bytes": lib_high, "torch_max_allocated_bytes": torch_high,
+                       "note": "torch holds every layer's inputs and outputs resident; the library's high-water "
+                               "mark is its masks plus per-call scratch"}}
 
     # ---- end to end through the C ABI with host buffers
     if not a.no_e2e:
         hq = [t.cpu().pin_memory() for t in qs]
         hk = [t.cpu().pin_memory() for t in ks]
         hv = [t.cpu().pin_memory() for t in vs]
-        ho = [[torch.empty(N, Hq, D, dtype=torch.bfloat16).pin_memory() for _ in range(L)] for _ in MODES]
+        ho = [[torch.empty(N, Hq, D, dtype=tdt).pin_memory() for _ in range(L)] for _ in runs]
         h2d = sum(t.numel() * t.element_size() for t in hq + hk + hv)
         d2h = sum(t.numel() * t.element_size() for row in ho for t in row)
 
@@ -391,8 +525,8 @@ def main():
         h2d_s, d2h_s = torch.cuda.Stream(), torch.cuda.Stream()
         in_ready = [torch.cuda.Event() for _ in range(L)]
         layer_free = [torch.cuda.Event() for _ in range(L)]
-        out_ready = [[torch.cuda.Event() for _ in range(L)] for _ in MODES]
-        out_free = [[torch.cuda.Event() for _ in range(L)] for _ in MODES]
+        out_ready = [[torch.cuda.Event() for _ in range(L)] for _ in runs]
+        out_free = [[torch.cuda.Event() for _ in range(L)] for _ in runs]
         first = [True]
 
         def e2e_step():
@@ -404,20 +538,20 @@ def main():
                     ks[layer].copy_(hk[layer], non_blocking=True)
                     vs[layer].copy_(hv[layer], non_blocking=True)
                     in_ready[layer].record(h2d_s)
-            for mi, (name, mode) in enumerate(MODES):
-                m = ris.ris_mask_generate(N, Hkv, mode, a.density, seeds)
+            for ri, (name, mode, dens, ns) in enumerate(runs):
+                m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)))
                 for layer in range(L):
                     stream.wait_event(in_ready[layer])
                     if not first[0]:
-                        stream.wait_event(out_free[mi][layer])
-                    ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[mi][layer])
-                    out_ready[mi][layer].record(stream)
-                    if mi == len(MODES) - 1:
+                        stream.wait_event(out_free[ri][layer])
+                    ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[ri][layer])
+                    out_ready[ri][layer].record(stream)
+                    if ri == len(runs) - 1:
                         layer_free[layer].record(stream)
                     with torch.cuda.stream(d2h_s):
-                        d2h_s.wait_event(out_ready[mi][layer])
-                        ho[mi][layer].copy_(outs[mi][layer], non_blocking=True)
-                        out_free[mi][layer].record(d2h_s)
+                        d2h_s.wait_event(out_ready[ri][layer])
+                        ho[ri][layer].copy_(outs[ri][layer], non_blocking=True)
+                        out_free[ri][layer].record(d2h_s)
                 m.free()
             first[0] = False
 

@@ -231,6 +231,35 @@ int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim);
  * undefined. Blocks. Errors: RIS_ERR_CUDA. */
 ris_status ris_device_status(void *stream);
 
+/* ---- Measurement support (the paper has no counterpart) -------------------------------------
+ * Small kernels that measure the ceilings the attention kernels are compared against, for the
+ * current device. Each allocates its own device buffers, runs on `stream` (NULL: legacy default
+ * stream), synchronises it and frees what it allocated; none belongs on a hot path.
+ *
+ * ris_probe_l2_read: read bandwidth in GB/s (1e9 B/s) over a device buffer of `working_set`
+ * bytes (1 MiB .. 4 GiB, rounded down to 256 B) that is read repeatedly, best of five launches
+ * after one untimed launch. pattern 0: every thread streams 16-byte loads with a grid-wide
+ * stride; pattern 1: groups of 16 threads read whole 256-byte rows at pseudo-random row
+ * indices (the access pattern of the row-gathering attention kernels). Both load with .cg
+ * (cached in L2 only), so a working set below the L2 size measures L2 and one well above it
+ * measures HBM. Errors: RIS_ERR_INVALID (NULL gbs, size or pattern out of range), RIS_ERR_CUDA.
+ *
+ * ris_probe_ffma: FP32 fused multiply-add throughput in TFLOP/s (2 FLOPs per FFMA), eight
+ * independent chains per thread, four 512-thread blocks per SM. Errors: RIS_ERR_INVALID,
+ * RIS_ERR_CUDA.
+ *
+ * ris_probe_l2_bytes: L2 size in bytes as the driver reports it (cudaDevAttrL2CacheSize).
+ *
+ * ris_memory_stats: bytes in use now and the high-water mark of the current device's default
+ * stream-ordered memory pool, from which this library takes its masks and per-call scratch
+ * (the allocation-free entry point's fixed scratch is not counted). Other users of that pool
+ * in the same process are counted too. reset_high_water != 0 resets the mark to zero after
+ * reading it. Errors: RIS_ERR_INVALID (NULL outputs), RIS_ERR_CUDA. */
+ris_status ris_probe_l2_read(int64_t working_set, int32_t pattern, double *gbs, void *stream);
+ris_status ris_probe_ffma(double *tflops, void *stream);
+ris_status ris_probe_l2_bytes(int64_t *bytes);
+ris_status ris_memory_stats(int64_t *in_use, int64_t *high_water, int32_t reset_high_water);
+
 /* Text of the calling thread's last error ("" if none). The string is owned by the library. */
 const char *ris_last_error(void);
 

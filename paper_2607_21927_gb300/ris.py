@@ -89,6 +89,10 @@ _SIGS = {
     "ris_device_status": [ctypes.c_void_p],
     "ris_attention_design": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32],
     "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
+    "ris_probe_l2_read": [ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p],
+    "ris_probe_ffma": [ctypes.c_void_p, ctypes.c_void_p],
+    "ris_probe_l2_bytes": [ctypes.c_void_p],
+    "ris_memory_stats": [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32],
 }
 
 
@@ -146,6 +150,37 @@ def ris_kernel_timer_read():
     ms, n = ctypes.c_double(), ctypes.c_int64()
     _check("ris_kernel_timer_read", lib().ris_kernel_timer_read(ctypes.byref(ms), ctypes.byref(n)))
     return ms.value, n.value
+
+
+def ris_probe_l2_read(working_set: int, pattern: int = 0, stream=None) -> float:
+    """Measured read bandwidth (GB/s) over a `working_set`-byte buffer: pattern 0 streaming
+    16-byte loads, 1 whole 256-byte rows at pseudo-random indices."""
+    g = ctypes.c_double()
+    _check("ris_probe_l2_read", lib().ris_probe_l2_read(int(working_set), int(pattern), ctypes.byref(g),
+                                                        _stream(stream)))
+    return g.value
+
+
+def ris_probe_ffma(stream=None) -> float:
+    """Measured FP32 FFMA throughput (TFLOP/s)."""
+    t = ctypes.c_double()
+    _check("ris_probe_ffma", lib().ris_probe_ffma(ctypes.byref(t), _stream(stream)))
+    return t.value
+
+
+def ris_probe_l2_bytes() -> int:
+    """L2 size in bytes as the driver reports it."""
+    b = ctypes.c_int64()
+    _check("ris_probe_l2_bytes", lib().ris_probe_l2_bytes(ctypes.byref(b)))
+    return b.value
+
+
+def ris_memory_stats(reset_high_water: bool = False):
+    """(bytes in use, high-water mark) of the default stream-ordered pool the library allocates from."""
+    cur, high = ctypes.c_int64(), ctypes.c_int64()
+    _check("ris_memory_stats", lib().ris_memory_stats(ctypes.byref(cur), ctypes.byref(high),
+                                                      int(bool(reset_high_water))))
+    return cur.value, high.value
 
 
 def _check(name: str, st: int) -> None:
