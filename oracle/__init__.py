@@ -121,7 +121,7 @@ class _Spec(ctypes.Structure):
         ("n_anchor", ctypes.c_int32),
         ("head_key", ctypes.c_uint32),
         ("layer_key", ctypes.c_uint32),
-        ("pad_", ctypes.c_int32),
+        ("sampler", ctypes.c_int32),
     ]
 
 
@@ -138,6 +138,7 @@ class MaskSpec:
     n_anchor: int = 0
     head_key: int = 0
     layer_key: int = 0
+    sampler: int = 0  # 0: Bernoulli test per causal pair; 1: index draws with replacement
     _seeds_arr: np.ndarray = field(default=None, repr=False)
 
     def _c(self) -> _Spec:
@@ -145,7 +146,7 @@ class MaskSpec:
         return _Spec(
             int(self.N), int(self.mode), len(self.seeds), float(self.density),
             self._seeds_arr.ctypes.data, int(self.seed_index), int(self.local_window),
-            int(self.n_anchor), int(self.head_key), int(self.layer_key), 0,
+            int(self.n_anchor), int(self.head_key), int(self.layer_key), int(self.sampler),
         )
 
 

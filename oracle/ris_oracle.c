@@ -26,7 +26,14 @@
  *     number of causal clique pairs, d_global = max(0, d - d_clique);
  *   - the forced set of row i is the local window {i-W < j <= i} plus the anchors
  *     {j < A}; W >= 1 keeps the diagonal so no row is empty;
- *   - density 1 (or the dense mode) is every causal pair j <= i.
+ *   - density 1 (or the dense mode) is every causal pair j <= i;
+ *   - the index-draw sampler (the paper's torch.randint wording, Methods, "Memory-Bounded
+ *     Geometry Generation") replaces the per-pair Bernoulli test of the random part: row i
+ *     of seed s draws K indices with replacement, draw t being j_t = floor(u_t * N / 2^32)
+ *     with u_t word (t mod 4) of Philox4x32-10 with key (seed, head_key) and counter
+ *     (t/4, i, stream + 2, layer_key); draws with j_t < i are kept (causal filter) and
+ *     repeats merge (set semantics). K = floor(d N + 0.5) for Stochastic and
+ *     floor(d_global N + 0.5) for the Structural global part.
  */
 #include <math.h>
 #include <stdint.h>
@@ -133,14 +140,15 @@ typedef struct {
     int32_t n_anchor;     /* A >= 0 */
     uint32_t head_key;
     uint32_t layer_key;
-    int32_t pad_;
+    int32_t sampler; /* 0: Bernoulli test per causal pair; 1: index draws with replacement */
 } ora_mask_spec;
 
 typedef struct {
     int dense;
     uint32_t stream;
     uint64_t thr;
-    int64_t B; /* Structural block size, 0 for Stochastic */
+    int64_t B;     /* Structural block size, 0 for Stochastic */
+    int64_t draws; /* index draws per row and seed (sampler 1) */
 } mask_derived;
 
 static mask_derived derive(const ora_mask_spec *m)
@@ -155,10 +163,12 @@ static mask_derived derive(const ora_mask_spec *m)
         x.B = B;
         x.stream = 1;
         x.thr = ora_threshold(dg);
+        x.draws = (int64_t)floor(dg * (double)m->N + 0.5);
     } else {
         x.B = 0;
         x.stream = 0;
         x.thr = ora_threshold(m->density);
+        x.draws = (int64_t)floor(m->density * (double)m->N + 0.5);
     }
     return x;
 }
@@ -182,6 +192,7 @@ static int keep_pair(const ora_mask_spec *m, const mask_derived *x, int64_t i, i
     if (j > i - m->local_window) return 1;      /* local window, includes the diagonal */
     if (j < m->n_anchor) return 1;              /* global anchors over the first tokens */
     if (m->mode == 1 && (i / x->B) == (j / x->B)) return 1; /* Structural block clique */
+    if (m->sampler != 0) return 0; /* random part comes from the index draws */
     /* stochastic draws (Stochastic: whole budget; Structural: global remainder) */
     int s0 = m->seed_index < 0 ? 0 : m->seed_index;
     int s1 = m->seed_index < 0 ? m->n_seeds : m->seed_index + 1;
@@ -191,6 +202,30 @@ static int keep_pair(const ora_mask_spec *m, const mask_derived *x, int64_t i, i
     return 0;
 }
 
+/* Index-draw sampler: mark hit[j] = 1 for every j < i drawn for row i by the selected seeds. */
+static void row_draws(const ora_mask_spec *m, const mask_derived *x, int64_t i, unsigned char *hit)
+{
+    int s0 = m->seed_index < 0 ? 0 : m->seed_index;
+    int s1 = m->seed_index < 0 ? m->n_seeds : m->seed_index + 1;
+    for (int s = s0; s < s1; ++s) {
+        for (int64_t t = 0; t < x->draws; ++t) {
+            uint32_t ctr[4] = {(uint32_t)(t / 4), (uint32_t)i, x->stream + 2, m->layer_key};
+            uint32_t key[2] = {m->seeds[s], m->head_key};
+            uint32_t out[4];
+            ora_philox4x32_10(ctr, key, out);
+            int64_t j = (int64_t)(((uint64_t)out[t % 4] * (uint64_t)m->N) >> 32);
+            if (j < i) hit[j] = 1;
+        }
+    }
+}
+
+/* Membership of keys 0..i of row i: keep[j] = 1 iff (i, j) is in the mask. */
+static void row_members(const ora_mask_spec *m, const mask_derived *x, int64_t i, unsigned char *keep)
+{
+    for (int64_t j = 0; j <= i; ++j) keep[j] = (unsigned char)keep_pair(m, x, i, j);
+    if (m->sampler != 0 && !x->dense) row_draws(m, x, i, keep);
+}
+
 /* Number of kept keys of each requested row. */
 void ora_mask_counts(const ora_mask_spec *m, const int64_t *rows, int64_t nrows, int64_t *counts)
 {
@@ -198,7 +233,10 @@ void ora_mask_counts(const ora_mask_spec *m, const int64_t *rows, int64_t nrows,
 #pragma omp parallel for schedule(dynamic, 1)
     for (int64_t r = 0; r < nrows; ++r) {
         int64_t i = rows[r], c = 0;
-        for (int64_t j = 0; j <= i; ++j) c += keep_pair(m, &x, i, j);
+        unsigned char *keep = (unsigned char *)malloc((size_t)i + 1);
+        row_members(m, &x, i, keep);
+        for (int64_t j = 0; j <= i; ++j) c += keep[j];
+        free(keep);
         counts[r] = c;
     }
 }
@@ -211,8 +249,11 @@ void ora_mask_cols(const ora_mask_spec *m, const int64_t *rows, int64_t nrows, c
 #pragma omp parallel for schedule(dynamic, 1)
     for (int64_t r = 0; r < nrows; ++r) {
         int64_t i = rows[r], w = off[r];
+        unsigned char *keep = (unsigned char *)malloc((size_t)i + 1);
+        row_members(m, &x, i, keep);
         for (int64_t j = 0; j <= i; ++j)
-            if (keep_pair(m, &x, i, j)) cols[w++] = j;
+            if (keep[j]) cols[w++] = j;
+        free(keep);
     }
 }
 
@@ -226,9 +267,12 @@ void ora_mask_bits(const ora_mask_spec *m, const int64_t *rows, int64_t nrows, i
     for (int64_t r = 0; r < nrows; ++r) {
         int64_t i = rows[r];
         uint32_t *out = bits + r * words_per_row;
+        unsigned char *keep = (unsigned char *)malloc((size_t)i + 1);
+        row_members(m, &x, i, keep);
         memset(out, 0, sizeof(uint32_t) * (size_t)words_per_row);
         for (int64_t j = 0; j <= i && j / 32 < words_per_row; ++j)
-            if (keep_pair(m, &x, i, j)) out[j / 32] |= (uint32_t)1 << (j % 32);
+            if (keep[j]) out[j / 32] |= (uint32_t)1 << (j % 32);
+        free(keep);
     }
 }
 

@@ -405,3 +405,97 @@ def test_attention_with_rope_is_rope_then_attention(oracle):
     ref, ref_lse = _sdpa(qr, kr, v, oracle.mask_dense(spec), Hq // Hkv)
     np.testing.assert_allclose(out, ref[rows], rtol=1e-10, atol=1e-12)
     np.testing.assert_allclose(lse, ref_lse[rows], rtol=1e-12, atol=1e-12)
+
+
+# ----------------------------------------------------------------------------- index-draw sampler
+def _triton_philox(tmp_path, ctr, key):
+    n = len(ctr)
+    n2 = 1 << max(0, (n - 1).bit_length())  # the kernel's arange needs a power of two
+    ctr = np.concatenate([ctr, np.zeros((n2 - n, 4), np.uint32)])
+    key = np.concatenate([key, np.zeros((n2 - n, 2), np.uint32)])
+    inp, outp, script = tmp_path / "din.npz", tmp_path / "dout.npy", tmp_path / "dtp.py"
+    np.savez(inp, ctr=ctr, key=key)
+    script.write_text(_TRITON_PHILOX)
+    env = dict(os.environ, TRITON_INTERPRET="1")
+    subprocess.run([sys.executable, str(script), str(inp), str(outp)], check=True, env=env, timeout=300)
+    return np.load(outp)[:n]
+
+
+def test_draw_sampler_matches_triton_draws(oracle, tmp_path):
+    """Index-draw sampler (the torch.randint wording of Methods, Memory-Bounded Geometry
+    Generation): the rows' key sets are rebuilt here from draws made by Triton's independent
+    Philox (counter (t/4, i, stream+2, layer_key), key (seed, head_key), word t mod 4), mapped
+    to j = floor(u N / 2^32), causally filtered and merged, plus the forced diagonal and, for
+    Structural, the block clique."""
+    pytest.importorskip("triton")
+    N, seeds = 500, [3, 9]
+    rows = np.array([0, 1, 37, 250, 499], dtype=np.int64)
+    cases = [(oracle.MODE_STOCHASTIC, 0.04, 0, 0), (oracle.MODE_STRUCTURAL, 0.06, 2, 5)]
+    ctr, key, meta = [], [], []
+    for mode, d, hk, lk in cases:
+        if mode == oracle.MODE_STRUCTURAL:
+            g = oracle.structural(N, d)
+            K, stream = int(math.floor(g["d_global"] * N + 0.5)), 3
+        else:
+            K, stream = int(math.floor(d * N + 0.5)), 2
+        assert K > 0
+        for i in rows:
+            for s in seeds:
+                for t in range(K):
+                    ctr.append((t // 4, i, stream, lk))
+                    key.append((s, hk))
+                    meta.append((0, mode, int(i), t % 4))
+    ctr = np.array(ctr, dtype=np.uint32)
+    key = np.array(key, dtype=np.uint32)
+    words = _triton_philox(tmp_path, ctr, key)
+    u = words[np.arange(len(meta)), [m[3] for m in meta]].astype(np.uint64)
+    j = (u * np.uint64(N)) >> np.uint64(32)
+    for mode, d, hk, lk in cases:
+        spec = oracle.MaskSpec(N=N, mode=mode, density=d, seeds=seeds, head_key=hk, layer_key=lk, sampler=1)
+        off, cols = oracle.mask_cols(spec, rows)
+        B = oracle.structural(N, d)["B"] if mode == oracle.MODE_STRUCTURAL else None
+        for r, i in enumerate(rows):
+            sel = np.array([m[1] == mode and m[2] == i for m in meta])
+            want = {int(x) for x in j[sel] if x < i} | {int(i)}
+            if B is not None:
+                want |= set(range((i // B) * B, i + 1))
+            assert set(cols[off[r]:off[r + 1]].tolist()) == want, (mode, i)
+            assert (np.diff(cols[off[r]:off[r + 1]]) > 0).all()
+
+
+def test_draw_sampler_density(oracle):
+    """S seeds of K = round(dN) draws over [0, N): each earlier key of row i is hit with
+    probability q = 1 - (1 - 1/N)^(S K); the total kept count is within 5 sigma of q * sum(i)."""
+    N, d, S = 1000, 0.02, 5
+    spec = oracle.MaskSpec(N=N, mode=0, density=d, seeds=list(range(S)), sampler=1)
+    c = oracle.mask_counts(spec) - 1  # diagonal forced
+    K = int(math.floor(d * N + 0.5))
+    q = 1 - (1 - 1 / N) ** (S * K)
+    n = N * (N - 1) / 2
+    assert abs(c.sum() - q * n) < 5 * math.sqrt(n * q * (1 - q))
+    # uniform over key positions: early and late halves of the causal range are hit alike
+    m = oracle.mask_dense(spec)
+    low = np.tril(np.ones((N, N), bool), -1)
+    half = np.arange(N)[None, :] < (np.arange(N)[:, None] // 2)
+    a, b = m[low & half].mean(), m[low & ~half].mean()
+    assert abs(a - b) < 5 * math.sqrt(2 * q * (1 - q) / (low.sum() / 2))
+
+
+def test_draw_sampler_union_and_edges(oracle):
+    """Union over seeds is the OR of the per-seed draw masks; K = 0 leaves the forced set only;
+    density 1 is dense causal whatever the sampler."""
+    N, seeds = 300, [10, 20, 30]
+    for mode in (oracle.MODE_STOCHASTIC, oracle.MODE_STRUCTURAL):
+        u = oracle.mask_dense(oracle.MaskSpec(N=N, mode=mode, density=0.04, seeds=seeds, sampler=1))
+        per = [oracle.mask_dense(oracle.MaskSpec(N=N, mode=mode, density=0.04, seeds=seeds, seed_index=s,
+                                                 sampler=1)) for s in range(3)]
+        np.testing.assert_array_equal(u, per[0] | per[1] | per[2])
+        assert not (per[0] == per[1]).all()
+    m = oracle.mask_dense(oracle.MaskSpec(N=N, mode=0, density=0.001, seeds=[1], local_window=4, sampler=1))
+    i, j = np.indices((N, N))
+    np.testing.assert_array_equal(m, (j <= i) & (j > i - 4))
+    m = oracle.mask_dense(oracle.MaskSpec(N=N, mode=0, density=1.0, seeds=[1], sampler=1))
+    np.testing.assert_array_equal(m, np.tril(np.ones((N, N), bool)))
+    a = oracle.mask_dense(oracle.MaskSpec(N=N, mode=0, density=0.05, seeds=[1], sampler=1))
+    b = oracle.mask_dense(oracle.MaskSpec(N=N, mode=0, density=0.05, seeds=[1], sampler=0))
+    assert (a != b).any()
