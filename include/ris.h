@@ -65,6 +65,11 @@ typedef struct {
     int32_t n_anchor;     /* A >= 0: keys j < A always kept (global anchors, default 0) */
     int32_t per_head;     /* 0: one mask shared by all heads (default); 1: one mask per KV head */
     uint32_t layer_key;   /* mixed into every draw; 0 = shared across layers (default) */
+    int32_t sampler;      /* random part: 0 = Bernoulli keep test per causal pair (default);
+                             1 = index draws: per row and seed, `draws` indices j drawn with
+                             replacement uniformly over [0, N), kept when j < i, repeats merged
+                             (the torch.randint wording of Methods, "Memory-Bounded Geometry
+                             Generation") */
 } ris_mask_opts;
 
 /* Derived scalars of one call, resolved on the host. */
@@ -79,6 +84,8 @@ typedef struct {
     int32_t dense;           /* 1 when every causal pair is kept (dense mode or density 1) */
     double rope_factor;      /* resolved s */
     double rope_mscale;      /* 0.1 ln s + 1 for YaRN, else 1 */
+    int64_t draws;           /* index-draw sampler: draws per row and seed, floor(d N + 0.5) for
+                                Stochastic, floor(d_global N + 0.5) for Structural */
 } ris_params;
 
 /* Opaque handle to a mask held in device memory. */
@@ -126,7 +133,10 @@ ris_status ris_rope_freqs(const ris_rope_cfg *rope, int64_t N, int32_t head_dim,
 
 /* Build the RIS mask of N tokens (Methods, "Memory-Bounded Geometry Generation" and
  * "Sampling Modes"): for every seed, keep causal pair (i, j<i) iff Philox4x32-10 word
- * (j mod 4) of key (seed, head_key) and counter (j/4, i, stream, layer_key) is below thr;
+ * (j mod 4) of key (seed, head_key) and counter (j/4, i, stream, layer_key) is below thr
+ * (opts->sampler 0), or (sampler 1) iff j < i is one of the row's `draws` indices
+ * j_t = floor(u_t N / 2^32), u_t word (t mod 4) of key (seed, head_key) and counter
+ * (t/4, i, stream + 2, layer_key);
  * Structural adds the block cliques; the forced local window and anchors are added; with
  * per_seed = 0 all seeds are OR-merged into one master mask, with per_seed = 1 each seed
  * keeps its own mask. Output: bitmap + CSR in device memory owned by *out_mask.

@@ -8,6 +8,10 @@
 //   k_mask_bits : per (mask, row) CTA, per 32-key word: Philox4x32-10 draws of every seed
 //                 (8 calls = 32 keys per seed), OR, forced window/anchors, Structural
 //                 block clique, causal cut; writes the word and the row's key count.
+//   k_mask_draws: index-draw sampler only: per (mask, row) CTA, the row's index draws of
+//                 every seed (one Philox call = 4 draws), j = floor(u N / 2^32), kept when
+//                 j < i by an atomic OR into the zeroed bitmap row; k_mask_bits then ORs the
+//                 forced and clique keys into those words and counts the row.
 //   k_scan_*    : exclusive scan of the counts into row_ptr (int64).
 //   k_mask_fill : per (mask, row) CTA, expands the bitmap row into ascending key indices.
 //
@@ -77,7 +81,8 @@ __global__ void __launch_bounds__(kBitsThreads) k_mask_bits(const MaskBitsArgs a
     for (int64_t w = threadIdx.x; w < nw; w += kBitsThreads) {
         const int64_t j0 = w << 5;
         // forced keys: local window (i-W, i], anchors [0, A), Structural clique [blk0, i]
-        uint32_t bits = range_bits(j0, i - a.W + 1, i);
+        uint32_t bits = a.or_existing ? row[w] : 0u;
+        bits |= range_bits(j0, i - a.W + 1, i);
         bits |= range_bits(j0, 0, (int64_t)a.A - 1);
         bits |= range_bits(j0, blk0, i);
         const uint32_t causal = range_bits(j0, 0, i - 1);  // drawn pairs are j < i
@@ -116,6 +121,36 @@ __global__ void __launch_bounds__(kBitsThreads) k_mask_bits(const MaskBitsArgs a
 #pragma unroll
         for (int k = 0; k < kBitsThreads / 32; ++k) t += red[k];
         a.counts[(int64_t)m * a.N + i] = t;
+    }
+}
+
+constexpr int kDrawThreads = 128;
+
+__global__ void __launch_bounds__(kDrawThreads) k_mask_draws(const MaskBitsArgs a)
+{
+    const int64_t r = (int64_t)blockIdx.x;
+    const int32_t m = (int32_t)(r % a.n_masks);
+    const int64_t i = a.N - 1 - r / a.n_masks;
+    if (i == 0) return;  // no j < 0
+    const uint32_t head_key = (a.heads_keyed > 1) ? (uint32_t)(m % a.heads_keyed) : 0u;
+    const int32_t s0 = a.per_seed ? m / a.heads_keyed : 0;
+    const int32_t s1 = a.per_seed ? s0 + 1 : a.n_seeds;
+    uint32_t *row = a.bitmap + (int64_t)m * a.words_per_mask + row_word_offset(i);
+    const int64_t groups = (a.draws + 3) >> 2;
+    const uint64_t n = (uint64_t)a.N;
+    for (int32_t s = s0; s < s1; ++s) {
+        const uint32_t seed = a.seeds.v[s];
+        for (int64_t g = threadIdx.x; g < groups; g += kDrawThreads) {
+            const uint4 u = philox4x32_10(make_uint4((uint32_t)g, (uint32_t)i, a.stream + 2u, a.layer_key), seed,
+                                          head_key);
+            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (4 * g + c >= a.draws) break;
+                const int64_t j = (int64_t)(((uint64_t)w4[c] * n) >> 32);
+                if (j < i) atomicOr(row + (j >> 5), 1u << (j & 31));
+            }
+        }
     }
 }
 
@@ -250,6 +285,14 @@ cudaError_t launch_mask_bits(const MaskBitsArgs &a, cudaStream_t s)
 {
     const int64_t blocks = (int64_t)a.n_masks * a.N;
     k_mask_bits<<<(unsigned)blocks, kBitsThreads, 0, s>>>(a);
+    note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_mask_draws(const MaskBitsArgs &a, cudaStream_t s)
+{
+    const int64_t blocks = (int64_t)a.n_masks * a.N;
+    k_mask_draws<<<(unsigned)blocks, kDrawThreads, 0, s>>>(a);
     note_launch();
     return cudaGetLastError();
 }

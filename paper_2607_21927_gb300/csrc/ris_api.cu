@@ -204,6 +204,7 @@ ris_status check_opts(const ris_mask_opts *o)
     if (o->local_window < 1) return fail(RIS_ERR_INVALID, "local_window %d must be >= 1", o->local_window);
     if (o->n_anchor < 0) return fail(RIS_ERR_INVALID, "n_anchor %d must be >= 0", o->n_anchor);
     if (o->per_head != 0 && o->per_head != 1) return fail(RIS_ERR_INVALID, "per_head must be 0 or 1");
+    if (o->sampler != 0 && o->sampler != 1) return fail(RIS_ERR_INVALID, "sampler %d must be 0 or 1", o->sampler);
     return RIS_OK;
 }
 
@@ -314,6 +315,7 @@ ris_status ris_resolve_params(int64_t N, int32_t mode, double density, const ris
         p.thr = keep_threshold(density);
         p.stream = 0;
     }
+    p.draws = (int64_t)std::floor((mode == RIS_MODE_STRUCTURAL ? p.d_global : density) * (double)N + 0.5);
     p.rope_factor = resolve_factor(rope, N);
     p.rope_mscale = (rope != nullptr && rope->kind == RIS_ROPE_YARN) ? 0.1 * std::log(p.rope_factor) + 1.0 : 1.0;
     *out = p;
@@ -360,7 +362,7 @@ ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double d
     RIS_TRY(check_seeds(seeds, n_seeds));
     RIS_TRY(check_opts(opts));
     if (per_seed != 0 && per_seed != 1) return fail(RIS_ERR_INVALID, "per_seed must be 0 or 1");
-    const ris_mask_opts o = opts ? *opts : ris_mask_opts{1, 0, 0, 0u};
+    const ris_mask_opts o = opts ? *opts : ris_mask_opts{1, 0, 0, 0u, 0};
     if (o.per_head && kv_heads < 1) return fail(RIS_ERR_INVALID, "kv_heads must be >= 1 with per_head");
     const int32_t heads_keyed = o.per_head ? kv_heads : 1;
     const int64_t n_masks = (int64_t)(per_seed ? n_seeds : 1) * heads_keyed;
@@ -418,7 +420,15 @@ ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double d
     a.words_per_mask = mk->words_per_mask;
     a.bitmap = mk->bitmap;
     a.counts = mk->row_ptr + 1;
+    a.draws = p.draws;
     for (int k = 0; k < n_seeds; ++k) a.seeds.v[k] = seeds[k];
+    if (o.sampler == 1) {
+        // index draws first, into a zeroed bitmap; the word pass then adds the forced keys
+        RIS_CUDA(cudaMemsetAsync(mk->bitmap, 0, sizeof(uint32_t) * (size_t)(n_masks * mk->words_per_mask), s));
+        if (p.draws > 0) RIS_CUDA(launch_mask_draws(a, s));
+        a.or_existing = 1;
+        a.thr = 0;
+    }
     RIS_CUDA(launch_mask_bits(a, s));
 
     Scratch partials;

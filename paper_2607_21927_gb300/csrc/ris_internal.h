@@ -31,6 +31,8 @@ struct MaskBitsArgs {
     uint32_t stream;      // Philox counter word 2
     uint64_t thr;         // keep iff word < thr
     int64_t B;            // Structural block size
+    int64_t draws;        // index-draw sampler: draws per row and seed
+    int32_t or_existing;  // 1: OR into the words already in the bitmap (index draws were set)
     int64_t words_per_mask;
     uint32_t *bitmap;     // [n_masks][words_per_mask]
     int64_t *counts;      // counts[m * N + i] (row_ptr + 1)
@@ -91,6 +93,7 @@ void set_error_text(const char *msg);
 
 // Launchers: each returns the launch error (cudaGetLastError) of its kernels.
 cudaError_t launch_mask_bits(const MaskBitsArgs &a, cudaStream_t s);
+cudaError_t launch_mask_draws(const MaskBitsArgs &a, cudaStream_t s);
 cudaError_t launch_scan_inplace(int64_t *x, int64_t n, int64_t *partials, cudaStream_t s);
 int64_t scan_partials_count(int64_t n);
 cudaError_t launch_mask_fill(const MaskFillArgs &a, cudaStream_t s);

@@ -38,14 +38,14 @@ class RopeCfg(ctypes.Structure):
 
 class MaskOpts(ctypes.Structure):
     _fields_ = [("local_window", ctypes.c_int32), ("n_anchor", ctypes.c_int32),
-                ("per_head", ctypes.c_int32), ("layer_key", ctypes.c_uint32)]
+                ("per_head", ctypes.c_int32), ("layer_key", ctypes.c_uint32), ("sampler", ctypes.c_int32)]
 
 
 class Params(ctypes.Structure):
     _fields_ = [("bmax", ctypes.c_int64), ("block", ctypes.c_int64), ("clique_pairs", ctypes.c_int64),
                 ("d_clique", ctypes.c_double), ("d_global", ctypes.c_double), ("thr", ctypes.c_uint64),
                 ("stream", ctypes.c_uint32), ("dense", ctypes.c_int32), ("rope_factor", ctypes.c_double),
-                ("rope_mscale", ctypes.c_double)]
+                ("rope_mscale", ctypes.c_double), ("draws", ctypes.c_int64)]
 
 
 class MaskDesc(ctypes.Structure):
@@ -62,8 +62,12 @@ def rope_cfg(kind: int = ROPE_PLAIN, theta: float = 1e6, native_len: int = 32768
                    float(yarn_beta))
 
 
-def mask_opts(local_window: int = 1, n_anchor: int = 0, per_head: bool = False, layer_key: int = 0) -> MaskOpts:
-    return MaskOpts(int(local_window), int(n_anchor), int(bool(per_head)), int(layer_key))
+SAMPLER_BERNOULLI, SAMPLER_DRAWS = 0, 1
+
+
+def mask_opts(local_window: int = 1, n_anchor: int = 0, per_head: bool = False, layer_key: int = 0,
+              sampler: int = SAMPLER_BERNOULLI) -> MaskOpts:
+    return MaskOpts(int(local_window), int(n_anchor), int(bool(per_head)), int(layer_key), int(sampler))
 
 
 _SIGS = {

@@ -67,6 +67,10 @@ def test_invalid_arguments_launch_nothing(ris):
     assert L.ris_mask_generate(64, 1, 0, 0.1, seeds, 2, ctypes.byref(bad_opts), 0, ctypes.byref(h), None) \
         == ris.RIS_ERR_INVALID
     assert h.value is None
+    bad_sampler = ris.mask_opts(sampler=2)
+    assert L.ris_mask_generate(64, 1, 0, 0.1, seeds, 2, ctypes.byref(bad_sampler), 0, ctypes.byref(h), None) \
+        == ris.RIS_ERR_INVALID
+    assert h.value is None
     assert L.ris_rope_apply(None, 1, 10, 1, 128, ctypes.byref(ris.rope_cfg()), None) == ris.RIS_ERR_INVALID
     assert ris.ris_launch_count() == before
 
@@ -91,6 +95,9 @@ def test_resolve_params_agrees_with_oracle(ris, N, d):
     assert (p["bmax"], p["block"], p["clique_pairs"]) == (g["K"], g["B"], g["C"])
     assert p["d_clique"] == g["d_clique"] and p["d_global"] == g["d_global"]
     assert p["thr"] == ora.threshold(g["d_global"]) and p["stream"] == 1
+    # index-draw sampler: K draws per row, the oracle's count for the Structural global part
+    assert p["draws"] == math.floor(g["d_global"] * N + 0.5)
+    assert ris.ris_resolve_params(N, 0, d)["draws"] == math.floor(d * N + 0.5)
     s = ris.ris_resolve_params(N, 0, d)
     assert s["thr"] == ora.threshold(d) and s["stream"] == 0 and s["dense"] == 0
     assert ris.ris_resolve_params(N, 0, 1.0)["dense"] == 1

@@ -30,10 +30,10 @@ def run_gpu(q, k, v, mode, d, seeds, rope_kind, theta, native, out_dtype=torch.f
 
 
 def run_oracle(qn, kn, vn, mode, d, seeds, rope_kind, theta, native, rows=None, seed_index=-1, W=1, A=0,
-               head_key=0):
+               head_key=0, sampler=0):
     N = qn.shape[0]
     spec = ora.MaskSpec(N=N, mode=mode, density=d, seeds=seeds, seed_index=seed_index, local_window=W,
-                        n_anchor=A, head_key=head_key)
+                        n_anchor=A, head_key=head_key, sampler=sampler)
     out, lse, _, _ = ora.sparse_attention(qn, kn, vn, spec, oracle_rope(rope_kind, theta, native), rows=rows)
     return out, lse
 
@@ -96,6 +96,18 @@ def test_attention_bf16_output_and_forced_set():
     assert out.dtype == torch.bfloat16
     ref, _ = run_oracle(qn, kn, vn, 0, 0.02, [1, 2], 1, 1e6, 32768, W=16, A=4)
     check_bf16_path(to_np(out), ref, out_bf16=True)
+
+
+@pytest.mark.parametrize("mode", [0, 1], ids=["stochastic", "structural"])
+def test_attention_index_draw_sampler(mode):
+    """The whole path on a mask from the index-draw sampler (torch.randint reading)."""
+    N, Hq, Hkv, D = 900, 6, 2, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=11, outliers=True)
+    opts = ris.mask_opts(sampler=ris.SAMPLER_DRAWS)
+    out, lse = run_gpu(q, k, v, mode, 0.03, [4, 5, 6], 3, 1e6, 256, opts=opts)
+    ref, ref_lse = run_oracle(qn, kn, vn, mode, 0.03, [4, 5, 6], 3, 1e6, 256, sampler=1)
+    check_bf16_path(to_np(out), ref)
+    np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-2)
 
 
 def test_attention_per_head_masks():

@@ -10,14 +10,14 @@ from paper_2607_21927_gb300 import ris
 pytestmark = pytest.mark.gpu
 
 
-def gpu_mask(N, mode, d, seeds, kv_heads=1, per_seed=False, W=1, A=0, per_head=False, layer_key=0):
-    opts = ris.mask_opts(local_window=W, n_anchor=A, per_head=per_head, layer_key=layer_key)
+def gpu_mask(N, mode, d, seeds, kv_heads=1, per_seed=False, W=1, A=0, per_head=False, layer_key=0, sampler=0):
+    opts = ris.mask_opts(local_window=W, n_anchor=A, per_head=per_head, layer_key=layer_key, sampler=sampler)
     return ris.ris_mask_generate(N, kv_heads, mode, d, seeds, opts=opts, per_seed=per_seed)
 
 
-def oracle_spec(N, mode, d, seeds, seed_index=-1, W=1, A=0, head_key=0, layer_key=0):
+def oracle_spec(N, mode, d, seeds, seed_index=-1, W=1, A=0, head_key=0, layer_key=0, sampler=0):
     return ora.MaskSpec(N=N, mode=mode, density=d, seeds=seeds, seed_index=seed_index, local_window=W,
-                        n_anchor=A, head_key=head_key, layer_key=layer_key)
+                        n_anchor=A, head_key=head_key, layer_key=layer_key, sampler=sampler)
 
 
 def check_rows(m, specs, rows, check_bits=True):
@@ -106,3 +106,37 @@ def test_mask_deterministic_and_keyed():
     assert torch.equal(a, b)
     c = gpu_mask(500, 0, 0.1, [3], layer_key=1).cols().cpu()
     assert a.shape != c.shape or not torch.equal(a, c)
+
+
+# ----------------------------------------------------------------------------- index-draw sampler
+@pytest.mark.parametrize("N,mode,d,S,W,A", [
+    (1, 0, 0.05, 1, 1, 0), (2, 0, 0.9, 3, 1, 0), (33, 0, 0.3, 2, 1, 0), (100, 1, 0.05, 3, 1, 0),
+    (300, 1, 0.2, 1, 4, 3), (513, 0, 1.0, 1, 1, 0), (1000, 1, 0.013, 10, 1, 0), (2048, 0, 0.05, 7, 1, 0),
+    (4133, 0, 0.002, 1, 1, 0), (3000, 0, 0.0001, 2, 5, 0)])
+def test_draw_sampler_full_small(N, mode, d, S, W, A):
+    """Index draws (with replacement, causal filter, merged) bit-exact against the oracle,
+    including K = 0 draws (forced set only) and density 1 (dense)."""
+    seeds = list(range(40, 40 + S))
+    m = gpu_mask(N, mode, d, seeds, W=W, A=A, sampler=1)
+    if m.info().dense:
+        assert m.info().n_pairs == N * (N + 1) // 2
+        return
+    assert m.info().params.draws == ris.ris_resolve_params(N, mode, d)["draws"]
+    check_rows(m, [oracle_spec(N, mode, d, seeds, W=W, A=A, sampler=1)], np.arange(N))
+
+
+def test_draw_sampler_per_seed_and_per_head():
+    N, seeds, Hkv = 600, [5, 6, 7], 2
+    m = gpu_mask(N, 0, 0.05, seeds, kv_heads=Hkv, per_seed=True, per_head=True, layer_key=9, sampler=1)
+    specs = [oracle_spec(N, 0, 0.05, seeds, seed_index=s, head_key=h, layer_key=9, sampler=1)
+             for s in range(3) for h in range(Hkv)]
+    check_rows(m, specs, np.arange(N))
+    m2 = gpu_mask(N, 1, 0.05, seeds, per_seed=True, sampler=1)
+    check_rows(m2, [oracle_spec(N, 1, 0.05, seeds, seed_index=s, sampler=1) for s in range(3)], np.arange(N))
+
+
+@pytest.mark.parametrize("N,mode,d,S", [(65536, 0, 0.01, 10), (65536, 1, 0.01, 10), (32768, 0, 0.01, 70)])
+def test_draw_sampler_config_sizes_sampled_rows(N, mode, d, S):
+    seeds = list(range(S))
+    m = gpu_mask(N, mode, d, seeds, sampler=1)
+    check_rows(m, [oracle_spec(N, mode, d, seeds, sampler=1)], sample_rows(N, 48, seed=N + mode))
