@@ -68,6 +68,15 @@ WORKLOADS = {
     "C5": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
                runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)],
                title="Qwen2-1.5B-shaped prefill attention stack, N=65536, 28 layers, YaRN s=2"),
+    # C5 with the paper's full geometry: local window 1024 and anchors over the first tokens
+    "C6": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+               runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)], geometry="paper",
+               title="C5 with the paper's geometry (local window 1024 + 4 anchor tokens)"),
+    # the sub-1% Structural sweep at 64k: d = 0.1% .. 0.9%, 50 .. 200 seeds, one layer each
+    "S1": dict(N=65536, layers=1, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+               runs=[(f"structural_{d / 10:.1f}pct_x{s}", 1, d / 1000, s) for d in range(1, 10)
+                     for s in (50, 100, 150, 200)],
+               title="sub-1% Structural sweep at N=65536 (36 masks, one layer each)"),
 }
 
 
@@ -122,6 +131,7 @@ def workload_config(a):
         "head_dim": w["D"], "rope": kind, "rope_theta": theta, "native_len": native,
         "runs": [{"name": n, "mode": m, "density": d, "seeds": s} for n, m, d, s in w["runs"]],
         "input_dtype": w["dtype"], "outlier_channels": "1% x8" if w["outliers"] else None,
+        "geometry": ("local window 1024 + 4 anchors" if w.get("geometry") == "paper" else "diagonal only"),
         "l2": (f"inputs larger than L2: each layer has its own q/k/v ({per_layer / 2**20:.0f} MiB), "
                f"{w['layers']} layers = {w['layers'] * per_layer / 2**20:.0f} MiB per run"),
     }
@@ -246,7 +256,9 @@ def oracle_sample(q_host, k_host, v_host, w, run, target_s, rng_seed):
 
     N = w["N"]
     name, mode, density, n_seeds = run
-    spec = oracle.MaskSpec(N=N, mode=mode, density=density, seeds=list(range(n_seeds)))
+    paper = w.get("geometry") == "paper"
+    spec = oracle.MaskSpec(N=N, mode=mode, density=density, seeds=list(range(n_seeds)),
+                           local_window=1024 if paper else 1, n_anchor=4 if paper else 0)
     cfg = oracle_rope(w)
     rng = np.random.default_rng(rng_seed)
     nrows, total_ph, total_t, used = 8, 0, 0.0, 0
@@ -384,6 +396,7 @@ def main():
     runs = w["runs"]
     kind, theta, native = w["rope"]
     rope = ris.rope_cfg(ROPE_KINDS[kind], theta, native)
+    geom = ris.paper_geometry() if w.get("geometry") == "paper" else None
 
     # inputs resident in HBM: one (q, k, v) per layer, layer L drawn from seed L
     qs, ks, vs = [], [], []
@@ -395,21 +408,23 @@ def main():
     outs = [[torch.empty(N, Hq, D, dtype=tdt, device=dev) for _ in range(L)] for _ in runs]
     stream = torch.cuda.current_stream()
     pairs, design = {}, {}
-    mask_events = []  # (start, end) around each mask build while `timing` is set
+    mask_events = []  # (run, start, mask built, layers done) events of each run while `timing` is set
     timing = [False]
 
     def step():
         for ri, (name, mode, dens, ns) in enumerate(runs):
             if timing[0]:
-                mask_events.append((torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)))
-                mask_events[-1][0].record(stream)
-            m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)))
-            if timing[0]:
+                mask_events.append((name,) + tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)))
                 mask_events[-1][1].record(stream)
+            m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom)
+            if timing[0]:
+                mask_events[-1][2].record(stream)
             pairs[name] = m.info().n_pairs
             design[name] = ris.ris_attention_design(m, tdt, D)
             for layer in range(L):
                 ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[ri][layer])
+            if timing[0]:
+                mask_events[-1][3].record(stream)
             m.free()
 
     for _ in range(a.warmup):
@@ -445,7 +460,10 @@ def main():
     lib_cur, lib_high = ris.ris_memory_stats()
     torch_high = torch.cuda.max_memory_allocated(dev)
 
-    mask_ms = max_over_ranks(sum(e0.elapsed_time(e1) for e0, e1 in mask_events) / a.steps, dist)
+    mask_ms = max_over_ranks(sum(e0.elapsed_time(e1) for _, e0, e1, _ in mask_events) / a.steps, dist)
+    layers_ms = {}  # per run: its layers' device time per step (RoPE + attention)
+    for name, _, e1, e2 in mask_events:
+        layers_ms[name] = layers_ms.get(name, 0.0) + e1.elapsed_time(e2) / a.steps
     total_pairs = sum(pairs.values())
     pair_heads_step = total_pairs * L * Hq
     value = world * pair_heads_step * a.steps / (elapsed_ms / 1e3)
@@ -485,6 +503,32 @@ def main():
             roofline["l2_note"] = ("the K/V working set is L2-resident, so the gather is served from L2: "
                                    "peak = this library's probe reading whole 256-byte rows at random indices "
                                    f"over {ceil['l2_rows_set_bytes'] / 2**20:.0f} MiB")
+    if len(kinds) > 1:
+        # several designs in one step: each design's work over its runs' layer time (RoPE included)
+        per = {}
+        for name, kd in design.items():
+            t = per.setdefault(kd, [0.0, 0])
+            t[0] += layers_ms[name]
+            t[1] += pairs[name]
+        roofline["per_design"] = {}
+        for kd, (ms, pr) in per.items():
+            if kd == 2:
+                ach = 4 * D * Hq * pr * L / (ms / 1e3) / 1e12
+                roofline["per_design"][ris.DESIGNS[kd]] = {"bound": "tensor", "achieved": ach, "peak": tc,
+                                                           "unit": "TFLOP/s", "frac": ach / tc, "ms_per_step": ms}
+            else:
+                ach = pr * L * kv_row_bytes / (ms / 1e3) / 1e9
+                ent = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+                       "ms_per_step": ms}
+                if "l2_rows_gbs" in ceil:
+                    ent["frac_of_l2_rows"] = ach / ceil["l2_rows_gbs"]
+                roofline["per_design"][ris.DESIGNS[kd]] = ent
+        dom = max(per, key=lambda kd: per[kd][0])
+        top = roofline["per_design"][ris.DESIGNS[dom]]
+        roofline.update({k: top[k] for k in ("bound", "achieved", "peak", "unit", "frac")})
+        roofline.pop("frac_of_l2_rows", None)
+        roofline["kernel"] = "mixed designs; headline = " + ris.DESIGNS[dom] + " (most device time)"
+        roofline["note"] = "per design: its runs' layer time per step (RoPE included), not the kernel alone"
     # the sampled-pair roofline: max(sampled FLOPs / tensor peak, min(row, tile) K/V bytes / bandwidth)
     flops = 4 * D * Hq * total_pairs * L
     b_row = total_pairs * L * kv_row_bytes
@@ -496,7 +540,7 @@ def main():
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps, "warmup": a.warmup,
             "ms_per_step": ms_step, "ms_per_layer": ms_step / (len(runs) * L), "higher_is_better": True,
-            "mask_ms_per_step": mask_ms,
+            "mask_ms_per_step": mask_ms, "layers_ms_per_run": layers_ms,
             "attn_ms_per_layer": (ms_step - mask_ms) / (len(runs) * L),
             "attn_pair_heads_per_s": world * pair_heads_step / ((ms_step - mask_ms) / 1e3),
             "scaling": "weak", "vs_baseline": None, "dtype": w["dtype"], "data": "synthetic",
@@ -539,7 +583,7 @@ def main():
                     vs[layer].copy_(hv[layer], non_blocking=True)
                     in_ready[layer].record(h2d_s)
             for ri, (name, mode, dens, ns) in enumerate(runs):
-                m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)))
+                m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom)
                 for layer in range(L):
                     stream.wait_event(in_ready[layer])
                     if not first[0]:

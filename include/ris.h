@@ -72,6 +72,14 @@ typedef struct {
                              Generation") */
 } ris_mask_opts;
 
+/* The paper's three-part geometry (Results, "Ensemble Stochastic Projection and Retrieval
+ * Coverage"): a dense local window of 1024 tokens, a global anchor over the initial tokens
+ * and the stochastic ensemble. The paper does not give the anchor count; 4 initial tokens
+ * (the attention-sink count of streaming attention) is this library's reading. Use as
+ * ris_mask_opts{RIS_PRESET_LOCAL_WINDOW, RIS_PRESET_ANCHORS, 0, 0, 0}. */
+#define RIS_PRESET_LOCAL_WINDOW 1024
+#define RIS_PRESET_ANCHORS 4
+
 /* Derived scalars of one call, resolved on the host. */
 typedef struct {
     int64_t bmax;            /* K = floor(d N + 0.5), the paper's B_max */

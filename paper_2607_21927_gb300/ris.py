@@ -63,11 +63,17 @@ def rope_cfg(kind: int = ROPE_PLAIN, theta: float = 1e6, native_len: int = 32768
 
 
 SAMPLER_BERNOULLI, SAMPLER_DRAWS = 0, 1
+PRESET_LOCAL_WINDOW, PRESET_ANCHORS = 1024, 4  # include/ris.h RIS_PRESET_*
 
 
 def mask_opts(local_window: int = 1, n_anchor: int = 0, per_head: bool = False, layer_key: int = 0,
               sampler: int = SAMPLER_BERNOULLI) -> MaskOpts:
     return MaskOpts(int(local_window), int(n_anchor), int(bool(per_head)), int(layer_key), int(sampler))
+
+
+def paper_geometry(per_head: bool = False, layer_key: int = 0, sampler: int = SAMPLER_BERNOULLI) -> MaskOpts:
+    """The paper's local window of 1024 tokens plus global anchors over the first tokens."""
+    return mask_opts(PRESET_LOCAL_WINDOW, PRESET_ANCHORS, per_head, layer_key, sampler)
 
 
 _SIGS = {

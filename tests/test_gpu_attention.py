@@ -158,11 +158,12 @@ def test_v_constant_gives_one():
 
 
 # ----------------------------------------------------------------------------- workload configurations
-def _config_case(N, shape, dtype, mode, d, S, kind, outliers, nrows, seed=0, per_seed=False):
+def _config_case(N, shape, dtype, mode, d, S, kind, outliers, nrows, seed=0, per_seed=False, opts=None):
     (q, k, v), (qn, kn, vn) = make_inputs(N, shape["Hq"], shape["Hkv"], shape["D"], dtype=dtype, seed=seed,
                                           outliers=outliers)
     seeds = list(range(S))
-    out, lse = run_gpu(q, k, v, mode, d, seeds, kind, shape["theta"], shape["native"], per_seed=per_seed)
+    out, lse = run_gpu(q, k, v, mode, d, seeds, kind, shape["theta"], shape["native"], per_seed=per_seed,
+                       opts=opts)
     rows = np.arange(N) if nrows is None else sample_rows(N, nrows, seed=N + S)
     got = to_np(out[rows] if not per_seed else out[:, rows])
     return got, (qn, kn, vn), seeds, rows, to_np(lse)
@@ -205,6 +206,16 @@ def test_c5_qwen_64k_layer(mode):
     got, (qn, kn, vn), seeds, rows, _ = _config_case(65536, QWEN, torch.bfloat16, mode, 0.01, 10, 3, True, 96,
                                                      seed=3)
     ref, _ = run_oracle(qn, kn, vn, mode, 0.01, seeds, 3, 1e6, 32768, rows=rows)
+    check_bf16_path(got, ref)
+
+
+@pytest.mark.parametrize("mode", [0, 1], ids=["stochastic", "structural"])
+def test_c6_paper_geometry_64k_layer(mode):
+    """The N=65536 layer with the paper's geometry (local window 1024 + 4 anchors); sampled rows."""
+    got, (qn, kn, vn), seeds, rows, _ = _config_case(65536, QWEN, torch.bfloat16, mode, 0.01, 10, 3, True, 64,
+                                                     seed=5, opts=ris.paper_geometry())
+    ref, _ = run_oracle(qn, kn, vn, mode, 0.01, seeds, 3, 1e6, 32768, rows=rows, W=ris.PRESET_LOCAL_WINDOW,
+                        A=ris.PRESET_ANCHORS)
     check_bf16_path(got, ref)
 
 

@@ -140,3 +140,28 @@ def test_draw_sampler_config_sizes_sampled_rows(N, mode, d, S):
     seeds = list(range(S))
     m = gpu_mask(N, mode, d, seeds, sampler=1)
     check_rows(m, [oracle_spec(N, mode, d, seeds, sampler=1)], sample_rows(N, 48, seed=N + mode))
+
+
+# ----------------------------------------------------------------------------- paper geometry and sweep
+@pytest.mark.parametrize("mode", [0, 1])
+def test_mask_paper_geometry_full_size(mode):
+    """Local window 1024 + 4 anchors at N=65536 (both modes, 1% x 10): sampled rows bit-exact,
+    every row keeps its whole window and the anchors."""
+    N, seeds = 65536, list(range(10))
+    m = gpu_mask(N, mode, 0.01, seeds, W=ris.PRESET_LOCAL_WINDOW, A=ris.PRESET_ANCHORS)
+    rows = sample_rows(N, 32, seed=77 + mode)
+    check_rows(m, [oracle_spec(N, mode, 0.01, seeds, W=1024, A=4)], rows)
+    counts = np.diff(m.row_ptr().cpu().numpy())
+    i = np.arange(N)
+    assert (counts >= np.minimum(i + 1, 1024)).all()
+    assert (counts[1027:] >= 1024 + 4).all()  # window and anchors are disjoint from row 1027 on
+
+
+@pytest.mark.parametrize("d,S", [(0.001, 200), (0.003, 150), (0.005, 100), (0.009, 50)])
+def test_mask_sub1pct_structural_sweep(d, S):
+    """Sub-1% Structural sweep points at N=65536: B_max as the paper's table, sampled rows bit-exact."""
+    N, seeds = 65536, list(range(S))
+    m = gpu_mask(N, 1, d, seeds)
+    p = m.info().params
+    assert p.bmax == int(np.floor(d * N + 0.5)) and p.block == min(N // 10, p.bmax)
+    check_rows(m, [oracle_spec(N, 1, d, seeds)], sample_rows(N, 16, seed=int(d * 1e4) + S))
