@@ -270,3 +270,40 @@ def sparse_attention(q, k, v, spec: MaskSpec, rope_cfg: Optional[RopeCfg] = None
     out, lse = attention(qr, kr, np.asarray(v, dtype=np.float64), off, cols)
     return out, lse, off, cols
 
+
+
+# ----------------------------------------------------------------------------- Hybrid Anchor decode
+def decode_anchor(spec: MaskSpec) -> np.ndarray:
+    """Stochastic Anchor (Methods, "Hybrid Anchor and Pre-Fusion Unified Softmax"): the key set
+    of the first generated token, at position t0 = spec.N (the prefill length), frozen for the
+    rest of the generation. Reading: it is row t0 of the RIS mask with the prefill's parameters
+    (mode, density, seeds, anchors, keys, sampler) and without its local window, i.e. every
+    kept key j < t0; the local part is the decode step's own sliding window."""
+    t0 = int(spec.N)
+    s = MaskSpec(N=spec.N, mode=spec.mode, density=spec.density, seeds=spec.seeds, seed_index=spec.seed_index,
+                 local_window=1, n_anchor=spec.n_anchor, head_key=spec.head_key, layer_key=spec.layer_key,
+                 sampler=spec.sampler)
+    off, cols = mask_cols(s, np.array([t0], dtype=np.int64))
+    return cols[cols < t0]
+
+
+def decode_keys(anchor: np.ndarray, t: int, window: int) -> np.ndarray:
+    """Keys of the token at position t: the frozen anchor merged with the Dynamic Local Window
+    {t - window < j <= t}, duplicates removed, ascending (the paper's unique() merge)."""
+    win = np.arange(max(0, t - window + 1), t + 1, dtype=np.int64)
+    return np.union1d(np.asarray(anchor, dtype=np.int64), win)
+
+
+def decode_step(q_t, k, v, t: int, anchor: np.ndarray, window: int, rope_cfg: Optional[RopeCfg], n_ctx: int):
+    """One generated token: q_t [Hq, D] at position t attends, with one softmax (PFUS), to the
+    merged key set over the cache k, v [T, Hkv, D] (T > t). RoPE of q at position t and of the
+    cache at positions 0..T-1, with the extension factor resolved for n_ctx tokens.
+    Returns (out[Hq, D], lse[Hq], keys)."""
+    k = np.asarray(k)
+    T = k.shape[0]
+    assert t < T
+    keys = decode_keys(anchor, t, window)
+    qr = rope(np.asarray(q_t)[None], np.array([float(t)]), rope_cfg, n_ctx)
+    kr = rope(k, np.arange(T, dtype=np.float64), rope_cfg, n_ctx)
+    out, lse = attention(qr, kr, np.asarray(v, dtype=np.float64), np.array([0, keys.shape[0]]), keys)
+    return out[0], lse[0], keys

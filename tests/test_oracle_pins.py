@@ -499,3 +499,68 @@ def test_draw_sampler_union_and_edges(oracle):
     a = oracle.mask_dense(oracle.MaskSpec(N=N, mode=0, density=0.05, seeds=[1], sampler=1))
     b = oracle.mask_dense(oracle.MaskSpec(N=N, mode=0, density=0.05, seeds=[1], sampler=0))
     assert (a != b).any()
+
+
+# ----------------------------------------------------------------------------- Hybrid Anchor decode
+def test_decode_anchor_matches_triton_bernoulli(oracle, tmp_path):
+    """The Stochastic Anchor is row t0 = N of the prefill's RIS mask without its window: each
+    j < t0 is kept iff some seed's Philox word (Triton's independent implementation, counter
+    (j/4, t0, stream, layer_key), key (seed, head_key)) is below thr, plus the anchor tokens
+    and, for Structural, the clique of t0's block."""
+    pytest.importorskip("triton")
+    N, seeds, A = 300, [4, 8], 3
+    cases = [(oracle.MODE_STOCHASTIC, 0.05, 0, 0), (oracle.MODE_STRUCTURAL, 0.08, 1, 2)]
+    for mode, d, hk, lk in cases:
+        g = oracle.structural(N, d)
+        p, stream = (g["d_global"], 1) if mode == oracle.MODE_STRUCTURAL else (d, 0)
+        js = np.arange(N)
+        ctr = np.array([(j // 4, N, stream, lk) for s in seeds for j in js], dtype=np.uint32)
+        key = np.array([(s, hk) for s in seeds for j in js], dtype=np.uint32)
+        words = _triton_philox(tmp_path, ctr, key).reshape(len(seeds), N, 4)
+        u = words[:, js, js % 4]
+        want = set(js[(u < oracle.threshold(p)).any(0)].tolist()) | set(range(A))
+        if mode == oracle.MODE_STRUCTURAL:
+            want |= set(range((N // g["B"]) * g["B"], N))
+        spec = oracle.MaskSpec(N=N, mode=mode, density=d, seeds=seeds, n_anchor=A, head_key=hk, layer_key=lk,
+                               local_window=7)
+        got = oracle.decode_anchor(spec)
+        assert set(got.tolist()) == want and (np.diff(got) > 0).all() and got.max() < N
+
+
+def test_decode_full_window_equals_dense_causal_row(oracle):
+    """A window that reaches position 0 covers every earlier key: the decode output is the last
+    row of dense causal attention (torch fp64 SDPA) over the rotated sequence."""
+    N, t, Hq, Hkv, D = 64, 70, 4, 2, 32
+    q, k, v = _rand((t + 1, Hq, D), 21), _rand((t + 1, Hkv, D), 22), _rand((t + 1, Hkv, D), 23)
+    cfg = oracle.RopeCfg(kind=3, theta=1e4, native_len=32)
+    anchor = oracle.decode_anchor(oracle.MaskSpec(N=N, mode=0, density=0.1, seeds=[1]))
+    out, lse, keys = oracle.decode_step(q[t], k, v, t, anchor, window=t + 1, rope_cfg=cfg, n_ctx=N)
+    np.testing.assert_array_equal(keys, np.arange(t + 1))
+    pos = np.arange(t + 1, dtype=np.float64)
+    qr, kr = oracle.rope(q, pos, cfg, N), oracle.rope(k, pos, cfg, N)
+    ref, ref_lse = _sdpa(qr, kr, v, np.tril(np.ones((t + 1, t + 1), bool)), Hq // Hkv)
+    np.testing.assert_allclose(out, ref[t], rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(lse, ref_lse[t], rtol=1e-12, atol=1e-12)
+
+
+def test_decode_merge_is_set_union_with_one_softmax(oracle):
+    """Window and anchor overlap: the key set is their set union (each key once), and the output
+    is one softmax over it (brute force in torch fp64 on the explicit key rows)."""
+    N, Hq, Hkv, D = 125, 6, 2, 16
+    anchor = oracle.decode_anchor(oracle.MaskSpec(N=N, mode=1, density=0.1, seeds=[3, 5]))
+    assert set(range(120, 125)) <= set(anchor.tolist())  # B = 12: t0 = 125 shares block [120, 132)
+    for t, W in ((125, 16), (128, 1), (130, 30), (200, 5)):
+        q, k, v = _rand((Hq, D), t), _rand((t + 1, Hkv, D), t + 1), _rand((t + 1, Hkv, D), t + 2)
+        out, lse, keys = oracle.decode_step(q, k, v, t, anchor, W, None, N)
+        want = sorted(set(anchor.tolist()) | set(range(max(0, t - W + 1), t + 1)))
+        np.testing.assert_array_equal(keys, want)
+        G = Hq // Hkv
+        for h in range(Hq):
+            kt = torch.from_numpy(k[keys, h // G])
+            s = kt @ torch.from_numpy(q[h]) / math.sqrt(D)
+            p = torch.softmax(s, 0)
+            np.testing.assert_allclose(out[h], (p[:, None] * torch.from_numpy(v[keys, h // G])).sum(0).numpy(),
+                                       rtol=1e-10, atol=1e-12)
+            np.testing.assert_allclose(lse[h], torch.logsumexp(s, 0).item(), rtol=1e-12)
+    out, _, _ = oracle.decode_step(q, k, np.ones_like(v), 200, anchor, 5, None, N)
+    np.testing.assert_allclose(out, 1.0, atol=1e-13)
