@@ -249,6 +249,54 @@ int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim);
  * undefined. Blocks. Errors: RIS_ERR_CUDA. */
 ris_status ris_device_status(void *stream);
 
+/* ---- Hybrid Anchor decode (Methods, "Hybrid Anchor and Pre-Fusion Unified Softmax (PFUS)") ----
+ * After a prefill of n_prefill tokens, the token generated at position t >= t0 = n_prefill
+ * attends, with one softmax, to the union of
+ *   - the Stochastic Anchor: the key set of the first generated token, computed once and frozen.
+ *     It is row t0 of the prefill's RIS mask (same mode, density, seeds, anchors n_anchor,
+ *     per_head / layer_key keying and sampler; parameters resolved for n_prefill tokens)
+ *     without its local window: every kept key j < t0;
+ *   - the Dynamic Local Window: keys t - window < j <= t.
+ * Duplicates are merged (each key counts once). The K/V cache holds the rotated keys. */
+typedef struct ris_anchor_s *ris_anchor_t;
+
+/* Build the Stochastic Anchor on the device (one mask row per KV head when opts->per_head,
+ * else one) and keep a host copy of its keys for the per-step merge. opts->local_window is
+ * ignored (the decode step has its own window). Blocks (reads the key count back).
+ * Errors: as ris_mask_generate; RIS_ERR_INVALID also for n_prefill >= 2^31 - 1. */
+ris_status ris_decode_anchor(int64_t n_prefill, int32_t kv_heads, int32_t mode, double density,
+                             const uint32_t *seeds, int32_t n_seeds, const ris_mask_opts *opts,
+                             ris_anchor_t *out, void *stream);
+
+/* Layout of an anchor: t0, number of keyed lists (1 or kv_heads), total keys, and DEVICE
+ * pointers to the keys (int32, ascending within each list) and the heads_keyed + 1 int64
+ * offsets (list m = keys[offsets[m] .. offsets[m+1])). Any output pointer may be NULL. */
+ris_status ris_anchor_info(ris_anchor_t anchor, int64_t *t0, int32_t *heads_keyed, int64_t *n_keys,
+                           const int32_t **keys, const int64_t **offsets);
+ris_status ris_anchor_free(ris_anchor_t anchor);
+
+/* Rotate x [n][heads][head_dim] (dtype) at positions pos0 .. pos0+n-1 into hi (same dtype)
+ * and, for bf16 when lo is not NULL, lo = bf16(y - bf16(y)) so that hi + lo carries the fp32
+ * rotation to ~16 bits: the format of a rotated K cache. The extension factor is resolved
+ * for n_ctx tokens (rope->factor <= 0). rope NULL or RIS_ROPE_NONE copies x (no rotation).
+ * x and hi may be the same buffer. Errors: RIS_ERR_INVALID, RIS_ERR_CUDA. */
+ris_status ris_rope_split(const void *x, int32_t dtype, int64_t n, int64_t pos0, int32_t heads, int32_t head_dim,
+                          int64_t n_ctx, const ris_rope_cfg *rope, void *hi, void *lo, void *stream);
+
+/* One decode step. q: [heads][head_dim] query of the token at position t, NOT rotated (the
+ * kernel rotates it at position t with the extension factor of n_ctx tokens). k (+ k_lo for
+ * bf16, may be NULL) and v: the cache [cache_len][kv_heads][head_dim] holding positions
+ * 0 .. cache_len-1 with rotated keys (ris_rope_split); it must already hold the token t's own
+ * key and value. out: [heads][head_dim] (out_dtype); lse: [heads] natural-log sum of
+ * exp(score) or NULL. Scores and probabilities are fp32. Asynchronous; per-step scratch comes
+ * from the stream-ordered pool. Errors: RIS_ERR_INVALID (t < t0, t >= cache_len, window < 1,
+ * shapes, pointers, anchor keyed for another kv_heads), RIS_ERR_UNSUPPORTED (kv_heads > 64),
+ * RIS_ERR_CUDA. */
+ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, const void *k_lo, const void *v,
+                           int64_t cache_len, int64_t t, int32_t window, int32_t heads, int32_t kv_heads,
+                           int32_t head_dim, int32_t dtype, int32_t out_dtype, int64_t n_ctx,
+                           const ris_rope_cfg *rope, void *out, float *lse, void *stream);
+
 /* ---- Measurement support (the paper has no counterpart) -------------------------------------
  * Small kernels that measure the ceilings the attention kernels are compared against, for the
  * current device. Each allocates its own device buffers, runs on `stream` (NULL: legacy default

@@ -69,12 +69,13 @@ __global__ void __launch_bounds__(kBitsThreads) k_mask_bits(const MaskBitsArgs a
     // rows are visited from the last (longest) to the first
     const int64_t r = (int64_t)blockIdx.x;
     const int32_t m = (int32_t)(r % a.n_masks);
-    const int64_t i = a.N - 1 - r / a.n_masks;
+    const bool one = a.single_row >= 0;
+    const int64_t i = one ? a.single_row : a.N - 1 - r / a.n_masks;
     const uint32_t head_key = (a.heads_keyed > 1) ? (uint32_t)(m % a.heads_keyed) : 0u;
     const int32_t s0 = a.per_seed ? m / a.heads_keyed : 0;
     const int32_t s1 = a.per_seed ? s0 + 1 : a.n_seeds;
     const int64_t nw = (i >> 5) + 1;
-    uint32_t *row = a.bitmap + (int64_t)m * a.words_per_mask + row_word_offset(i);
+    uint32_t *row = a.bitmap + (int64_t)m * a.words_per_mask + (one ? 0 : row_word_offset(i));
     const int64_t blk0 = (a.mode == RIS_MODE_STRUCTURAL) ? (i / a.B) * a.B : i + 1;
 
     int64_t count = 0;
@@ -106,7 +107,7 @@ __global__ void __launch_bounds__(kBitsThreads) k_mask_bits(const MaskBitsArgs a
                 }
             }
         }
-        bits &= range_bits(j0, 0, i);
+        bits &= range_bits(j0, 0, one ? i - 1 : i);  // a single row keeps keys j < i only
         row[w] = bits;
         count += __popc(bits);
     }
@@ -120,7 +121,7 @@ __global__ void __launch_bounds__(kBitsThreads) k_mask_bits(const MaskBitsArgs a
         int64_t t = 0;
 #pragma unroll
         for (int k = 0; k < kBitsThreads / 32; ++k) t += red[k];
-        a.counts[(int64_t)m * a.N + i] = t;
+        a.counts[one ? (int64_t)m : (int64_t)m * a.N + i] = t;
     }
 }
 
@@ -130,12 +131,13 @@ __global__ void __launch_bounds__(kDrawThreads) k_mask_draws(const MaskBitsArgs 
 {
     const int64_t r = (int64_t)blockIdx.x;
     const int32_t m = (int32_t)(r % a.n_masks);
-    const int64_t i = a.N - 1 - r / a.n_masks;
+    const bool one = a.single_row >= 0;
+    const int64_t i = one ? a.single_row : a.N - 1 - r / a.n_masks;
     if (i == 0) return;  // no j < 0
     const uint32_t head_key = (a.heads_keyed > 1) ? (uint32_t)(m % a.heads_keyed) : 0u;
     const int32_t s0 = a.per_seed ? m / a.heads_keyed : 0;
     const int32_t s1 = a.per_seed ? s0 + 1 : a.n_seeds;
-    uint32_t *row = a.bitmap + (int64_t)m * a.words_per_mask + row_word_offset(i);
+    uint32_t *row = a.bitmap + (int64_t)m * a.words_per_mask + (one ? 0 : row_word_offset(i));
     const int64_t groups = (a.draws + 3) >> 2;
     const uint64_t n = (uint64_t)a.N;
     for (int32_t s = s0; s < s1; ++s) {
@@ -242,10 +244,11 @@ __global__ void __launch_bounds__(kFillThreads) k_mask_fill(const MaskFillArgs a
     __shared__ int64_t warp_tot[kFillThreads / 32];
     const int64_t r = (int64_t)blockIdx.x;
     const int32_t m = (int32_t)(r % a.n_masks);
-    const int64_t i = a.N - 1 - r / a.n_masks;
+    const bool one = a.single_row >= 0;
+    const int64_t i = one ? a.single_row : a.N - 1 - r / a.n_masks;
     const int64_t nw = (i >> 5) + 1;
-    const uint32_t *row = a.bitmap + (int64_t)m * a.words_per_mask + row_word_offset(i);
-    TIdx *col = reinterpret_cast<TIdx *>(a.col) + a.row_ptr[(int64_t)m * a.N + i];
+    const uint32_t *row = a.bitmap + (int64_t)m * a.words_per_mask + (one ? 0 : row_word_offset(i));
+    TIdx *col = reinterpret_cast<TIdx *>(a.col) + a.row_ptr[one ? (int64_t)m : (int64_t)m * a.N + i];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     int64_t carry = 0;
     for (int64_t w0 = 0; w0 < nw; w0 += kFillThreads) {
@@ -283,7 +286,7 @@ __global__ void __launch_bounds__(kFillThreads) k_mask_fill(const MaskFillArgs a
 
 cudaError_t launch_mask_bits(const MaskBitsArgs &a, cudaStream_t s)
 {
-    const int64_t blocks = (int64_t)a.n_masks * a.N;
+    const int64_t blocks = (int64_t)a.n_masks * (a.single_row >= 0 ? 1 : a.N);
     k_mask_bits<<<(unsigned)blocks, kBitsThreads, 0, s>>>(a);
     note_launch();
     return cudaGetLastError();
@@ -291,7 +294,7 @@ cudaError_t launch_mask_bits(const MaskBitsArgs &a, cudaStream_t s)
 
 cudaError_t launch_mask_draws(const MaskBitsArgs &a, cudaStream_t s)
 {
-    const int64_t blocks = (int64_t)a.n_masks * a.N;
+    const int64_t blocks = (int64_t)a.n_masks * (a.single_row >= 0 ? 1 : a.N);
     k_mask_draws<<<(unsigned)blocks, kDrawThreads, 0, s>>>(a);
     note_launch();
     return cudaGetLastError();
@@ -311,7 +314,7 @@ cudaError_t launch_scan_inplace(int64_t *x, int64_t n, int64_t *partials, cudaSt
 
 cudaError_t launch_mask_fill(const MaskFillArgs &a, cudaStream_t s)
 {
-    const int64_t blocks = (int64_t)a.n_masks * a.N;
+    const int64_t blocks = (int64_t)a.n_masks * (a.single_row >= 0 ? 1 : a.N);
     if (a.col_bytes == 2)
         k_mask_fill<uint16_t><<<(unsigned)blocks, kFillThreads, 0, s>>>(a);
     else

@@ -3,6 +3,7 @@
 // file only decides, allocates (stream-ordered pool) and launches.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <atomic>
 #include <cmath>
 #include <cstdarg>
@@ -40,6 +41,17 @@ struct ris_mask_s {
     int64_t *row_ptr = nullptr;
     void *col = nullptr;
     uint32_t *bitmap = nullptr;
+    ris_params params{};
+    cudaStream_t stream = nullptr;
+};
+
+struct ris_anchor_s {
+    int64_t t0 = 0;  // position of the first generated token (the prefill length)
+    int32_t heads_keyed = 1, kv_heads = 1;
+    int32_t *keys = nullptr;  // device, ascending per mask
+    int64_t *off = nullptr;   // device, heads_keyed + 1 offsets
+    std::vector<int32_t> h_keys;
+    std::vector<int64_t> h_off;
     ris_params params{};
     cudaStream_t stream = nullptr;
 };
@@ -405,6 +417,7 @@ ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double d
     RIS_CUDA(cudaMemsetAsync(mk->row_ptr, 0, sizeof(int64_t), s));
 
     MaskBitsArgs a{};
+    a.single_row = -1;
     a.N = N;
     a.n_seeds = n_seeds;
     a.per_seed = per_seed;
@@ -442,6 +455,7 @@ ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double d
     RIS_CUDA(cudaMallocAsync(&mk->col, (size_t)(total > 0 ? total : 1) * mk->col_bytes, s));
 
     MaskFillArgs f{};
+    f.single_row = -1;
     f.N = N;
     f.n_masks = (int32_t)n_masks;
     f.col_bytes = mk->col_bytes;
@@ -697,6 +711,239 @@ ris_status ris_ensemble_batch(const void *q, const void *k, const void *v, void 
 {
     return fwd_common(q, k, v, out, N, heads, kv_heads, head_dim, mode, density, seeds, n_seeds, dtype,
                       out_dtype, rope, opts, lse, stream, 1);
+}
+
+// ---------------------------------------------------------------- Hybrid Anchor decode
+ris_status ris_decode_anchor(int64_t n_prefill, int32_t kv_heads, int32_t mode, double density,
+                             const uint32_t *seeds, int32_t n_seeds, const ris_mask_opts *opts, ris_anchor_t *out,
+                             void *stream)
+{
+    if (out == nullptr) return fail(RIS_ERR_INVALID, "out is NULL");
+    *out = nullptr;
+    RIS_TRY(check_N(n_prefill));
+    if (n_prefill >= 2147483647LL) return fail(RIS_ERR_INVALID, "n_prefill must be < 2^31 - 1");
+    RIS_TRY(check_mode_density(mode, density));
+    RIS_TRY(check_seeds(seeds, n_seeds));
+    RIS_TRY(check_opts(opts));
+    const ris_mask_opts o = opts ? *opts : ris_mask_opts{1, 0, 0, 0u, 0};
+    if (o.per_head && (kv_heads < 1 || kv_heads > kMaxDecodeKvHeads))
+        return fail(RIS_ERR_INVALID, "kv_heads %d outside [1, %d]", kv_heads, kMaxDecodeKvHeads);
+    ris_params p{};
+    RIS_TRY(ris_resolve_params(n_prefill, mode, density, nullptr, &p));
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const int32_t hk = o.per_head ? kv_heads : 1;
+    const int64_t t0 = n_prefill;
+
+    ris_anchor_s *an = new (std::nothrow) ris_anchor_s();
+    if (an == nullptr) return fail(RIS_ERR_OOM, "host allocation failed");
+    struct Guard {
+        ris_anchor_s *a;
+        ~Guard()
+        {
+            if (a) ris_anchor_free(a);
+        }
+    } guard{an};
+    an->t0 = t0;
+    an->heads_keyed = hk;
+    an->kv_heads = kv_heads;
+    an->params = p;
+    an->stream = s;
+    prepare_pool_once();
+    RIS_CUDA(cudaMallocAsync((void **)&an->off, sizeof(int64_t) * (size_t)(hk + 1), s));
+    if (p.dense) {
+        // every earlier key: 0 .. t0-1 for each mask
+        an->h_keys.resize((size_t)(hk * t0));
+        an->h_off.resize((size_t)hk + 1);
+        for (int32_t m = 0; m < hk; ++m) {
+            an->h_off[m] = m * t0;
+            for (int64_t j = 0; j < t0; ++j) an->h_keys[(size_t)(m * t0 + j)] = (int32_t)j;
+        }
+        an->h_off[hk] = hk * t0;
+        RIS_CUDA(cudaMallocAsync((void **)&an->keys, sizeof(int32_t) * (size_t)(hk * t0), s));
+        RIS_CUDA(cudaMemcpyAsync(an->keys, an->h_keys.data(), sizeof(int32_t) * (size_t)(hk * t0),
+                                 cudaMemcpyHostToDevice, s));
+        RIS_CUDA(cudaMemcpyAsync(an->off, an->h_off.data(), sizeof(int64_t) * (size_t)(hk + 1),
+                                 cudaMemcpyHostToDevice, s));
+        RIS_CUDA(cudaStreamSynchronize(s));
+        guard.a = nullptr;
+        *out = an;
+        return RIS_OK;
+    }
+    // row t0 of the prefill's mask, without its local window (the decode window replaces it)
+    const int64_t words = (t0 >> 5) + 1;
+    Scratch bits, partials;
+    RIS_CUDA(bits.alloc(sizeof(uint32_t) * (size_t)(hk * words), s));
+    MaskBitsArgs a{};
+    a.single_row = t0;
+    a.N = n_prefill;
+    a.n_seeds = n_seeds;
+    a.per_seed = 0;
+    a.heads_keyed = hk;
+    a.n_masks = hk;
+    a.mode = mode;
+    a.W = 0;
+    a.A = o.n_anchor;
+    a.layer_key = o.layer_key;
+    a.stream = p.stream;
+    a.thr = p.thr;
+    a.B = p.block;
+    a.draws = p.draws;
+    a.words_per_mask = words;
+    a.bitmap = (uint32_t *)bits.p;
+    a.counts = an->off + 1;
+    for (int k = 0; k < n_seeds; ++k) a.seeds.v[k] = seeds[k];
+    if (o.sampler == 1) {
+        RIS_CUDA(cudaMemsetAsync(bits.p, 0, sizeof(uint32_t) * (size_t)(hk * words), s));
+        if (p.draws > 0) RIS_CUDA(launch_mask_draws(a, s));
+        a.or_existing = 1;
+        a.thr = 0;
+    }
+    RIS_CUDA(cudaMemsetAsync(an->off, 0, sizeof(int64_t), s));
+    RIS_CUDA(launch_mask_bits(a, s));
+    RIS_CUDA(partials.alloc(sizeof(int64_t) * (size_t)scan_partials_count(hk), s));
+    RIS_CUDA(launch_scan_inplace(an->off + 1, hk, (int64_t *)partials.p, s));
+    an->h_off.resize((size_t)hk + 1);
+    RIS_CUDA(cudaMemcpyAsync(an->h_off.data(), an->off, sizeof(int64_t) * (size_t)(hk + 1), cudaMemcpyDeviceToHost, s));
+    RIS_CUDA(cudaStreamSynchronize(s));
+    const int64_t total = an->h_off[hk];
+    RIS_CUDA(cudaMallocAsync((void **)&an->keys, sizeof(int32_t) * (size_t)(total > 0 ? total : 1), s));
+    MaskFillArgs f{};
+    f.single_row = t0;
+    f.N = n_prefill;
+    f.n_masks = hk;
+    f.col_bytes = 4;
+    f.words_per_mask = words;
+    f.bitmap = (const uint32_t *)bits.p;
+    f.row_ptr = an->off;
+    f.col = an->keys;
+    RIS_CUDA(launch_mask_fill(f, s));
+    an->h_keys.resize((size_t)total);
+    if (total > 0)
+        RIS_CUDA(cudaMemcpyAsync(an->h_keys.data(), an->keys, sizeof(int32_t) * (size_t)total,
+                                 cudaMemcpyDeviceToHost, s));
+    RIS_CUDA(cudaStreamSynchronize(s));
+    guard.a = nullptr;
+    *out = an;
+    return RIS_OK;
+}
+
+ris_status ris_anchor_info(ris_anchor_t anchor, int64_t *t0, int32_t *heads_keyed, int64_t *n_keys,
+                           const int32_t **keys, const int64_t **offsets)
+{
+    if (anchor == nullptr) return fail(RIS_ERR_INVALID, "anchor is NULL");
+    if (t0) *t0 = anchor->t0;
+    if (heads_keyed) *heads_keyed = anchor->heads_keyed;
+    if (n_keys) *n_keys = anchor->h_off.empty() ? 0 : anchor->h_off.back();
+    if (keys) *keys = anchor->keys;
+    if (offsets) *offsets = anchor->off;
+    return RIS_OK;
+}
+
+ris_status ris_anchor_free(ris_anchor_t anchor)
+{
+    if (anchor == nullptr) return RIS_OK;
+    cudaError_t e = cudaSuccess;
+    if (anchor->keys) e = cudaFreeAsync(anchor->keys, anchor->stream);
+    if (anchor->off) {
+        cudaError_t e2 = cudaFreeAsync(anchor->off, anchor->stream);
+        if (e == cudaSuccess) e = e2;
+    }
+    delete anchor;
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFreeAsync");
+    return RIS_OK;
+}
+
+ris_status ris_rope_split(const void *x, int32_t dtype, int64_t n, int64_t pos0, int32_t heads, int32_t head_dim,
+                          int64_t n_ctx, const ris_rope_cfg *rope, void *hi, void *lo, void *stream)
+{
+    RIS_TRY(check_ptr(x, "x"));
+    RIS_TRY(check_ptr(hi, "hi"));
+    RIS_TRY(check_dtype(dtype, "dtype"));
+    RIS_TRY(check_N(n));
+    RIS_TRY(check_N(n_ctx));
+    if (pos0 < 0 || pos0 + n > 2147483647LL) return fail(RIS_ERR_INVALID, "positions outside [0, 2^31-1)");
+    if (heads < 1) return fail(RIS_ERR_INVALID, "heads must be >= 1");
+    if (head_dim < 8 || (head_dim % 8) || head_dim > 2 * kMaxHeadDimHalf)
+        return fail(RIS_ERR_INVALID, "head_dim %d must be a multiple of 8 in [8, 128]", head_dim);
+    if (dtype == RIS_F32 && lo != nullptr) return fail(RIS_ERR_INVALID, "lo must be NULL for fp32");
+    if (lo != nullptr && !aligned16(lo)) return fail(RIS_ERR_INVALID, "lo is not 16-byte aligned");
+    RIS_TRY(check_rope(rope));
+    RopeArgs a{};
+    double ms = 1.0;
+    if (rope != nullptr && rope->kind != RIS_ROPE_NONE) RIS_TRY(ris_rope_freqs(rope, n_ctx, head_dim, a.f, &ms));
+    a.x_in = x;
+    a.x_out = hi;
+    a.x_out_lo = lo;
+    a.N = n;
+    a.H = heads;
+    a.D = head_dim;
+    a.mscale = (float)ms;
+    a.pos0 = pos0;
+    RIS_CUDA(launch_rope(a, dtype, dtype, reinterpret_cast<cudaStream_t>(stream)));
+    return RIS_OK;
+}
+
+ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, const void *k_lo, const void *v,
+                           int64_t cache_len, int64_t t, int32_t window, int32_t heads, int32_t kv_heads,
+                           int32_t head_dim, int32_t dtype, int32_t out_dtype, int64_t n_ctx,
+                           const ris_rope_cfg *rope, void *out, float *lse, void *stream)
+{
+    if (anchor == nullptr) return fail(RIS_ERR_INVALID, "anchor is NULL");
+    RIS_TRY(validate_attention(q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse));
+    if (k_lo != nullptr && (dtype != RIS_BF16 || !aligned16(k_lo)))
+        return fail(RIS_ERR_INVALID, "k_lo must be NULL for fp32 and 16-byte aligned for bf16");
+    if (kv_heads > kMaxDecodeKvHeads) return fail(RIS_ERR_UNSUPPORTED, "kv_heads %d > %d", kv_heads, kMaxDecodeKvHeads);
+    if (anchor->heads_keyed > 1 && anchor->heads_keyed != kv_heads)
+        return fail(RIS_ERR_INVALID, "anchor keyed for %d KV heads, call has %d", anchor->heads_keyed, kv_heads);
+    if (t < anchor->t0) return fail(RIS_ERR_INVALID, "t=%lld precedes the first generated token %lld", (long long)t,
+                                    (long long)anchor->t0);
+    if (t >= cache_len || cache_len > 2147483647LL)
+        return fail(RIS_ERR_INVALID, "t=%lld must be < cache_len=%lld < 2^31", (long long)t, (long long)cache_len);
+    if (window < 1) return fail(RIS_ERR_INVALID, "window %d must be >= 1", window);
+    RIS_TRY(check_N(n_ctx));
+
+    DecodeArgs a{};
+    a.q = q;
+    a.k = k;
+    a.k_lo = k_lo;
+    a.v = v;
+    a.anchor = anchor->keys;
+    a.anchor_off = anchor->off;
+    a.heads_keyed = anchor->heads_keyed;
+    a.Hq = heads;
+    a.Hkv = kv_heads;
+    a.G = heads / kv_heads;
+    a.D = head_dim;
+    a.t = t;
+    a.win_lo = t - window + 1 > 0 ? t - window + 1 : 0;
+    int64_t n_max = 0;
+    for (int32_t g = 0; g < kv_heads; ++g) {
+        const int32_t m = anchor->heads_keyed > 1 ? g : 0;
+        const int32_t *b = anchor->h_keys.data() + anchor->h_off[m];
+        const int32_t *e = anchor->h_keys.data() + anchor->h_off[m + 1];
+        // anchor keys at or after the window's first key are duplicates of window keys
+        const int64_t nA = std::lower_bound(b, e, (int32_t)a.win_lo) - b;
+        a.n_anchor_keys[g] = (int32_t)nA;
+        n_max = std::max<int64_t>(n_max, nA + (t - a.win_lo + 1));
+    }
+    a.n_chunks = (int32_t)((n_max + kDecodeChunk - 1) / kDecodeChunk);
+    double ms = 1.0;
+    if (rope != nullptr && rope->kind != RIS_ROPE_NONE) RIS_TRY(ris_rope_freqs(rope, n_ctx, head_dim, a.f, &ms));
+    a.mscale = (float)ms;
+    // the keys were rotated with the same scale: scores carry mscale^2
+    a.scale_log2 = (float)(1.4426950408889634074 / std::sqrt((double)head_dim));
+    a.out = out;
+    a.lse = lse;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    prepare_pool_once();
+    Scratch po, pml;
+    const size_t slots = (size_t)kv_heads * a.n_chunks * a.G;
+    RIS_CUDA(po.alloc(sizeof(float) * slots * head_dim, s));
+    RIS_CUDA(pml.alloc(sizeof(float2) * slots, s));
+    a.part_o = (float *)po.p;
+    a.part_ml = (float2 *)pml.p;
+    RIS_CUDA(launch_decode(a, dtype, out_dtype, s));
+    return RIS_OK;
 }
 
 }  // extern "C"

@@ -33,6 +33,8 @@ struct MaskBitsArgs {
     int64_t B;            // Structural block size
     int64_t draws;        // index-draw sampler: draws per row and seed
     int32_t or_existing;  // 1: OR into the words already in the bitmap (index draws were set)
+    int64_t single_row;   // -1: rows 0..N-1; >= 0: only this row, one CTA per mask, its words at
+                          // bitmap + m * words_per_mask and its count at counts[m]
     int64_t words_per_mask;
     uint32_t *bitmap;     // [n_masks][words_per_mask]
     int64_t *counts;      // counts[m * N + i] (row_ptr + 1)
@@ -48,6 +50,7 @@ struct MaskFillArgs {
     const uint32_t *bitmap;
     const int64_t *row_ptr;
     void *col;
+    int64_t single_row;   // as MaskBitsArgs::single_row (keys of mask m from col + row_ptr[m])
 };
 
 // Arguments of the RoPE kernels: x_out[p][h][c], x_out[p][h][c + D/2] from x_in.
@@ -60,6 +63,7 @@ struct RopeArgs {
     int32_t D;
     double f[kMaxHeadDimHalf];  // rotation frequencies (fp64)
     float mscale;
+    int64_t pos0;    // position of token 0 of x_in
 };
 
 // Arguments of the attention kernels. One warp handles one task = (set s, row i, KV head g).
@@ -85,6 +89,37 @@ struct AttnArgs {
     int64_t n_tasks;       // n_sets * N * Hkv
 };
 
+// Arguments of the Hybrid Anchor decode kernels (one generated token at position t). The
+// key set of KV head g is the first n_anchor_keys[g] keys of its anchor list followed by the
+// window win_lo .. t; it is cut into chunks of kDecodeChunk keys, one CTA per (chunk, g).
+constexpr int kDecodeChunk = 32;
+constexpr int kMaxDecodeKvHeads = 64;
+
+struct DecodeArgs {
+    const void *q;             // [Hq][D] query of the token, not rotated (dtype)
+    const void *k;             // [T][Hkv][D] rotated keys: bf16 high parts, or fp32
+    const void *k_lo;          // bf16 low parts (k~ = k + k_lo), or null
+    const void *v;             // [T][Hkv][D]
+    const int32_t *anchor;     // anchor keys, ascending; mask m: anchor[anchor_off[m] .. anchor_off[m+1])
+    const int64_t *anchor_off;
+    int32_t heads_keyed;       // 1, or Hkv for per-head anchors
+    int32_t Hq;
+    int32_t Hkv;
+    int32_t G;
+    int32_t D;
+    int32_t n_chunks;          // chunks per KV head (grid.x)
+    int64_t t;
+    int64_t win_lo;            // first key of the local window, max(0, t - W + 1)
+    int32_t n_anchor_keys[kMaxDecodeKvHeads];  // anchor keys below win_lo, per KV head
+    double f[kMaxHeadDimHalf]; // rotation frequencies of q (fp64)
+    float mscale;
+    float scale_log2;          // log2(e) / sqrt(D)
+    float *part_o;             // [Hkv * n_chunks][G][D] partial outputs
+    float2 *part_ml;           // [Hkv * n_chunks][G] partial (max, sum) in the log2 domain
+    void *out;                 // [Hq][D]
+    float *lse;                // [Hq] or null
+};
+
 // Library-wide kernel launch counter (ris_launch_count).
 void note_launch(int n = 1);
 
@@ -97,6 +132,9 @@ cudaError_t launch_mask_draws(const MaskBitsArgs &a, cudaStream_t s);
 cudaError_t launch_scan_inplace(int64_t *x, int64_t n, int64_t *partials, cudaStream_t s);
 int64_t scan_partials_count(int64_t n);
 cudaError_t launch_mask_fill(const MaskFillArgs &a, cudaStream_t s);
+
+// Decode step: partial softmax per (chunk, KV head), then one combine per query head.
+cudaError_t launch_decode(const DecodeArgs &a, int dtype, int out_dtype, cudaStream_t s);
 
 // dtype_in / dtype_out are ris_dtype values.
 cudaError_t launch_rope(const RopeArgs &a, int dtype_in, int dtype_out, cudaStream_t s);

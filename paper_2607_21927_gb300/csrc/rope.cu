@@ -39,7 +39,7 @@ __global__ void k_rope(const RopeArgs a)
     const int64_t p = (int64_t)blockIdx.x * kRopeTokens + threadIdx.y;
     if (p >= a.N || c >= half) return;
     // angle in fp64, reduced by the nearest multiple of 2 pi (two-term 2 pi)
-    const double ang = (double)p * a.f[c];
+    const double ang = (double)(p + a.pos0) * a.f[c];
     const double n = rint(ang * 0.15915494309189533577);  // 1 / (2 pi)
     double red = fma(-n, 6.28318530717958623200, ang);  // 2 pi, high part
     red = fma(-n, 2.4492935982947064e-16, red);            // 2 pi, low part

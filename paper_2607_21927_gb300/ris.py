@@ -99,6 +99,16 @@ _SIGS = {
     "ris_device_status": [ctypes.c_void_p],
     "ris_attention_design": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32],
     "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
+    "ris_decode_anchor": [ctypes.c_int64, ctypes.c_int32, ctypes.c_int32, ctypes.c_double, ctypes.c_void_p,
+                          ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p],
+    "ris_anchor_info": [ctypes.c_void_p] * 6,
+    "ris_anchor_free": [ctypes.c_void_p],
+    "ris_rope_split": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32,
+                       ctypes.c_int32, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                       ctypes.c_void_p],
+    "ris_decode_step": [ctypes.c_void_p] * 5 + [ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                        ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
+                        ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p],
     "ris_probe_l2_read": [ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p],
     "ris_probe_ffma": [ctypes.c_void_p, ctypes.c_void_p],
     "ris_probe_l2_bytes": [ctypes.c_void_p],
@@ -399,3 +409,76 @@ def ris_attention_masked_noalloc(mask: Mask, q, k, v, out: torch.Tensor, rope: O
         mask.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(out), Hq, Hkv, D, _dtype(q), _dtype(out), _ref(rope),
         _ptr(lse), _stream(stream)))
     return out
+
+
+# ----------------------------------------------------------------------------- Hybrid Anchor decode
+class Anchor:
+    """The frozen Stochastic Anchor of a generation (ris_decode_anchor); freed by ``free()``."""
+
+    def __init__(self, handle: ctypes.c_void_p, kv_heads: int):
+        self.handle = handle
+        self.kv_heads = kv_heads
+
+    def info(self):
+        """(t0, heads_keyed, n_keys, keys device tensor int64, offsets device tensor int64)."""
+        t0, hk, n = ctypes.c_int64(), ctypes.c_int32(), ctypes.c_int64()
+        keys, off = ctypes.c_void_p(), ctypes.c_void_p()
+        _check("ris_anchor_info", lib().ris_anchor_info(self.handle, ctypes.byref(t0), ctypes.byref(hk),
+                                                        ctypes.byref(n), ctypes.byref(keys), ctypes.byref(off)))
+        k = _device_view(keys.value, n.value, torch.int32).to(torch.int64)
+        o = _device_view(off.value, hk.value + 1, torch.int64)
+        return t0.value, hk.value, n.value, k, o
+
+    def free(self) -> None:
+        if self.handle:
+            _check("ris_anchor_free", lib().ris_anchor_free(self.handle))
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def ris_decode_anchor(n_prefill: int, kv_heads: int, mode: int, density: float, seeds: Sequence[int],
+                      opts: Optional[MaskOpts] = None, stream=None) -> Anchor:
+    arr, n = _seeds(seeds)
+    h = ctypes.c_void_p()
+    _check("ris_decode_anchor", lib().ris_decode_anchor(int(n_prefill), int(kv_heads), int(mode), float(density),
+                                                        arr, n, _ref(opts), ctypes.byref(h), _stream(stream)))
+    return Anchor(h, kv_heads)
+
+
+def ris_rope_split(x: torch.Tensor, n_ctx: int, rope: Optional[RopeCfg], pos0: int = 0, hi=None, lo=None,
+                   split: bool = True, stream=None):
+    """Rotated copy of x [n, H, D] at positions pos0.. as (hi, lo); lo (bf16 only) carries the
+    residual of the bf16 rounding when split is set, else None."""
+    assert x.is_cuda and x.is_contiguous() and x.dim() == 3
+    n, H, D = x.shape
+    hi = _alloc_out(hi, x.shape, x.dtype, x.device)
+    if split and x.dtype == torch.bfloat16:
+        lo = _alloc_out(lo, x.shape, torch.bfloat16, x.device)
+    else:
+        lo = None
+    _check("ris_rope_split", lib().ris_rope_split(_ptr(x), _dtype(x), int(n), int(pos0), int(H), int(D), int(n_ctx),
+                                                  _ref(rope), _ptr(hi), _ptr(lo), _stream(stream)))
+    return hi, lo
+
+
+def ris_decode_step(anchor: Anchor, q: torch.Tensor, k: torch.Tensor, k_lo: Optional[torch.Tensor],
+                    v: torch.Tensor, t: int, window: int, n_ctx: int, rope: Optional[RopeCfg] = None,
+                    out=None, out_dtype=None, return_lse: bool = False, stream=None):
+    """q [Hq, D] of the token at position t (not rotated); k/k_lo/v the rotated cache [T, Hkv, D]."""
+    assert q.is_cuda and q.is_contiguous() and q.dim() == 2
+    for x in (k, v) + ((k_lo,) if k_lo is not None else ()):
+        assert x.is_cuda and x.is_contiguous() and x.dim() == 3 and x.shape == k.shape
+    Hq, D = q.shape
+    T, Hkv, _ = k.shape
+    out = _alloc_out(out, (Hq, D), out_dtype or q.dtype, q.device)
+    lse = torch.empty(Hq, dtype=torch.float32, device=q.device) if return_lse else None
+    _check("ris_decode_step", lib().ris_decode_step(
+        anchor.handle, _ptr(q), _ptr(k), _ptr(k_lo), _ptr(v), int(T), int(t), int(window), int(Hq), int(Hkv), int(D),
+        _dtype(q), _dtype(out), int(n_ctx), _ref(rope), _ptr(out), _ptr(lse), _stream(stream)))
+    return (out, lse) if return_lse else out
+
