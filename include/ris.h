@@ -288,14 +288,23 @@ ris_status ris_rope_split(const void *x, int32_t dtype, int64_t n, int64_t pos0,
  * bf16, may be NULL) and v: the cache [cache_len][kv_heads][head_dim] holding positions
  * 0 .. cache_len-1 with rotated keys (ris_rope_split); it must already hold the token t's own
  * key and value. out: [heads][head_dim] (out_dtype); lse: [heads] natural-log sum of
- * exp(score) or NULL. Scores and probabilities are fp32. Asynchronous; per-step scratch comes
- * from the stream-ordered pool. Errors: RIS_ERR_INVALID (t < t0, t >= cache_len, window < 1,
- * shapes, pointers, anchor keyed for another kv_heads), RIS_ERR_UNSUPPORTED (kv_heads > 64),
- * RIS_ERR_CUDA. */
+ * exp(score) or NULL. Scores and probabilities are fp32.
+ * Position: t (host value) when t_dev is NULL; otherwise the int64 at t_dev (device memory,
+ * 8-byte aligned) is read when the step runs and t is ignored, and with advance != 0 the
+ * step adds 1 to *t_dev when it has finished. Nothing in the launch then depends on the
+ * position, so a captured CUDA graph of a token's steps can be replayed token after token.
+ * A device-side position outside [t0, cache_len) makes the step attend to nothing (undefined
+ * output) and is reported by ris_device_status as RIS_ERR_INVALID.
+ * Partial results live in a buffer owned by the anchor, grown by the first call of a larger
+ * shape (stream-ordered pool allocation: make that call before any stream capture); steps on
+ * one anchor must therefore be ordered on the GPU (one stream, or events between streams).
+ * Errors: RIS_ERR_INVALID (host t outside [t0, cache_len), window < 1, shapes, pointers,
+ * anchor keyed for another kv_heads, advance without t_dev), RIS_ERR_UNSUPPORTED
+ * (kv_heads > 64), RIS_ERR_CUDA. */
 ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, const void *k_lo, const void *v,
-                           int64_t cache_len, int64_t t, int32_t window, int32_t heads, int32_t kv_heads,
-                           int32_t head_dim, int32_t dtype, int32_t out_dtype, int64_t n_ctx,
-                           const ris_rope_cfg *rope, void *out, float *lse, void *stream);
+                           int64_t cache_len, int64_t t, int64_t *t_dev, int32_t advance, int32_t window,
+                           int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t dtype, int32_t out_dtype,
+                           int64_t n_ctx, const ris_rope_cfg *rope, void *out, float *lse, void *stream);
 
 /* ---- Measurement support (the paper has no counterpart) -------------------------------------
  * Small kernels that measure the ceilings the attention kernels are compared against, for the

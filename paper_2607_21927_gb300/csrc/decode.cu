@@ -4,9 +4,11 @@
 // Window t - W < j <= t, with one softmax over the merged set.
 //
 // The merge needs no sort: the anchor keys at or above the window's first key are exactly the
-// duplicates, so the merged set is the anchor list cut at win_lo (the host finds the cut by
-// binary search in its copy of the list) followed by the contiguous window. Key number k of
-// KV head g is therefore anchor[k] for k < n_anchor_keys[g], else win_lo + (k - n_anchor_keys[g]).
+// duplicates, so the merged set is the anchor list cut at win_lo followed by the contiguous
+// window. The cut is one load from a rank table built with the anchor (rank[j] = anchor keys
+// below j). Key number k of KV head g is anchor[k] for k < nA, else win_lo + (k - nA).
+// Nothing in the launch depends on t, so the position may live in device memory and a
+// captured CUDA graph of a whole token can be replayed token after token.
 //
 //   k_decode_partial : one CTA per (chunk of 32 keys, KV head): rotates the G query heads of
 //                      the KV head at position t (fp64 angle, as the prefill RoPE), stages the
@@ -27,6 +29,8 @@
 
 namespace ris {
 namespace {
+
+__device__ unsigned int g_ris_decode_error;
 
 constexpr int kDecodeThreads = 128;
 constexpr int kMaxG = 8;
@@ -59,26 +63,34 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
 
     const int g = blockIdx.y, chunk = blockIdx.x, tid = threadIdx.x;
     const int D = a.D, G = a.G, half = D >> 1;
-    const int64_t nA = a.n_anchor_keys[g];
-    const int64_t n = nA + (a.t - a.win_lo + 1);
-    const int64_t k0 = (int64_t)chunk * kDecodeChunk;
     const int64_t slot = (int64_t)g * a.n_chunks + chunk;
-    if (k0 >= n) {  // this KV head has fewer chunks: an empty partial
+    const int64_t t = a.t_dev != nullptr ? *a.t_dev : a.t;
+    if (t < a.t0 || t >= a.cache_len) {  // only reachable through t_dev: flag it, attend to nothing
+        if (tid == 0 && chunk == 0 && g == 0) atomicOr(&g_ris_decode_error, 2u);
+        for (int h = tid; h < G; h += kDecodeThreads) a.part_ml[slot * G + h] = make_float2(-INFINITY, 0.f);
+        return;
+    }
+    const int64_t win_lo = t - a.window + 1 > 0 ? t - a.window + 1 : 0;
+    const int m = a.heads_keyed > 1 ? g : 0;
+    const int64_t nA = a.rank[(int64_t)m * (a.t0 + 1) + (win_lo < a.t0 ? win_lo : a.t0)];
+    const int64_t n = nA + (t - win_lo + 1);
+    const int64_t k0 = (int64_t)chunk * kDecodeChunk;
+    if (k0 >= n) {  // fewer keys than the grid covers: an empty partial
         for (int h = tid; h < G; h += kDecodeThreads) a.part_ml[slot * G + h] = make_float2(-INFINITY, 0.f);
         return;
     }
     const int nk = (int)((n - k0) < kDecodeChunk ? (n - k0) : kDecodeChunk);
-    const int32_t *anchor = a.anchor + a.anchor_off[a.heads_keyed > 1 ? g : 0];
+    const int32_t *anchor = a.anchor + a.anchor_off[m];
     if (tid < kDecodeChunk) {
         const int64_t kk = k0 + tid;
         int64_t key = 0;  // rows past the set read key 0 and are masked out below
-        if (kk < n) key = kk < nA ? (int64_t)anchor[kk] : a.win_lo + (kk - nA);
+        if (kk < n) key = kk < nA ? (int64_t)anchor[kk] : win_lo + (kk - nA);
         keys[tid] = (int32_t)key;
     }
     for (int idx = tid; idx < G * half; idx += kDecodeThreads) {
         const int h = idx / half, c = idx - h * half;
         float sn, cs;
-        sincos_reduced((double)a.t * a.f[c], &sn, &cs);
+        sincos_reduced((double)t * a.f[c], &sn, &cs);
         const T *qp = reinterpret_cast<const T *>(a.q) + (int64_t)(g * G + h) * D;
         const float x0 = ldf(qp + c), x1 = ldf(qp + c + half);
         qs[h][c] = fmaf(x0, cs, -x1 * sn) * a.mscale;
@@ -145,9 +157,47 @@ __global__ void k_decode_combine(const DecodeArgs a)
     else
         reinterpret_cast<__nv_bfloat16 *>(a.out)[(int64_t)h * a.D + c] = __float2bfloat16_rn(o);
     if (c == 0 && a.lse != nullptr) a.lse[h] = (M + log2f(L)) * 0.69314718055994530942f;
+    // the partial kernel, the only reader of t, has finished: move to the next position
+    if (a.advance && a.t_dev != nullptr && h == 0 && c == 0) *a.t_dev += 1;
+}
+
+// rank[m][j] = lower_bound(keys of list m, j) - start, for j = 0 .. t0
+__global__ void k_anchor_rank(const int32_t *keys, const int64_t *off, int32_t n_masks, int64_t t0, int32_t *rank)
+{
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (int64_t)n_masks * (t0 + 1)) return;
+    const int32_t m = (int32_t)(idx / (t0 + 1));
+    const int64_t j = idx - (int64_t)m * (t0 + 1);
+    int64_t lo = off[m], hi = off[m + 1];
+    const int64_t b = lo;
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if ((int64_t)keys[mid] < j)
+            lo = mid + 1;
+        else
+            hi = mid;
+    }
+    rank[idx] = (int32_t)(lo - b);
 }
 
 }  // namespace
+
+cudaError_t launch_anchor_rank(const int32_t *keys, const int64_t *off, int32_t n_masks, int64_t t0, int32_t *rank,
+                               cudaStream_t s)
+{
+    const int64_t n = (int64_t)n_masks * (t0 + 1);
+    k_anchor_rank<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(keys, off, n_masks, t0, rank);
+    note_launch();
+    return cudaGetLastError();
+}
+
+unsigned int read_decode_error()
+{
+    unsigned int v = 0, zero = 0;
+    if (cudaMemcpyFromSymbol(&v, g_ris_decode_error, sizeof(v)) != cudaSuccess) return 0;
+    if (v != 0) cudaMemcpyToSymbol(g_ris_decode_error, &zero, sizeof(zero));
+    return v;
+}
 
 cudaError_t launch_decode(const DecodeArgs &a, int dtype, int out_dtype, cudaStream_t s)
 {

@@ -50,8 +50,11 @@ struct ris_anchor_s {
     int32_t heads_keyed = 1, kv_heads = 1;
     int32_t *keys = nullptr;  // device, ascending per mask
     int64_t *off = nullptr;   // device, heads_keyed + 1 offsets
-    std::vector<int32_t> h_keys;
+    int32_t *rank = nullptr;  // device, [heads_keyed][t0 + 1]: keys below j
+    int64_t max_keys = 0;     // longest list
     std::vector<int64_t> h_off;
+    void *scratch = nullptr;  // decode partials, reused by every step on this anchor
+    size_t scratch_bytes = 0;
     ris_params params{};
     cudaStream_t stream = nullptr;
 };
@@ -677,8 +680,11 @@ ris_status ris_device_status(void *stream)
     unsigned int word = 0, tile_word = 0;
     RIS_CUDA(read_device_error(&word, reinterpret_cast<cudaStream_t>(stream)));
     RIS_CUDA(read_tile_error(&tile_word));
+    const unsigned int decode_word = read_decode_error();
     word |= tile_word;
     if (word != 0u) return fail(RIS_ERR_DEVICE_TIMEOUT, "a device-side wait gave up (error word 0x%x)", word);
+    if (decode_word != 0u)
+        return fail(RIS_ERR_INVALID, "a decode step read a position outside [t0, cache_len) from t_dev");
     return RIS_OK;
 }
 
@@ -750,26 +756,8 @@ ris_status ris_decode_anchor(int64_t n_prefill, int32_t kv_heads, int32_t mode, 
     an->stream = s;
     prepare_pool_once();
     RIS_CUDA(cudaMallocAsync((void **)&an->off, sizeof(int64_t) * (size_t)(hk + 1), s));
-    if (p.dense) {
-        // every earlier key: 0 .. t0-1 for each mask
-        an->h_keys.resize((size_t)(hk * t0));
-        an->h_off.resize((size_t)hk + 1);
-        for (int32_t m = 0; m < hk; ++m) {
-            an->h_off[m] = m * t0;
-            for (int64_t j = 0; j < t0; ++j) an->h_keys[(size_t)(m * t0 + j)] = (int32_t)j;
-        }
-        an->h_off[hk] = hk * t0;
-        RIS_CUDA(cudaMallocAsync((void **)&an->keys, sizeof(int32_t) * (size_t)(hk * t0), s));
-        RIS_CUDA(cudaMemcpyAsync(an->keys, an->h_keys.data(), sizeof(int32_t) * (size_t)(hk * t0),
-                                 cudaMemcpyHostToDevice, s));
-        RIS_CUDA(cudaMemcpyAsync(an->off, an->h_off.data(), sizeof(int64_t) * (size_t)(hk + 1),
-                                 cudaMemcpyHostToDevice, s));
-        RIS_CUDA(cudaStreamSynchronize(s));
-        guard.a = nullptr;
-        *out = an;
-        return RIS_OK;
-    }
-    // row t0 of the prefill's mask, without its local window (the decode window replaces it)
+    // row t0 of the prefill's mask, without its local window (the decode window replaces it);
+    // the dense mode keeps every earlier key
     const int64_t words = (t0 >> 5) + 1;
     Scratch bits, partials;
     RIS_CUDA(bits.alloc(sizeof(uint32_t) * (size_t)(hk * words), s));
@@ -785,14 +773,15 @@ ris_status ris_decode_anchor(int64_t n_prefill, int32_t kv_heads, int32_t mode, 
     a.A = o.n_anchor;
     a.layer_key = o.layer_key;
     a.stream = p.stream;
-    a.thr = p.thr;
+    a.thr = p.dense ? (uint64_t(1) << 32) : p.thr;
+    a.mode = p.dense ? RIS_MODE_STOCHASTIC : mode;
     a.B = p.block;
     a.draws = p.draws;
     a.words_per_mask = words;
     a.bitmap = (uint32_t *)bits.p;
     a.counts = an->off + 1;
     for (int k = 0; k < n_seeds; ++k) a.seeds.v[k] = seeds[k];
-    if (o.sampler == 1) {
+    if (o.sampler == 1 && !p.dense) {
         RIS_CUDA(cudaMemsetAsync(bits.p, 0, sizeof(uint32_t) * (size_t)(hk * words), s));
         if (p.draws > 0) RIS_CUDA(launch_mask_draws(a, s));
         a.or_existing = 1;
@@ -817,10 +806,9 @@ ris_status ris_decode_anchor(int64_t n_prefill, int32_t kv_heads, int32_t mode, 
     f.row_ptr = an->off;
     f.col = an->keys;
     RIS_CUDA(launch_mask_fill(f, s));
-    an->h_keys.resize((size_t)total);
-    if (total > 0)
-        RIS_CUDA(cudaMemcpyAsync(an->h_keys.data(), an->keys, sizeof(int32_t) * (size_t)total,
-                                 cudaMemcpyDeviceToHost, s));
+    RIS_CUDA(cudaMallocAsync((void **)&an->rank, sizeof(int32_t) * (size_t)(hk * (t0 + 1)), s));
+    RIS_CUDA(launch_anchor_rank(an->keys, an->off, hk, t0, an->rank, s));
+    for (int32_t m = 0; m < hk; ++m) an->max_keys = std::max(an->max_keys, an->h_off[m + 1] - an->h_off[m]);
     RIS_CUDA(cudaStreamSynchronize(s));
     guard.a = nullptr;
     *out = an;
@@ -843,9 +831,9 @@ ris_status ris_anchor_free(ris_anchor_t anchor)
 {
     if (anchor == nullptr) return RIS_OK;
     cudaError_t e = cudaSuccess;
-    if (anchor->keys) e = cudaFreeAsync(anchor->keys, anchor->stream);
-    if (anchor->off) {
-        cudaError_t e2 = cudaFreeAsync(anchor->off, anchor->stream);
+    for (void *p : {(void *)anchor->keys, (void *)anchor->off, (void *)anchor->rank, anchor->scratch}) {
+        if (p == nullptr) continue;
+        cudaError_t e2 = cudaFreeAsync(p, anchor->stream);
         if (e == cudaSuccess) e = e2;
     }
     delete anchor;
@@ -884,9 +872,9 @@ ris_status ris_rope_split(const void *x, int32_t dtype, int64_t n, int64_t pos0,
 }
 
 ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, const void *k_lo, const void *v,
-                           int64_t cache_len, int64_t t, int32_t window, int32_t heads, int32_t kv_heads,
-                           int32_t head_dim, int32_t dtype, int32_t out_dtype, int64_t n_ctx,
-                           const ris_rope_cfg *rope, void *out, float *lse, void *stream)
+                           int64_t cache_len, int64_t t, int64_t *t_dev, int32_t advance, int32_t window,
+                           int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t dtype, int32_t out_dtype,
+                           int64_t n_ctx, const ris_rope_cfg *rope, void *out, float *lse, void *stream)
 {
     if (anchor == nullptr) return fail(RIS_ERR_INVALID, "anchor is NULL");
     RIS_TRY(validate_attention(q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse));
@@ -895,10 +883,15 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     if (kv_heads > kMaxDecodeKvHeads) return fail(RIS_ERR_UNSUPPORTED, "kv_heads %d > %d", kv_heads, kMaxDecodeKvHeads);
     if (anchor->heads_keyed > 1 && anchor->heads_keyed != kv_heads)
         return fail(RIS_ERR_INVALID, "anchor keyed for %d KV heads, call has %d", anchor->heads_keyed, kv_heads);
-    if (t < anchor->t0) return fail(RIS_ERR_INVALID, "t=%lld precedes the first generated token %lld", (long long)t,
-                                    (long long)anchor->t0);
-    if (t >= cache_len || cache_len > 2147483647LL)
-        return fail(RIS_ERR_INVALID, "t=%lld must be < cache_len=%lld < 2^31", (long long)t, (long long)cache_len);
+    if (cache_len <= anchor->t0 || cache_len > 2147483647LL)
+        return fail(RIS_ERR_INVALID, "cache_len=%lld must exceed t0=%lld and be < 2^31", (long long)cache_len,
+                    (long long)anchor->t0);
+    if (t_dev == nullptr && (t < anchor->t0 || t >= cache_len))
+        return fail(RIS_ERR_INVALID, "t=%lld outside [t0=%lld, cache_len=%lld)", (long long)t, (long long)anchor->t0,
+                    (long long)cache_len);
+    if (t_dev != nullptr && (reinterpret_cast<uintptr_t>(t_dev) & 7u))
+        return fail(RIS_ERR_INVALID, "t_dev is not 8-byte aligned");
+    if (advance != 0 && t_dev == nullptr) return fail(RIS_ERR_INVALID, "advance needs t_dev");
     if (window < 1) return fail(RIS_ERR_INVALID, "window %d must be >= 1", window);
     RIS_TRY(check_N(n_ctx));
 
@@ -909,24 +902,20 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     a.v = v;
     a.anchor = anchor->keys;
     a.anchor_off = anchor->off;
+    a.rank = anchor->rank;
+    a.t0 = anchor->t0;
+    a.cache_len = cache_len;
     a.heads_keyed = anchor->heads_keyed;
     a.Hq = heads;
     a.Hkv = kv_heads;
     a.G = heads / kv_heads;
     a.D = head_dim;
+    a.window = window;
+    a.advance = advance;
     a.t = t;
-    a.win_lo = t - window + 1 > 0 ? t - window + 1 : 0;
-    int64_t n_max = 0;
-    for (int32_t g = 0; g < kv_heads; ++g) {
-        const int32_t m = anchor->heads_keyed > 1 ? g : 0;
-        const int32_t *b = anchor->h_keys.data() + anchor->h_off[m];
-        const int32_t *e = anchor->h_keys.data() + anchor->h_off[m + 1];
-        // anchor keys at or after the window's first key are duplicates of window keys
-        const int64_t nA = std::lower_bound(b, e, (int32_t)a.win_lo) - b;
-        a.n_anchor_keys[g] = (int32_t)nA;
-        n_max = std::max<int64_t>(n_max, nA + (t - a.win_lo + 1));
-    }
-    a.n_chunks = (int32_t)((n_max + kDecodeChunk - 1) / kDecodeChunk);
+    a.t_dev = t_dev;
+    // the grid covers the largest merged set (every anchor key plus a full window), whatever t is
+    a.n_chunks = (int32_t)((anchor->max_keys + window + kDecodeChunk - 1) / kDecodeChunk);
     double ms = 1.0;
     if (rope != nullptr && rope->kind != RIS_ROPE_NONE) RIS_TRY(ris_rope_freqs(rope, n_ctx, head_dim, a.f, &ms));
     a.mscale = (float)ms;
@@ -935,14 +924,25 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     a.out = out;
     a.lse = lse;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    prepare_pool_once();
-    Scratch po, pml;
     const size_t slots = (size_t)kv_heads * a.n_chunks * a.G;
-    RIS_CUDA(po.alloc(sizeof(float) * slots * head_dim, s));
-    RIS_CUDA(pml.alloc(sizeof(float2) * slots, s));
-    a.part_o = (float *)po.p;
-    a.part_ml = (float2 *)pml.p;
+    const size_t o_bytes = (sizeof(float) * slots * head_dim + 255) & ~size_t(255);
+    const size_t need = o_bytes + sizeof(float2) * slots;
+    if (need > anchor->scratch_bytes) {
+        // grow the anchor's partials buffer (stream-ordered; the first call of a shape allocates)
+        prepare_pool_once();
+        if (anchor->scratch) RIS_CUDA(cudaFreeAsync(anchor->scratch, s));
+        anchor->scratch = nullptr;
+        anchor->scratch_bytes = 0;
+        RIS_CUDA(cudaMallocAsync(&anchor->scratch, need, s));
+        anchor->scratch_bytes = need;
+        anchor->stream = s;
+    }
+    a.part_o = (float *)anchor->scratch;
+    a.part_ml = (float2 *)((char *)anchor->scratch + o_bytes);
+    const auto ev = timer_pair();
+    if (ev.first) RIS_CUDA(cudaEventRecord(ev.first, s));
     RIS_CUDA(launch_decode(a, dtype, out_dtype, s));
+    if (ev.second) RIS_CUDA(cudaEventRecord(ev.second, s));
     return RIS_OK;
 }
 

@@ -90,8 +90,10 @@ struct AttnArgs {
 };
 
 // Arguments of the Hybrid Anchor decode kernels (one generated token at position t). The
-// key set of KV head g is the first n_anchor_keys[g] keys of its anchor list followed by the
-// window win_lo .. t; it is cut into chunks of kDecodeChunk keys, one CTA per (chunk, g).
+// key set of KV head g is its anchor keys below win_lo = max(0, t - W + 1) (their count is
+// rank[min(win_lo, t0)]) followed by the window win_lo .. t; it is cut into chunks of
+// kDecodeChunk keys, one CTA per (chunk, g). The grid covers the largest possible set
+// (anchor size + W), so it does not depend on t, and t may be read from device memory.
 constexpr int kDecodeChunk = 32;
 constexpr int kMaxDecodeKvHeads = 64;
 
@@ -102,15 +104,20 @@ struct DecodeArgs {
     const void *v;             // [T][Hkv][D]
     const int32_t *anchor;     // anchor keys, ascending; mask m: anchor[anchor_off[m] .. anchor_off[m+1])
     const int64_t *anchor_off;
+    const int32_t *rank;       // [heads_keyed][t0 + 1]: anchor keys of mask m below j
+    int64_t t0;                // first generated position (the prefill length)
+    int64_t cache_len;
     int32_t heads_keyed;       // 1, or Hkv for per-head anchors
     int32_t Hq;
     int32_t Hkv;
     int32_t G;
     int32_t D;
     int32_t n_chunks;          // chunks per KV head (grid.x)
-    int64_t t;
-    int64_t win_lo;            // first key of the local window, max(0, t - W + 1)
-    int32_t n_anchor_keys[kMaxDecodeKvHeads];  // anchor keys below win_lo, per KV head
+    int32_t window;            // W >= 1
+    int32_t advance;           // with t_dev: the combine kernel adds 1 to *t_dev when done
+    int64_t t;                 // position of the token (when t_dev is null)
+    int64_t *t_dev;            // device position of the token, or null
+    unsigned int *error;       // device error word: bit 1 = t outside [t0, cache_len)
     double f[kMaxHeadDimHalf]; // rotation frequencies of q (fp64)
     float mscale;
     float scale_log2;          // log2(e) / sqrt(D)
@@ -135,6 +142,11 @@ cudaError_t launch_mask_fill(const MaskFillArgs &a, cudaStream_t s);
 
 // Decode step: partial softmax per (chunk, KV head), then one combine per query head.
 cudaError_t launch_decode(const DecodeArgs &a, int dtype, int out_dtype, cudaStream_t s);
+// rank[m][j] = number of keys of anchor list m below j, j = 0 .. t0
+cudaError_t launch_anchor_rank(const int32_t *keys, const int64_t *off, int32_t n_masks, int64_t t0, int32_t *rank,
+                               cudaStream_t s);
+// Reads and clears the decode error word (bit 1: a step's device-side t was out of range).
+unsigned int read_decode_error();
 
 // dtype_in / dtype_out are ris_dtype values.
 cudaError_t launch_rope(const RopeArgs &a, int dtype_in, int dtype_out, cudaStream_t s);

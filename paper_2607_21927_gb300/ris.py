@@ -106,9 +106,10 @@ _SIGS = {
     "ris_rope_split": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32,
                        ctypes.c_int32, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                        ctypes.c_void_p],
-    "ris_decode_step": [ctypes.c_void_p] * 5 + [ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
-                        ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
-                        ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p],
+    "ris_decode_step": [ctypes.c_void_p] * 5 + [ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p, ctypes.c_int32,
+                        ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                        ctypes.c_int32, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                        ctypes.c_void_p],
     "ris_probe_l2_read": [ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p],
     "ris_probe_ffma": [ctypes.c_void_p, ctypes.c_void_p],
     "ris_probe_l2_bytes": [ctypes.c_void_p],
@@ -468,8 +469,11 @@ def ris_rope_split(x: torch.Tensor, n_ctx: int, rope: Optional[RopeCfg], pos0: i
 
 def ris_decode_step(anchor: Anchor, q: torch.Tensor, k: torch.Tensor, k_lo: Optional[torch.Tensor],
                     v: torch.Tensor, t: int, window: int, n_ctx: int, rope: Optional[RopeCfg] = None,
-                    out=None, out_dtype=None, return_lse: bool = False, stream=None):
-    """q [Hq, D] of the token at position t (not rotated); k/k_lo/v the rotated cache [T, Hkv, D]."""
+                    out=None, out_dtype=None, return_lse: bool = False, t_dev: Optional[torch.Tensor] = None,
+                    advance: bool = False, stream=None):
+    """q [Hq, D] of the token at position t (not rotated); k/k_lo/v the rotated cache [T, Hkv, D].
+    With t_dev (a one-element int64 CUDA tensor) the position is read on the device instead of t,
+    and advance adds 1 to it once the step has run."""
     assert q.is_cuda and q.is_contiguous() and q.dim() == 2
     for x in (k, v) + ((k_lo,) if k_lo is not None else ()):
         assert x.is_cuda and x.is_contiguous() and x.dim() == 3 and x.shape == k.shape
@@ -477,8 +481,11 @@ def ris_decode_step(anchor: Anchor, q: torch.Tensor, k: torch.Tensor, k_lo: Opti
     T, Hkv, _ = k.shape
     out = _alloc_out(out, (Hq, D), out_dtype or q.dtype, q.device)
     lse = torch.empty(Hq, dtype=torch.float32, device=q.device) if return_lse else None
+    if t_dev is not None:
+        assert t_dev.is_cuda and t_dev.dtype == torch.int64 and t_dev.numel() == 1
     _check("ris_decode_step", lib().ris_decode_step(
-        anchor.handle, _ptr(q), _ptr(k), _ptr(k_lo), _ptr(v), int(T), int(t), int(window), int(Hq), int(Hkv), int(D),
-        _dtype(q), _dtype(out), int(n_ctx), _ref(rope), _ptr(out), _ptr(lse), _stream(stream)))
+        anchor.handle, _ptr(q), _ptr(k), _ptr(k_lo), _ptr(v), int(T), int(t), _ptr(t_dev), int(bool(advance)),
+        int(window), int(Hq), int(Hkv), int(D), _dtype(q), _dtype(out), int(n_ctx), _ref(rope), _ptr(out), _ptr(lse),
+        _stream(stream)))
     return (out, lse) if return_lse else out
 

@@ -144,3 +144,43 @@ def test_decode_rejects_bad_steps():
     with pytest.raises(ris.RisError):
         ris.ris_decode_step(an, q[0].contiguous(), k_hi, k_lo, v, 160, 0, 150)  # empty window
     an.free()
+
+
+def test_decode_device_position_and_graph_replay():
+    """The position read from device memory, advanced by each step: one captured CUDA graph of
+    the step replayed token after token gives the oracle's outputs for t0, t0 + 1, ..."""
+    N, T, Hq, Hkv, D = 600, 700, 12, 2, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(T, Hq, Hkv, D, seed=21, outliers=True)
+    rope = ris.rope_cfg(ris.ROPE_YARN, 1e6, 256)
+    k_hi, k_lo = ris.ris_rope_split(k, N, rope)
+    an = ris.ris_decode_anchor(N, Hkv, 1, 0.03, [5, 6])
+    A = ora.decode_anchor(anchor_spec(N, 1, 0.03, [5, 6]))
+    W = 48
+    qbuf = torch.empty(Hq, D, dtype=q.dtype, device="cuda")
+    out = torch.empty(Hq, D, dtype=torch.float32, device="cuda")
+    t_dev = torch.tensor([N], dtype=torch.int64, device="cuda")
+    qbuf.copy_(q[N])
+    ris.ris_decode_step(an, qbuf, k_hi, k_lo, v, 0, W, N, rope, out=out, t_dev=t_dev, advance=True)  # allocates
+    torch.cuda.synchronize()
+    assert int(t_dev.item()) == N + 1
+    ref, _, _ = ora.decode_step(qn[N], kn, vn, N, A, W, oracle_rope(3, 1e6, 256), N)
+    check_bf16_path(to_np(out), ref)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        ris.ris_decode_step(an, qbuf, k_hi, k_lo, v, 0, W, N, rope, out=out, t_dev=t_dev, advance=True)
+    for t in (N + 1, N + 2, N + 60):
+        t_dev.fill_(t)
+        qbuf.copy_(q[t])
+        g.replay()
+        torch.cuda.synchronize()
+        assert int(t_dev.item()) == t + 1
+        ref, _, _ = ora.decode_step(qn[t], kn, vn, t, A, W, oracle_rope(3, 1e6, 256), N)
+        check_bf16_path(to_np(out), ref)
+    ris.ris_device_status()
+    # a device-side position past the cache is flagged and attends to nothing
+    t_dev.fill_(T)
+    g.replay()
+    with pytest.raises(ris.RisError):
+        ris.ris_device_status()
+    ris.ris_device_status()  # the report cleared the flag
+    an.free()
