@@ -72,6 +72,11 @@ WORKLOADS = {
     "C6": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
                runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)], geometry="paper",
                title="C5 with the paper's geometry (local window 1024 + 4 anchor tokens)"),
+    # Hybrid Anchor decode after the C5 prefill: 32 generated tokens x 28 layers per run, the
+    # anchor of each run frozen at the first token, a 1024-token sliding window
+    "D5": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+               runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)], kind="decode", gen=32, window=1024,
+               title="Hybrid Anchor decode after the N=65536 prefill, 28 layers, YaRN s=2"),
     # the sub-1% Structural sweep at 64k: d = 0.1% .. 0.9%, 50 .. 200 seeds, one layer each
     "S1": dict(N=65536, layers=1, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
                runs=[(f"structural_{d / 10:.1f}pct_x{s}", 1, d / 1000, s) for d in range(1, 10)
@@ -134,7 +139,10 @@ def workload_config(a):
         "geometry": ("local window 1024 + 4 anchors" if w.get("geometry") == "paper" else "diagonal only"),
         "l2": (f"inputs larger than L2: each layer has its own q/k/v ({per_layer / 2**20:.0f} MiB), "
                f"{w['layers']} layers = {w['layers'] * per_layer / 2**20:.0f} MiB per run"),
-    }
+    } | ({"decode": {"generated_tokens": w["gen"], "window": w["window"],
+                     "cache": "rotated K (bf16 hi + lo) and V of every layer, N + generated tokens rows",
+                     "l2": "every token reads 28 layers' selected K/V rows (~300 MB), more than L2"}}
+         if w.get("kind") == "decode" else {})
 
 
 # ----------------------------------------------------------------------------- distributed plumbing
@@ -353,6 +361,234 @@ def recorded_traffic(kernel_file: str):
     return None
 
 
+# ----------------------------------------------------------------------------- decode workload
+def oracle_decode_sample(w, target_s, rng_seed):
+    """Time the fp64 oracle's decode step on random (run, generated token) samples of layer 0;
+    returns (pair-heads, seconds, steps)."""
+    import numpy as np
+
+    import oracle
+    from paper_2607_21927_gb300 import inputs
+
+    import torch
+
+    N, gen = w["N"], w["gen"]
+    T = N + gen
+    q, k, v = inputs.make_qkv(T, w["Hq"], w["Hkv"], w["D"], dtype=torch.bfloat16, seed=0, outliers=w["outliers"])
+    qn, kn, vn = (x.float().numpy().astype("float64") for x in (q, k, v))
+    cfg = oracle_rope(w)
+    anchors = [oracle.decode_anchor(oracle.MaskSpec(N=N, mode=m, density=d, seeds=list(range(s))))
+               for _, m, d, s in w["runs"]]
+    rng = np.random.default_rng(rng_seed)
+    ph, secs, steps = 0, 0.0, 0
+    while secs < target_s:
+        ri = int(rng.integers(len(anchors)))
+        t = N + int(rng.integers(gen))
+        t0 = time.perf_counter()
+        out, lse, keys = oracle.decode_step(qn[t], kn, vn, t, anchors[ri], w["window"], cfg, N)
+        secs += time.perf_counter() - t0
+        ph += keys.shape[0] * w["Hq"]
+        steps += 1
+    return ph, secs, steps
+
+
+def run_reference_decode(a, rank):
+    if rank != 0:
+        return
+    import oracle
+
+    w = a.w
+    oracle.set_threads(os.cpu_count() or 1)
+    oracle_decode_sample(w, 0.5, 99)
+    ph, secs, steps = oracle_decode_sample(w, max(2.0, a.cpu_seconds / 2) * a.steps, 7)
+    value = ph / secs
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": a.gpus,
+            "steps": a.steps, "warmup": a.warmup, "ms_per_step": 1e3 * secs / a.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(a),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.get_threads(), "kind": "oracle",
+                             "sample": f"{steps} decode steps of layer 0 (random run and token), {ph} pair-heads "
+                                       f"in {secs:.1f} s"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main_decode(a, rank, world, dist):
+    """Decode workload: per run, the anchor is frozen once (timed apart), then each step generates
+    `gen` tokens through all layers; one CUDA graph per (run, token) position-independent chain of
+    layers is captured once and replayed, the position living in device memory."""
+    import tempfile
+
+    import torch
+
+    from paper_2607_21927_gb300 import inputs, ris
+
+    w = a.w
+    dev = torch.device("cuda", torch.cuda.current_device())
+    N, L, Hq, Hkv, D, gen, W = w["N"], w["layers"], w["Hq"], w["Hkv"], w["D"], w["gen"], w["window"]
+    T = N + gen
+    kind, theta, native = w["rope"]
+    rope = ris.rope_cfg(ROPE_KINDS[kind], theta, native)
+    runs = w["runs"]
+    # per layer: the rotated cache of N + gen positions (prefill and generated tokens' keys)
+    k_hi, k_lo, vs = [], [], []
+    for layer in range(L):
+        _, k, v = inputs.make_qkv(T, Hq, Hkv, D, dtype=torch.bfloat16, seed=layer, outliers=w["outliers"], device=dev)
+        hi, lo = ris.ris_rope_split(k, N, rope)
+        k_hi.append(hi)
+        k_lo.append(lo)
+        vs.append(v)
+        del k
+    gq = torch.Generator(device=dev)
+    gq.manual_seed(1234)
+    qs = torch.randn(gen, L, Hq, D, generator=gq, device=dev).to(torch.bfloat16)
+    outs = torch.empty(len(runs), gen, L, Hq, D, dtype=torch.float32, device=dev)
+    qbuf = torch.empty(L, Hq, D, dtype=torch.bfloat16, device=dev)
+    obuf = torch.empty(L, Hq, D, dtype=torch.float32, device=dev)
+    t_dev = torch.zeros(1, dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream()
+
+    ev_a0, ev_a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev_a0.record(stream)
+    anchors = [ris.ris_decode_anchor(N, Hkv, m, d, list(range(s))) for _, m, d, s in runs]
+    ev_a1.record(stream)
+    torch.cuda.synchronize()
+    anchor_ms = ev_a0.elapsed_time(ev_a1) / len(runs)
+    n_anchor = [an.info()[2] for an in anchors]
+
+    def token_chain(an):
+        for layer in range(L):
+            ris.ris_decode_step(an, qbuf[layer], k_hi[layer], k_lo[layer], vs[layer], N, W, N, rope,
+                                out=obuf[layer], t_dev=t_dev, advance=(layer == L - 1))
+
+    graphs = []
+    for an in anchors:
+        t_dev.fill_(N)
+        token_chain(an)  # sizes the anchor's partials buffer before capture
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            token_chain(an)
+        graphs.append(g)
+    t_start = torch.tensor([N], dtype=torch.int64).pin_memory()
+
+    def step():
+        for ri, g in enumerate(graphs):
+            t_dev.copy_(t_start, non_blocking=True)
+            for tok in range(gen):
+                qbuf.copy_(qs[tok])
+                g.replay()
+                outs[ri, tok].copy_(obuf)
+
+    for _ in range(a.warmup):
+        step()
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    ceil = ceilings(ris, w, a.no_probes)
+
+    clocks_path = os.path.join(tempfile.gettempdir(), f"ris_bench_clocks_{os.getpid()}.csv")
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(dist)
+    torch.cuda.synchronize()
+    with ClockSampler(clocks_path) as clk:
+        ev0.record(stream)
+        for _ in range(a.steps):
+            step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    # graph replays bypass the library's host launch counter: two kernels per layer and token
+    launches = 2 * L * gen * len(runs) * a.steps
+    barrier(dist)
+    elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1), dist)
+    ris.ris_device_status()
+
+    # keys per token: the anchor keys below the window plus the window (t - W < j <= t)
+    pairs = 0
+    for an, na in zip(anchors, n_anchor):
+        keys = an.info()[3].cpu()
+        for tok in range(gen):
+            t = N + tok
+            lo = max(0, t - W + 1)
+            pairs += int((keys < lo).sum()) + (t - lo + 1)
+    pair_heads_step = pairs * L * Hq
+    value = world * pair_heads_step * a.steps / (elapsed_ms / 1e3)
+    ms_step = elapsed_ms / a.steps
+    tokens_step = gen * len(runs)
+    bytes_step = pairs * L * Hkv * 2 * D * 2  # K and V rows (bf16) of every selected key, all KV heads
+    achieved = bytes_step / (ms_step / 1e3) / 1e9
+    hbm = ceil["hbm_gbs"]
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                "traffic": None, "kernel": "k_decode_partial + k_decode_combine (whole token chain)",
+                "peak_source": ceil["hbm_source"],
+                "bytes": "algorithmic: K and V rows (bf16) of every selected key, all KV heads, over the step time "
+                         "(graph replays: no per-launch timer)"}
+    clocks = clk.summary(getattr(torch.cuda.get_device_properties(dev), "pci_bus_id", None))
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps, "warmup": a.warmup,
+            "ms_per_step": ms_step, "us_per_token": 1e3 * ms_step / tokens_step,
+            "us_per_token_layer": 1e3 * ms_step / (tokens_step * L), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload_config(a),
+            "anchor_ms": anchor_ms, "anchor_keys": dict(zip([r[0] for r in runs], n_anchor)),
+            "roofline": roofline, "ceilings": ceil, "clocks": clocks, "gpu_launches": launches}
+
+    # host-driven loop (no graph) for comparison: one Python + C call per layer and token
+    def host_step():
+        for ri, an in enumerate(anchors):
+            for tok in range(gen):
+                for layer in range(L):
+                    ris.ris_decode_step(an, qs[tok, layer], k_hi[layer], k_lo[layer], vs[layer], N + tok, W, N,
+                                        rope, out=outs[ri, tok, layer])
+
+    host_step()
+    torch.cuda.synchronize()
+    h0, h1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    h0.record(stream)
+    host_step()
+    h1.record(stream)
+    torch.cuda.synchronize()
+    line["host_loop_us_per_token"] = 1e3 * h0.elapsed_time(h1) / tokens_step
+
+    if not a.no_e2e:
+        hq = qs.cpu().pin_memory()
+        ho = torch.empty(outs.shape, dtype=outs.dtype).pin_memory()
+
+        def e2e_step():
+            for ri, g in enumerate(graphs):
+                t_dev.copy_(t_start, non_blocking=True)
+                for tok in range(gen):
+                    qbuf.copy_(hq[tok], non_blocking=True)
+                    g.replay()
+                    ho[ri, tok].copy_(obuf, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(a.steps):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = max_over_ranks(e0.elapsed_time(e1), dist)
+        line["e2e"] = {"value": world * pair_heads_step * a.steps / (e_ms / 1e3), "unit": UNIT,
+                       "h2d_bytes_per_step": len(runs) * hq.numel() * hq.element_size(),
+                       "d2h_bytes_per_step": ho.numel() * ho.element_size(), "ms_per_step": e_ms / a.steps}
+    else:
+        line["e2e"] = None
+    if rank == 0 and world == 1 and not a.no_cpu_baseline:
+        import oracle
+
+        oracle.set_threads(os.cpu_count() or 1)
+        ph, secs, steps = oracle_decode_sample(w, a.cpu_seconds, 5)
+        line["cpu_baseline"] = {"value": ph / secs, "unit": UNIT, "cores": oracle.get_threads(), "kind": "oracle",
+                                "sample": f"{steps} decode steps of layer 0 (random run and token), {ph} pair-heads "
+                                          f"in {secs:.1f} s"}
+    for an in anchors:
+        an.free()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
 # ----------------------------------------------------------------------------- our arm
 def ceilings(ris, w, no_probes):
     """Peaks: MEASURED_PEAKS.json (HBM copy, bf16 GEMM) plus this library's L2 and FFMA probes."""
@@ -381,7 +617,13 @@ def main():
     a = parse_args()
     rank, world, dist = dist_init()
     if a.impl == "reference":
-        run_reference(a, rank)
+        if a.w.get("kind") == "decode":
+            run_reference_decode(a, rank)
+        else:
+            run_reference(a, rank)
+        return
+    if a.w.get("kind") == "decode":
+        main_decode(a, rank, world, dist)
         return
 
     import torch

@@ -10,16 +10,20 @@
 // Nothing in the launch depends on t, so the position may live in device memory and a
 // captured CUDA graph of a whole token can be replayed token after token.
 //
-//   k_decode_partial : one CTA per (chunk of 32 keys, KV head): rotates the G query heads of
-//                      the KV head at position t (fp64 angle, as the prefill RoPE), stages the
-//                      chunk's K~ (high + low parts, fp32) and V rows in shared memory, and
-//                      writes each head's partial (max, sum) and unnormalised output.
-//   k_decode_combine : one CTA per query head: rescales the partials to the global maximum,
-//                      sums and normalises; optional natural-log LSE.
+//   k_decode_partial : one CTA per (chunk of 32 keys, KV head): issues all of the chunk's
+//                      16-byte K~ (high + low parts) and V row loads at once, rotates the G
+//                      query heads of the KV head at position t (fp64 angle, as the prefill
+//                      RoPE) while they are in flight, and computes each head's partial
+//                      (max, sum, unnormalised output) in shared memory; clusters of 8 CTAs
+//                      merge their partials through distributed shared memory, and the first
+//                      CTA of each cluster writes one partial.
+//   k_decode_combine : one CTA per query head: rescales the cluster partials to the global
+//                      maximum, sums and normalises; optional natural-log LSE.
 //
 // A decode step is one query row: a GEMV-shaped product that reads each selected K/V row once,
 // so it runs on the FP32 pipes (no tensor-core tile to fill) and is bound by the K/V row
 // reads; fp32 scores and probabilities keep it well inside the bf16 tolerance.
+#include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
 #include <cmath>
@@ -27,14 +31,15 @@
 
 #include "ris_internal.h"
 
+namespace cg = cooperative_groups;
+
 namespace ris {
 namespace {
 
 __device__ unsigned int g_ris_decode_error;
 
-constexpr int kDecodeThreads = 128;
+constexpr int kDecodeThreads = 256;  // eight warps: one per query head of the KV head
 constexpr int kMaxG = 8;
-constexpr int kMaxD = 128;
 
 template <typename T>
 __device__ __forceinline__ float ldf(const T *p);
@@ -52,113 +57,273 @@ __device__ __forceinline__ void sincos_reduced(double a, float *sn, float *cs)
     sincosf((float)red, sn, cs);
 }
 
-template <typename T, bool LO>
-__global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeArgs a)
-{
-    __shared__ float qs[kMaxG][kMaxD];
-    __shared__ float ks[kDecodeChunk][kMaxD + 1];  // +1: rows fall in distinct banks
-    __shared__ float vs[kDecodeChunk][kMaxD];
-    __shared__ float ps[kMaxG][kDecodeChunk];
-    __shared__ int32_t keys[kDecodeChunk];
+// 16-byte row pieces of the staged K/V rows: bf16 holds 8 values per piece, fp32 holds 4.
+template <typename T>
+struct Piece {
+    static constexpr int kVals = 16 / sizeof(T);
+};
 
-    const int g = blockIdx.y, chunk = blockIdx.x, tid = threadIdx.x;
-    const int D = a.D, G = a.G, half = D >> 1;
-    const int64_t slot = (int64_t)g * a.n_chunks + chunk;
-    const int64_t t = a.t_dev != nullptr ? *a.t_dev : a.t;
-    if (t < a.t0 || t >= a.cache_len) {  // only reachable through t_dev: flag it, attend to nothing
-        if (tid == 0 && chunk == 0 && g == 0) atomicOr(&g_ris_decode_error, 2u);
-        for (int h = tid; h < G; h += kDecodeThreads) a.part_ml[slot * G + h] = make_float2(-INFINITY, 0.f);
-        return;
-    }
-    const int64_t win_lo = t - a.window + 1 > 0 ? t - a.window + 1 : 0;
-    const int m = a.heads_keyed > 1 ? g : 0;
-    const int64_t nA = a.rank[(int64_t)m * (a.t0 + 1) + (win_lo < a.t0 ? win_lo : a.t0)];
-    const int64_t n = nA + (t - win_lo + 1);
-    const int64_t k0 = (int64_t)chunk * kDecodeChunk;
-    if (k0 >= n) {  // fewer keys than the grid covers: an empty partial
-        for (int h = tid; h < G; h += kDecodeThreads) a.part_ml[slot * G + h] = make_float2(-INFINITY, 0.f);
-        return;
-    }
-    const int nk = (int)((n - k0) < kDecodeChunk ? (n - k0) : kDecodeChunk);
-    const int32_t *anchor = a.anchor + a.anchor_off[m];
-    if (tid < kDecodeChunk) {
-        const int64_t kk = k0 + tid;
-        int64_t key = 0;  // rows past the set read key 0 and are masked out below
-        if (kk < n) key = kk < nA ? (int64_t)anchor[kk] : win_lo + (kk - nA);
-        keys[tid] = (int32_t)key;
-    }
-    for (int idx = tid; idx < G * half; idx += kDecodeThreads) {
-        const int h = idx / half, c = idx - h * half;
-        float sn, cs;
-        sincos_reduced((double)t * a.f[c], &sn, &cs);
-        const T *qp = reinterpret_cast<const T *>(a.q) + (int64_t)(g * G + h) * D;
-        const float x0 = ldf(qp + c), x1 = ldf(qp + c + half);
-        qs[h][c] = fmaf(x0, cs, -x1 * sn) * a.mscale;
-        qs[h][c + half] = fmaf(x1, cs, x0 * sn) * a.mscale;
-    }
-    __syncthreads();
-    for (int idx = tid; idx < kDecodeChunk * D; idx += kDecodeThreads) {
-        const int r = idx / D, c = idx - r * D;
-        const int64_t off = ((int64_t)keys[r] * a.Hkv + g) * D + c;
-        float kv = ldf(reinterpret_cast<const T *>(a.k) + off);
-        if (LO) kv += ldf(reinterpret_cast<const __nv_bfloat16 *>(a.k_lo) + off);
-        ks[r][c] = kv;
-        vs[r][c] = ldf(reinterpret_cast<const T *>(a.v) + off);
-    }
-    __syncthreads();
-    for (int idx = tid; idx < G * kDecodeChunk; idx += kDecodeThreads) {
-        const int h = idx / kDecodeChunk, r = idx - h * kDecodeChunk;
-        float s = 0.f;
-        for (int c = 0; c < D; ++c) s = fmaf(qs[h][c], ks[r][c], s);
-        ps[h][r] = r < nk ? s * a.scale_log2 : -INFINITY;
-    }
-    __syncthreads();
-    const int warp = tid >> 5, lane = tid & 31;
-    for (int h = warp; h < G; h += kDecodeThreads / 32) {  // kDecodeChunk == 32: one key per lane
-        const float x = ps[h][lane];
-        float mx = x;
+__device__ __forceinline__ void unpack(const uint4 &u, float *o, const __nv_bfloat16 *)
+{
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
-        const float p = exp2f(x - mx);  // the chunk holds at least one key, so mx is finite
-        float l = p;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, o);
-        ps[h][lane] = p;
-        if (lane == 0) a.part_ml[slot * G + h] = make_float2(mx, l);
-    }
-    __syncthreads();
-    for (int idx = tid; idx < G * D; idx += kDecodeThreads) {
-        const int h = idx / D, c = idx - h * D;
-        float acc = 0.f;
-        for (int r = 0; r < nk; ++r) acc = fmaf(ps[h][r], vs[r][c], acc);
-        a.part_o[(slot * G + h) * D + c] = acc;
+    for (int i = 0; i < 4; ++i) {
+        o[2 * i] = __uint_as_float(w[i] << 16);
+        o[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
     }
 }
 
-template <typename TO>
-__global__ void k_decode_combine(const DecodeArgs a)
+__device__ __forceinline__ void unpack(const uint4 &u, float *o, const float *)
 {
-    const int h = blockIdx.x, c = threadIdx.x;
-    const int g = h / a.G, hl = h - g * a.G;
-    const int64_t base = (int64_t)g * a.n_chunks;
-    float M = -INFINITY;
-    for (int ch = 0; ch < a.n_chunks; ++ch) M = fmaxf(M, a.part_ml[(base + ch) * a.G + hl].x);
-    float L = 0.f, acc = 0.f;
-    for (int ch = 0; ch < a.n_chunks; ++ch) {
-        const float2 ml = a.part_ml[(base + ch) * a.G + hl];
-        if (ml.x == -INFINITY) continue;  // empty chunk: no output was written
-        const float w = exp2f(ml.x - M);
-        L = fmaf(ml.y, w, L);
-        acc = fmaf(a.part_o[((base + ch) * a.G + hl) * a.D + c], w, acc);
+    o[0] = __uint_as_float(u.x);
+    o[1] = __uint_as_float(u.y);
+    o[2] = __uint_as_float(u.z);
+    o[3] = __uint_as_float(u.w);
+}
+
+// One CTA per (chunk of kDecodeChunk keys, KV head); kDecodeCluster consecutive chunks form a
+// thread-block cluster whose first CTA merges the cluster's partials through distributed
+// shared memory, so only one partial per cluster goes to global memory. The dependent global
+// loads on the way to the K/V rows are the position, then (in parallel) its rank-table entry
+// and this chunk's slice of the anchor list, then the rows themselves.
+template <typename T, bool LO, int D>
+__global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecodeThreads)
+    k_decode_partial(const DecodeArgs a)
+{
+    constexpr int kPiecesRow = D * (int)sizeof(T) / 16;                   // 16-byte pieces per row
+    constexpr int kPieces = kDecodeChunk * kPiecesRow / kDecodeThreads;  // per thread and plane
+    constexpr int kHalf = D / 2;
+    constexpr int kQuarter = D / 4;
+    static_assert(kDecodeChunk * kPiecesRow % kDecodeThreads == 0, "pieces per thread");
+    static_assert(D <= kDecodeThreads, "one thread per channel in the value product");
+    __shared__ __align__(16) float qs[kMaxG][D];
+    __shared__ __align__(16) float ks[kDecodeChunk][D + 4];  // +4: 16-byte rows in distinct bank groups
+    __shared__ float vs[kDecodeChunk][D];
+    __shared__ __align__(16) float ps[kMaxG][kDecodeChunk];
+    __shared__ __align__(16) float os[kMaxG][D];  // this CTA's unnormalised outputs
+    __shared__ float2 ml[kMaxG];                  // this CTA's (max, sum), log2 domain
+    __shared__ float wt[kMaxG][kDecodeCluster];   // merge weights (first CTA of the cluster)
+    __shared__ float2 rot[kHalf];                 // (cos, sin) of t * f_c
+    __shared__ int32_t keys[kDecodeChunk];
+
+    cg::cluster_group cluster = cg::this_cluster();
+    const int g = blockIdx.y, chunk = blockIdx.x, tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int G = a.G;
+    const int m = a.heads_keyed > 1 ? g : 0;
+    const int64_t k0 = (int64_t)chunk * kDecodeChunk;
+    // this thread's anchor slot, loaded alongside the position (the cut decides if it is used)
+    int32_t spec = 0;
+    if (tid < kDecodeChunk && k0 + tid < a.anchor_len[m]) spec = __ldg(a.anchor + a.anchor_base[m] + k0 + tid);
+    const int64_t t = a.t_dev != nullptr ? *a.t_dev : a.t;
+    const bool valid = t >= a.t0 && t < a.cache_len;  // only a device-side t can be outside
+    if (!valid && tid == 0 && chunk == 0 && g == 0) atomicOr(&g_ris_decode_error, 2u);
+    const int64_t win_lo = t - a.window + 1 > 0 ? t - a.window + 1 : 0;
+    const int64_t nA = valid ? __ldg(a.rank + (int64_t)m * (a.t0 + 1) + (win_lo < a.t0 ? win_lo : a.t0)) : 0;
+    const int64_t n = valid ? nA + (t - win_lo + 1) : 0;
+    const bool active = k0 < n;  // block-uniform; inactive CTAs still take part in the cluster syncs
+    const int nk = active ? (int)((n - k0) < kDecodeChunk ? (n - k0) : kDecodeChunk) : 0;
+
+    if (active) {
+        if (tid < kDecodeChunk) {
+            const int64_t kk = k0 + tid;
+            int64_t key = 0;  // rows past the set read key 0 and are masked out below
+            if (kk < n) key = kk < nA ? (int64_t)spec : win_lo + (kk - nA);
+            keys[tid] = (int32_t)key;
+        }
+        __syncthreads();
+        // every row load of the chunk is issued before any is used
+        uint4 kh[kPieces], kl[kPieces], vv[kPieces];
+#pragma unroll
+        for (int j = 0; j < kPieces; ++j) {
+            const int u = tid + j * kDecodeThreads, r = u / kPiecesRow, pc = u - r * kPiecesRow;
+            const int64_t row = ((int64_t)keys[r] * a.Hkv + g) * D;
+            kh[j] = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const T *>(a.k) + row) + pc);
+            if (LO) kl[j] = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(a.k_lo) + row) + pc);
+            vv[j] = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const T *>(a.v) + row) + pc);
+        }
+        // rotate the G query heads at position t while the rows are in flight
+        if (tid < kHalf) {
+            float sn, cs;
+            sincos_reduced((double)t * a.f[tid], &sn, &cs);
+            rot[tid] = make_float2(cs, sn);
+        }
+        __syncthreads();
+        for (int idx = tid; idx < G * kHalf; idx += kDecodeThreads) {
+            const int h = idx / kHalf, c = idx - h * kHalf;
+            const float2 cs = rot[c];
+            const T *qp = reinterpret_cast<const T *>(a.q) + (int64_t)(g * G + h) * D;
+            const float x0 = ldf(qp + c), x1 = ldf(qp + c + kHalf);
+            qs[h][c] = fmaf(x0, cs.x, -x1 * cs.y) * a.mscale;
+            qs[h][c + kHalf] = fmaf(x1, cs.x, x0 * cs.y) * a.mscale;
+        }
+#pragma unroll
+        for (int j = 0; j < kPieces; ++j) {
+            const int u = tid + j * kDecodeThreads, r = u / kPiecesRow, pc = u - r * kPiecesRow;
+            constexpr int nv = Piece<T>::kVals;
+            float x[nv], y[nv];
+            unpack(kh[j], x, (const T *)nullptr);
+            if (LO) {
+                float lo8[8];
+                unpack(kl[j], lo8, (const __nv_bfloat16 *)nullptr);
+#pragma unroll
+                for (int e = 0; e < nv; ++e) x[e] += lo8[e];
+            }
+            unpack(vv[j], y, (const T *)nullptr);
+#pragma unroll
+            for (int e = 0; e < nv; e += 4) {
+                *reinterpret_cast<float4 *>(&ks[r][pc * nv + e]) = make_float4(x[e], x[e + 1], x[e + 2], x[e + 3]);
+                *reinterpret_cast<float4 *>(&vs[r][pc * nv + e]) = make_float4(y[e], y[e + 1], y[e + 2], y[e + 3]);
+            }
+        }
+        __syncthreads();
+        // scores and the chunk's softmax: warp h takes query head h, lane r takes key r
+        if (warp < G) {
+            const int h = warp, r = lane;
+            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll 8
+            for (int c = 0; c < D; c += 4) {
+                const float4 q4 = *reinterpret_cast<const float4 *>(&qs[h][c]);
+                const float4 k4 = *reinterpret_cast<const float4 *>(&ks[r][c]);
+                s0 = fmaf(q4.x, k4.x, s0);
+                s1 = fmaf(q4.y, k4.y, s1);
+                s2 = fmaf(q4.z, k4.z, s2);
+                s3 = fmaf(q4.w, k4.w, s3);
+            }
+            const float x = r < nk ? ((s0 + s1) + (s2 + s3)) * a.scale_log2 : -INFINITY;
+            float mx = x;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+            const float p = exp2f(x - mx);  // an active chunk holds at least one key: mx is finite
+            float l = p;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, o);
+            ps[h][r] = p;
+            if (lane == 0) ml[h] = make_float2(mx, l);
+        }
+        __syncthreads();
+        // value product: thread (channel c, head set hs) over heads hs, hs + step, ...
+        {
+            constexpr int kStep = kDecodeThreads / D;
+            constexpr int kPer = (kMaxG + kStep - 1) / kStep;
+            const int c = tid % D, hs = tid / D;
+            float acc[kPer];
+#pragma unroll
+            for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
+            for (int r = 0; r < nk; r += 4) {  // ps beyond nk is 0 and vs rows there are finite
+                const float v0 = vs[r][c], v1 = vs[r + 1][c], v2 = vs[r + 2][c], v3 = vs[r + 3][c];
+#pragma unroll
+                for (int e = 0; e < kPer; ++e) {
+                    const int h = hs + e * kStep;
+                    if (h < G) {
+                        const float4 p4 = *reinterpret_cast<const float4 *>(&ps[h][r]);
+                        acc[e] = fmaf(p4.x, v0, fmaf(p4.y, v1, fmaf(p4.z, v2, fmaf(p4.w, v3, acc[e]))));
+                    }
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < kPer; ++e) {
+                const int h = hs + e * kStep;
+                if (h < G) os[h][c] = acc[e];
+            }
+        }
+    } else if (tid < kMaxG) {
+        ml[tid] = make_float2(-INFINITY, 0.f);
     }
-    const float o = acc / L;
-    if constexpr (sizeof(TO) == 4)
-        reinterpret_cast<float *>(a.out)[(int64_t)h * a.D + c] = o;
-    else
-        reinterpret_cast<__nv_bfloat16 *>(a.out)[(int64_t)h * a.D + c] = __float2bfloat16_rn(o);
-    if (c == 0 && a.lse != nullptr) a.lse[h] = (M + log2f(L)) * 0.69314718055994530942f;
-    // the partial kernel, the only reader of t, has finished: move to the next position
-    if (a.advance && a.t_dev != nullptr && h == 0 && c == 0) *a.t_dev += 1;
+    cluster.sync();
+    if (cluster.block_rank() == 0) {
+        // merge the cluster's partials (distributed shared memory) into one
+        const int grp = chunk / kDecodeCluster;
+        const int64_t slot = (int64_t)g * a.n_groups + grp;
+        if (tid < G) {
+            float2 mr[kDecodeCluster];
+            float M = -INFINITY;
+#pragma unroll
+            for (int r = 0; r < kDecodeCluster; ++r) {
+                mr[r] = cluster.map_shared_rank(&ml[0], r)[tid];
+                M = fmaxf(M, mr[r].x);
+            }
+            float L = 0.f;
+#pragma unroll
+            for (int r = 0; r < kDecodeCluster; ++r) {
+                const float w = mr[r].x == -INFINITY ? 0.f : exp2f(mr[r].x - M);
+                wt[tid][r] = w;
+                L = fmaf(mr[r].y, w, L);
+            }
+            a.part_ml[slot * G + tid] = make_float2(M, L);
+        }
+        __syncthreads();
+        for (int idx = tid; idx < G * kQuarter; idx += kDecodeThreads) {
+            const int h = idx / kQuarter, c4 = (idx - h * kQuarter) * 4;
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int r = 0; r < kDecodeCluster; ++r) {
+                const float w = wt[h][r];
+                if (w == 0.f) continue;  // empty chunk: its outputs were never written
+                const float4 o = *reinterpret_cast<const float4 *>(cluster.map_shared_rank(&os[0][0], r) + h * D + c4);
+                acc.x = fmaf(o.x, w, acc.x);
+                acc.y = fmaf(o.y, w, acc.y);
+                acc.z = fmaf(o.z, w, acc.z);
+                acc.w = fmaf(o.w, w, acc.w);
+            }
+            *reinterpret_cast<float4 *>(a.part_o + (slot * G + h) * D + c4) = acc;
+        }
+    }
+    cluster.sync();  // the other CTAs' shared memory stays alive until the merge has read it
+}
+
+// One CTA per (query head, 32-channel slice); each of its 8 warps folds a strided subset of
+// the cluster partials with an online maximum, then the warps are merged in shared memory.
+constexpr int kCombineWarps = 8;
+
+template <typename TO>
+__global__ void __launch_bounds__(kCombineWarps * 32) k_decode_combine(const DecodeArgs a)
+{
+    __shared__ float wm[kCombineWarps], wl[kCombineWarps], wacc[kCombineWarps][32];
+    const int h = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int c = blockIdx.y * 32 + lane;
+    const int g = h / a.G, hl = h - g * a.G;
+    const float2 *ml = a.part_ml + (int64_t)g * a.n_groups * a.G + hl;
+    const float *po = a.part_o + ((int64_t)g * a.n_groups * a.G + hl) * a.D + c;
+    float M = -INFINITY, L = 0.f, acc = 0.f;
+#pragma unroll 4
+    for (int i = warp; i < a.n_groups; i += kCombineWarps) {
+        const float2 mi = ml[(int64_t)i * a.G];
+        const float oi = po[(int64_t)i * a.G * a.D];
+        if (mi.x == -INFINITY) continue;
+        const float nm = fmaxf(M, mi.x);
+        const float so = exp2f(M - nm), si = exp2f(mi.x - nm);  // M = -inf gives so = 0
+        L = fmaf(L, so, mi.y * si);
+        acc = fmaf(acc, so, oi * si);
+        M = nm;
+    }
+    if (lane == 0) {
+        wm[warp] = M;
+        wl[warp] = L;
+    }
+    wacc[warp][lane] = acc;
+    __syncthreads();
+    if (warp == 0) {
+        float Mt = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < kCombineWarps; ++w) Mt = fmaxf(Mt, wm[w]);
+        float Lt = 0.f, o = 0.f;
+#pragma unroll
+        for (int w = 0; w < kCombineWarps; ++w) {
+            if (wm[w] == -INFINITY) continue;
+            const float s = exp2f(wm[w] - Mt);
+            Lt = fmaf(wl[w], s, Lt);
+            o = fmaf(wacc[w][lane], s, o);
+        }
+        o /= Lt;
+        if constexpr (sizeof(TO) == 4)
+            reinterpret_cast<float *>(a.out)[(int64_t)h * a.D + c] = o;
+        else
+            reinterpret_cast<__nv_bfloat16 *>(a.out)[(int64_t)h * a.D + c] = __float2bfloat16_rn(o);
+        if (lane == 0 && blockIdx.y == 0 && a.lse != nullptr) a.lse[h] = (Mt + log2f(Lt)) * 0.69314718055994530942f;
+        // the partial kernel, the only reader of t, has finished: move to the next position
+        if (a.advance && a.t_dev != nullptr && h == 0 && blockIdx.y == 0 && lane == 0) *a.t_dev += 1;
+    }
 }
 
 // rank[m][j] = lower_bound(keys of list m, j) - start, for j = 0 .. t0
@@ -199,19 +364,30 @@ unsigned int read_decode_error()
     return v;
 }
 
+template <int D>
+void launch_partial(const DecodeArgs &a, int dtype, dim3 grid, cudaStream_t s)
+{
+    if (dtype == RIS_F32)
+        k_decode_partial<float, false, D><<<grid, kDecodeThreads, 0, s>>>(a);
+    else if (a.k_lo != nullptr)
+        k_decode_partial<__nv_bfloat16, true, D><<<grid, kDecodeThreads, 0, s>>>(a);
+    else
+        k_decode_partial<__nv_bfloat16, false, D><<<grid, kDecodeThreads, 0, s>>>(a);
+}
+
 cudaError_t launch_decode(const DecodeArgs &a, int dtype, int out_dtype, cudaStream_t s)
 {
+    // n_chunks is a multiple of the cluster size (the host rounds it up)
     const dim3 grid_p((unsigned)a.n_chunks, (unsigned)a.Hkv);
-    if (dtype == RIS_F32)
-        k_decode_partial<float, false><<<grid_p, kDecodeThreads, 0, s>>>(a);
-    else if (a.k_lo != nullptr)
-        k_decode_partial<__nv_bfloat16, true><<<grid_p, kDecodeThreads, 0, s>>>(a);
+    if (a.D == 128)
+        launch_partial<128>(a, dtype, grid_p, s);
     else
-        k_decode_partial<__nv_bfloat16, false><<<grid_p, kDecodeThreads, 0, s>>>(a);
+        launch_partial<64>(a, dtype, grid_p, s);
+    const dim3 grid_c((unsigned)a.Hq, (unsigned)(a.D / 32));
     if (out_dtype == RIS_F32)
-        k_decode_combine<float><<<a.Hq, a.D, 0, s>>>(a);
+        k_decode_combine<float><<<grid_c, kCombineWarps * 32, 0, s>>>(a);
     else
-        k_decode_combine<__nv_bfloat16><<<a.Hq, a.D, 0, s>>>(a);
+        k_decode_combine<__nv_bfloat16><<<grid_c, kCombineWarps * 32, 0, s>>>(a);
     note_launch(2);
     return cudaGetLastError();
 }

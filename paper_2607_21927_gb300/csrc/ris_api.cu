@@ -901,7 +901,10 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     a.k_lo = k_lo;
     a.v = v;
     a.anchor = anchor->keys;
-    a.anchor_off = anchor->off;
+    for (int32_t m = 0; m < anchor->heads_keyed; ++m) {
+        a.anchor_base[m] = anchor->h_off[m];
+        a.anchor_len[m] = (int32_t)(anchor->h_off[m + 1] - anchor->h_off[m]);
+    }
     a.rank = anchor->rank;
     a.t0 = anchor->t0;
     a.cache_len = cache_len;
@@ -915,7 +918,9 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     a.t = t;
     a.t_dev = t_dev;
     // the grid covers the largest merged set (every anchor key plus a full window), whatever t is
-    a.n_chunks = (int32_t)((anchor->max_keys + window + kDecodeChunk - 1) / kDecodeChunk);
+    const int64_t chunks = (anchor->max_keys + window + kDecodeChunk - 1) / kDecodeChunk;
+    a.n_groups = (int32_t)((chunks + kDecodeCluster - 1) / kDecodeCluster);
+    a.n_chunks = a.n_groups * kDecodeCluster;
     double ms = 1.0;
     if (rope != nullptr && rope->kind != RIS_ROPE_NONE) RIS_TRY(ris_rope_freqs(rope, n_ctx, head_dim, a.f, &ms));
     a.mscale = (float)ms;
@@ -924,7 +929,7 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     a.out = out;
     a.lse = lse;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    const size_t slots = (size_t)kv_heads * a.n_chunks * a.G;
+    const size_t slots = (size_t)kv_heads * a.n_groups * a.G;
     const size_t o_bytes = (sizeof(float) * slots * head_dim + 255) & ~size_t(255);
     const size_t need = o_bytes + sizeof(float2) * slots;
     if (need > anchor->scratch_bytes) {

@@ -95,6 +95,7 @@ struct AttnArgs {
 // kDecodeChunk keys, one CTA per (chunk, g). The grid covers the largest possible set
 // (anchor size + W), so it does not depend on t, and t may be read from device memory.
 constexpr int kDecodeChunk = 32;
+constexpr int kDecodeCluster = 8;  // chunks merged on chip per partial written
 constexpr int kMaxDecodeKvHeads = 64;
 
 struct DecodeArgs {
@@ -102,8 +103,9 @@ struct DecodeArgs {
     const void *k;             // [T][Hkv][D] rotated keys: bf16 high parts, or fp32
     const void *k_lo;          // bf16 low parts (k~ = k + k_lo), or null
     const void *v;             // [T][Hkv][D]
-    const int32_t *anchor;     // anchor keys, ascending; mask m: anchor[anchor_off[m] .. anchor_off[m+1])
-    const int64_t *anchor_off;
+    const int32_t *anchor;     // anchor keys, ascending; mask m: anchor[anchor_base[m] ..] (anchor_len[m] keys)
+    int64_t anchor_base[kMaxDecodeKvHeads];
+    int32_t anchor_len[kMaxDecodeKvHeads];
     const int32_t *rank;       // [heads_keyed][t0 + 1]: anchor keys of mask m below j
     int64_t t0;                // first generated position (the prefill length)
     int64_t cache_len;
@@ -112,7 +114,8 @@ struct DecodeArgs {
     int32_t Hkv;
     int32_t G;
     int32_t D;
-    int32_t n_chunks;          // chunks per KV head (grid.x)
+    int32_t n_chunks;          // chunks per KV head (grid.x), a multiple of kDecodeCluster
+    int32_t n_groups;          // n_chunks / kDecodeCluster: partials per KV head
     int32_t window;            // W >= 1
     int32_t advance;           // with t_dev: the combine kernel adds 1 to *t_dev when done
     int64_t t;                 // position of the token (when t_dev is null)
@@ -121,8 +124,8 @@ struct DecodeArgs {
     double f[kMaxHeadDimHalf]; // rotation frequencies of q (fp64)
     float mscale;
     float scale_log2;          // log2(e) / sqrt(D)
-    float *part_o;             // [Hkv * n_chunks][G][D] partial outputs
-    float2 *part_ml;           // [Hkv * n_chunks][G] partial (max, sum) in the log2 domain
+    float *part_o;             // [Hkv * n_groups][G][D] partial outputs
+    float2 *part_ml;           // [Hkv * n_groups][G] partial (max, sum) in the log2 domain
     void *out;                 // [Hq][D]
     float *lse;                // [Hq] or null
 };
