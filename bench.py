@@ -22,9 +22,10 @@ mask_ms_per_step / attn_ms_per_layer
              is reported with the mask build amortised separately.
 roofline   = the dominant attention kernel: for the gathering designs its algorithmic bytes
              (K and V rows of every sampled pair, all KV heads) per launch over the mean
-             CUDA-event launch time against the measured HBM copy bandwidth, and against this
-             library's L2 row-gather probe; for the tcgen05 tile design its algorithmic FLOPs
-             (4 * head_dim per sampled pair-head) against the measured sustained bf16 peak.
+             CUDA-event launch time, against this library's L2 row-gather probe when the
+             layer's K/V working set fits in L2 (bound "l2", the HBM fraction beside it), else
+             the measured HBM copy bandwidth; for the tcgen05 tile design its algorithmic
+             FLOPs (4 * head_dim per sampled pair-head) against the measured sustained bf16 peak.
 
 --impl reference times the fp64 CPU oracle on the host cores on a bounded sample of the
 same workload (its own sample of rows per step) and prints the same line.
@@ -739,12 +740,16 @@ def main():
                     "peak_source": ceil["hbm_source"],
                     "bytes": "algorithmic: K and V rows of every sampled pair, all KV heads",
                     "mean_launch_ms": mean_launch_ms, "launches_timed": k_n}
-        if "l2_rows_gbs" in ceil:
-            roofline["l2_rows_peak"] = ceil["l2_rows_gbs"]
-            roofline["frac_of_l2_rows"] = achieved / ceil["l2_rows_gbs"]
-            roofline["l2_note"] = ("the K/V working set is L2-resident, so the gather is served from L2: "
-                                   "peak = this library's probe reading whole 256-byte rows at random indices "
-                                   f"over {ceil['l2_rows_set_bytes'] / 2**20:.0f} MiB")
+        kv_set = N * Hkv * D * e * (3 if e == 2 else 2)  # rotated K (hi + lo for bf16) and V of a layer
+        if "l2_rows_gbs" in ceil and kv_set < ceil["l2_bytes"]:
+            # the K/V working set is L2-resident: the gathered rows are served from L2, so L2 is
+            # the bound (HBM carries only the compulsory q/k/v/out traffic, `traffic`)
+            roofline.update({"bound": "l2", "peak": ceil["l2_rows_gbs"], "frac": achieved / ceil["l2_rows_gbs"],
+                             "peak_source": "measured in this run by the library's L2 probe: whole 256-byte rows "
+                                            f"at random indices over {ceil['l2_rows_set_bytes'] / 2**20:.0f} MiB "
+                                            "(L2 is not in MEASURED_PEAKS.json)",
+                             "hbm_peak": hbm, "frac_of_hbm": achieved / hbm,
+                             "bytes_read_per_algorithmic_byte": 1.5 if e == 2 else 1.0})
     if len(kinds) > 1:
         # several designs in one step: each design's work over its runs' layer time (RoPE included)
         per = {}
@@ -762,13 +767,17 @@ def main():
                 ach = pr * L * kv_row_bytes / (ms / 1e3) / 1e9
                 ent = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
                        "ms_per_step": ms}
-                if "l2_rows_gbs" in ceil:
-                    ent["frac_of_l2_rows"] = ach / ceil["l2_rows_gbs"]
+                kv_set = N * Hkv * D * e * (3 if e == 2 else 2)
+                if "l2_rows_gbs" in ceil and kv_set < ceil["l2_bytes"]:
+                    ent.update({"bound": "l2", "peak": ceil["l2_rows_gbs"], "frac": ach / ceil["l2_rows_gbs"],
+                                "frac_of_hbm": ach / hbm})
                 roofline["per_design"][ris.DESIGNS[kd]] = ent
         dom = max(per, key=lambda kd: per[kd][0])
         top = roofline["per_design"][ris.DESIGNS[dom]]
         roofline.update({k: top[k] for k in ("bound", "achieved", "peak", "unit", "frac")})
-        roofline.pop("frac_of_l2_rows", None)
+        for k in ("hbm_peak", "frac_of_hbm", "bytes_read_per_algorithmic_byte", "peak_source"):
+            roofline.pop(k, None)
+        roofline["peak_source"] = "per design, see per_design"
         roofline["kernel"] = "mixed designs; headline = " + ris.DESIGNS[dom] + " (most device time)"
         roofline["note"] = "per design: its runs' layer time per step (RoPE included), not the kernel alone"
     # the sampled-pair roofline: max(sampled FLOPs / tensor peak, min(row, tile) K/V bytes / bandwidth)
