@@ -129,6 +129,8 @@ __device__ __forceinline__ int velem(int j, int p)
     return (WIDE && D == 128) ? 16 * p + 2 * j : 64 * (j >> 2) + 8 * p + 2 * (j & 3);
 }
 
+constexpr float kLazyLog2 = 8.f;  // rescale O only when the row maximum grows by more than 2^8
+
 #ifndef RIS_ATTN_MIN_BLOCKS
 #define RIS_ATTN_MIN_BLOCKS 1
 #endif
@@ -285,22 +287,30 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
             mx0 = fmaxf(mx0, __shfl_xor_sync(0xFFFFFFFFu, mx0, off));
             mx1 = fmaxf(mx1, __shfl_xor_sync(0xFFFFFFFFu, mx1, off));
         }
-        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-        const float mu0 = (mn0 == -INFINITY) ? 0.f : mn0, mu1 = (mn1 == -INFINITY) ? 0.f : mn1;
-        const float al0 = exp2f(m0 - mu0), al1 = exp2f(m1 - mu1);
-        m0 = mn0;
-        m1 = mn1;
+        // Lazy rescaling: the reference maximum only moves when a score exceeds it by more
+        // than 2^kLazyLog2 (probabilities then stay below 2^kLazyLog2 and the fp32 sums stay
+        // exact enough), so most groups skip the rescale of O; the branch is warp-uniform.
+        const bool need0 = mx0 > m0 + kLazyLog2, need1 = mx1 > m1 + kLazyLog2;
+        if (__any_sync(0xFFFFFFFFu, need0 || need1)) {
+            const float mn0 = need0 ? mx0 : m0, mn1 = need1 ? mx1 : m1;
+            const float al0 = need0 ? exp2f(m0 - mn0) : 1.f, al1 = need1 ? exp2f(m1 - mn1) : 1.f;
+            m0 = mn0;
+            m1 = mn1;
+            l0 *= al0;
+            l1 *= al1;
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt) {
+                o[mt][0] *= al0;
+                o[mt][1] *= al1;
+                o[mt][2] *= al0;
+                o[mt][3] *= al1;
+            }
+        }
+        const float mu0 = (m0 == -INFINITY) ? 0.f : m0, mu1 = (m1 == -INFINITY) ? 0.f : m1;
         const float p0 = exp2f(s0 - mu0), p1 = exp2f(s1 - mu1);
         const float p2 = exp2f(s2 - mu0), p3 = exp2f(s3 - mu1);
-        l0 = l0 * al0 + (p0 + p2);
-        l1 = l1 * al1 + (p1 + p3);
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            o[mt][0] *= al0;
-            o[mt][1] *= al1;
-            o[mt][2] *= al0;
-            o[mt][3] *= al1;
-        }
+        l0 += p0 + p2;
+        l1 += p1 + p3;
         // P = P_hi + P_lo in bf16; transposed into the B operand P[head p][keys 2q.., 2q+8..]
         const float h0 = __bfloat162float(__float2bfloat16_rn(p0)), h1 = __bfloat162float(__float2bfloat16_rn(p1));
         const float h2 = __bfloat162float(__float2bfloat16_rn(p2)), h3 = __bfloat162float(__float2bfloat16_rn(p3));
