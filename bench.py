@@ -78,6 +78,16 @@ WORKLOADS = {
     "D5": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
                runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)], kind="decode", gen=32, window=1024,
                title="Hybrid Anchor decode after the N=65536 prefill, 28 layers, YaRN s=2"),
+    # per-seed ensembles (ris_ensemble_batch's mode): one output per seed, all seeds in one launch
+    "E2": dict(N=8192, layers=0, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+               runs=[("stochastic", 0, 0.01, 10)], per_seed=True,
+               title="C2 as a per-seed ensemble (10 outputs per layer)"),
+    "E4a": dict(N=32768, layers=0, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+                runs=[("stochastic", 0, 0.01, 70)], per_seed=True,
+                title="C4a as a per-seed ensemble (70 outputs per layer)"),
+    "E5": dict(N=65536, layers=0, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+               runs=[("stochastic", 0, 0.01, 10)], per_seed=True,
+               title="C5 Stochastic as a per-seed ensemble (10 outputs per layer)"),
     # the sub-1% Structural sweep at 64k: d = 0.1% .. 0.9%, 50 .. 200 seeds, one layer each
     "S1": dict(N=65536, layers=1, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
                runs=[(f"structural_{d / 10:.1f}pct_x{s}", 1, d / 1000, s) for d in range(1, 10)
@@ -138,6 +148,7 @@ def workload_config(a):
         "runs": [{"name": n, "mode": m, "density": d, "seeds": s} for n, m, d, s in w["runs"]],
         "input_dtype": w["dtype"], "outlier_channels": "1% x8" if w["outliers"] else None,
         "geometry": ("local window 1024 + 4 anchors" if w.get("geometry") == "paper" else "diagonal only"),
+        "seed_outputs": "one per seed (per-seed masks)" if w.get("per_seed") else "one (union of the seeds)",
         "l2": (f"inputs larger than L2: each layer has its own q/k/v ({per_layer / 2**20:.0f} MiB), "
                f"{w['layers']} layers = {w['layers'] * per_layer / 2**20:.0f} MiB per run"),
     } | ({"decode": {"generated_tokens": w["gen"], "window": w["window"],
@@ -273,6 +284,8 @@ def oracle_sample(q_host, k_host, v_host, w, run, target_s, rng_seed):
     nrows, total_ph, total_t, used = 8, 0, 0.0, 0
     while total_t < target_s and nrows <= N:
         rows = np.sort(rng.choice(N, size=nrows, replace=False))
+        if w.get("per_seed"):  # one seed's own mask per sample
+            spec.seed_index = int(rng.integers(n_seeds))
         t0 = time.perf_counter()
         out, lse, off, cols = oracle.sparse_attention(q_host, k_host, v_host, spec, cfg, rows=rows)
         dt = time.perf_counter() - t0
@@ -648,7 +661,9 @@ def main():
         qs.append(q)
         ks.append(k)
         vs.append(v)
-    outs = [[torch.empty(N, Hq, D, dtype=tdt, device=dev) for _ in range(L)] for _ in runs]
+    per_seed = bool(w.get("per_seed"))
+    oshape = lambda ns: (ns, N, Hq, D) if per_seed else (N, Hq, D)  # noqa: E731
+    outs = [[torch.empty(oshape(ns), dtype=tdt, device=dev) for _ in range(L)] for (_, _, _, ns) in runs]
     stream = torch.cuda.current_stream()
     pairs, design = {}, {}
     mask_events = []  # (run, start, mask built, layers done) events of each run while `timing` is set
@@ -659,7 +674,7 @@ def main():
             if timing[0]:
                 mask_events.append((name,) + tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)))
                 mask_events[-1][1].record(stream)
-            m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom)
+            m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom, per_seed=per_seed)
             if timing[0]:
                 mask_events[-1][2].record(stream)
             pairs[name] = m.info().n_pairs
@@ -722,7 +737,7 @@ def main():
     if kinds == [2]:  # every launch on the tensor-core tile kernel
         flops_per_launch = 4 * D * Hq * total_pairs * L / launches_per_step
         achieved = flops_per_launch / (mean_launch_ms / 1e3) / 1e12
-        dense_flops = sum((4 * D * Hq * N * (N + 1) / 2) for _ in runs) * L / launches_per_step
+        dense_flops = sum((4 * D * Hq * N * (N + 1) / 2) * (r[3] if per_seed else 1) for r in runs) * L / launches_per_step
         roofline = {"bound": "tensor", "achieved": achieved, "peak": tc, "unit": "TFLOP/s", "frac": achieved / tc,
                     "traffic": None, "kernel": "k_attn_tile (tcgen05 masked tiles)", "peak_source": ceil["tc_source"],
                     "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
@@ -783,7 +798,7 @@ def main():
     # the sampled-pair roofline: max(sampled FLOPs / tensor peak, min(row, tile) K/V bytes / bandwidth)
     flops = 4 * D * Hq * total_pairs * L
     b_row = total_pairs * L * kv_row_bytes
-    b_tile = len(runs) * L * (N / 128) * (N / 2) * kv_row_bytes
+    b_tile = sum((r[3] if per_seed else 1) for r in runs) * L * (N / 128) * (N / 2) * kv_row_bytes
     in_l2 = N * kv_row_bytes < ceil["l2_bytes"]
     bw = ceil.get("l2_stream_gbs", hbm) if in_l2 else hbm
     t_roof = max(flops / (tc * 1e12), min(b_row, b_tile) / (bw * 1e9))
@@ -811,7 +826,7 @@ def main():
         hq = [t.cpu().pin_memory() for t in qs]
         hk = [t.cpu().pin_memory() for t in ks]
         hv = [t.cpu().pin_memory() for t in vs]
-        ho = [[torch.empty(N, Hq, D, dtype=tdt).pin_memory() for _ in range(L)] for _ in runs]
+        ho = [[torch.empty(oshape(ns), dtype=tdt).pin_memory() for _ in range(L)] for (_, _, _, ns) in runs]
         h2d = sum(t.numel() * t.element_size() for t in hq + hk + hv)
         d2h = sum(t.numel() * t.element_size() for row in ho for t in row)
 
@@ -834,7 +849,7 @@ def main():
                     vs[layer].copy_(hv[layer], non_blocking=True)
                     in_ready[layer].record(h2d_s)
             for ri, (name, mode, dens, ns) in enumerate(runs):
-                m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom)
+                m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom, per_seed=per_seed)
                 for layer in range(L):
                     stream.wait_event(in_ready[layer])
                     if not first[0]:

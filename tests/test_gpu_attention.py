@@ -219,6 +219,15 @@ def test_c6_paper_geometry_64k_layer(mode):
     check_bf16_path(got, ref)
 
 
+def test_c5_ensemble_per_seed_sampled():
+    """Per-seed ensemble at N=65536 (YaRN s=2, 10 seeds in one launch): sampled rows of three seeds."""
+    got, (qn, kn, vn), seeds, rows, _ = _config_case(65536, QWEN, torch.bfloat16, 0, 0.01, 10, 3, True, 24,
+                                                     seed=4, per_seed=True)
+    for s in (0, 5, 9):
+        ref, _ = run_oracle(qn, kn, vn, 0, 0.01, seeds, 3, 1e6, 32768, rows=rows, seed_index=s)
+        check_bf16_path(got[s], ref)
+
+
 def test_c2_ensemble_per_seed_sampled():
     got, (qn, kn, vn), seeds, rows, _ = _config_case(8192, QWEN, torch.bfloat16, 0, 0.01, 10, 1, True, 64,
                                                      per_seed=True)
