@@ -228,8 +228,8 @@ ris_status ris_attention_masked_noalloc(ris_mask_t mask, const void *q, const vo
                                         float *lse, void *stream);
 
 /* Kernel timer for measurement (off by default). While enabled, every attention kernel launch
- * (the fused QK^T -> softmax -> PV kernel, not RoPE or mask kernels) is bracketed by CUDA
- * events recorded on the stream it is launched on. Enabling or disabling clears the record.
+ * (the fused QK^T -> softmax -> PV kernel of a layer, or a decode step's two kernels; not
+ * RoPE or mask kernels) is bracketed by CUDA events recorded on the stream it is launched on. Enabling or disabling clears the record.
  * ris_kernel_timer_read blocks until the last recorded launch has finished, returns the summed
  * device milliseconds and the number of launches recorded since the last read, and clears
  * them. Intended for one thread at a time. Errors: RIS_ERR_INVALID (NULL outputs), RIS_ERR_CUDA. */
@@ -243,10 +243,11 @@ ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches);
  * RIS_FORCE_DESIGN = gather | tma | tile in the environment overrides (benchmarking). */
 int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim);
 
-/* Synchronise `stream` and report (then clear) the device error word set by kernels whose
- * bounded waits gave up: RIS_ERR_DEVICE_TIMEOUT if any did since the last call, else RIS_OK.
- * A kernel that sets the word skips the rest of its work, so outputs of that launch are
- * undefined. Blocks. Errors: RIS_ERR_CUDA. */
+/* Synchronise `stream` and report (then clear) the device error words: RIS_ERR_DEVICE_TIMEOUT
+ * if a kernel's bounded wait gave up since the last call, RIS_ERR_INVALID if a decode step
+ * read a position outside [t0, cache_len) from device memory, else RIS_OK. A kernel that sets
+ * a word skips the rest of its work, so outputs of that launch are undefined. Blocks.
+ * Errors: RIS_ERR_CUDA. */
 ris_status ris_device_status(void *stream);
 
 /* ---- Hybrid Anchor decode (Methods, "Hybrid Anchor and Pre-Fusion Unified Softmax (PFUS)") ----
