@@ -3,12 +3,14 @@
 // set of the first generated token, kept as an ascending list) merged with the Dynamic Local
 // Window t - W < j <= t, with one softmax over the merged set.
 //
-// The merge needs no sort: the anchor keys at or above the window's first key are exactly the
-// duplicates, so the merged set is the anchor list cut at win_lo followed by the contiguous
-// window. The cut is one load from a rank table built with the anchor (rank[j] = anchor keys
-// below j). Key number k of KV head g is anchor[k] for k < nA, else win_lo + (k - nA).
-// Nothing in the launch depends on t, so the position may live in device memory and a
-// captured CUDA graph of a whole token can be replayed token after token.
+// The merge needs no sort and no search: the anchor keys at or after the window's first key
+// win_lo = max(0, t - W + 1) are exactly the duplicates (every anchor key is below t0 <= t).
+// So the CTAs are split into anchor chunks (32 consecutive entries of the anchor list, a key
+// kept iff it is below win_lo) and window chunks (32 consecutive positions from win_lo, kept
+// iff at most t). A CTA needs only its slice of the list and the position, loaded side by
+// side, before it can request its rows; and nothing in the launch depends on t, so the
+// position may live in device memory and a captured CUDA graph of a whole token can be
+// replayed token after token.
 //
 //   k_decode_partial : one CTA per (chunk of 32 keys, KV head): issues all of the chunk's
 //                      16-byte K~ (high + low parts) and V row loads at once, rotates the G
@@ -83,9 +85,10 @@ __device__ __forceinline__ void unpack(const uint4 &u, float *o, const float *)
 
 // One CTA per (chunk of kDecodeChunk keys, KV head); kDecodeCluster consecutive chunks form a
 // thread-block cluster whose first CTA merges the cluster's partials through distributed
-// shared memory, so only one partial per cluster goes to global memory. The dependent global
-// loads on the way to the K/V rows are the position, then (in parallel) its rank-table entry
-// and this chunk's slice of the anchor list, then the rows themselves.
+// shared memory, so only one partial per cluster goes to global memory. Chunks below
+// n_anchor_chunks take anchor entries, the others window positions. On the way to the K/V
+// rows there is one round of dependent global loads: the position and this chunk's slice of
+// the anchor list, side by side.
 template <typename T, bool LO, int D>
 __global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecodeThreads)
     k_decode_partial(const DecodeArgs a)
@@ -106,32 +109,36 @@ __global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecode
     __shared__ float2 rot[kHalf];                 // (cos, sin) of t * f_c
     __shared__ int32_t keys[kDecodeChunk];
 
+    __shared__ uint32_t kept;  // bit r: key r of the chunk is in the merged set
+
     cg::cluster_group cluster = cg::this_cluster();
     const int g = blockIdx.y, chunk = blockIdx.x, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int G = a.G;
     const int m = a.heads_keyed > 1 ? g : 0;
-    const int64_t k0 = (int64_t)chunk * kDecodeChunk;
-    // this thread's anchor slot, loaded alongside the position (the cut decides if it is used)
-    int32_t spec = 0;
-    if (tid < kDecodeChunk && k0 + tid < a.anchor_len[m]) spec = __ldg(a.anchor + a.anchor_base[m] + k0 + tid);
+    const bool from_anchor = chunk < a.n_anchor_chunks;
+    const int64_t k0 = (int64_t)(from_anchor ? chunk : chunk - a.n_anchor_chunks) * kDecodeChunk;
+    // this lane's anchor entry, loaded alongside the position
+    int32_t spec = -1;
+    if (from_anchor && tid < kDecodeChunk && k0 + tid < a.anchor_len[m])
+        spec = __ldg(a.anchor + a.anchor_base[m] + k0 + tid);
     const int64_t t = a.t_dev != nullptr ? *a.t_dev : a.t;
     const bool valid = t >= a.t0 && t < a.cache_len;  // only a device-side t can be outside
     if (!valid && tid == 0 && chunk == 0 && g == 0) atomicOr(&g_ris_decode_error, 2u);
     const int64_t win_lo = t - a.window + 1 > 0 ? t - a.window + 1 : 0;
-    const int64_t nA = valid ? __ldg(a.rank + (int64_t)m * (a.t0 + 1) + (win_lo < a.t0 ? win_lo : a.t0)) : 0;
-    const int64_t n = valid ? nA + (t - win_lo + 1) : 0;
-    const bool active = k0 < n;  // block-uniform; inactive CTAs still take part in the cluster syncs
-    const int nk = active ? (int)((n - k0) < kDecodeChunk ? (n - k0) : kDecodeChunk) : 0;
+    if (warp == 0) {
+        // an anchor key stays unless the window holds it; a window position stays up to t
+        const int64_t key = from_anchor ? (int64_t)spec : win_lo + k0 + lane;
+        const bool in = valid && (from_anchor ? (spec >= 0 && key < win_lo) : key <= t);
+        const uint32_t bits = __ballot_sync(0xFFFFFFFFu, in);
+        keys[lane] = in ? (int32_t)key : 0;  // rows of dropped keys read key 0 and are masked out
+        if (lane == 0) kept = bits;
+    }
+    __syncthreads();
+    const uint32_t kbits = kept;
+    const bool active = kbits != 0u;  // block-uniform; inactive CTAs still take part in the cluster syncs
 
     if (active) {
-        if (tid < kDecodeChunk) {
-            const int64_t kk = k0 + tid;
-            int64_t key = 0;  // rows past the set read key 0 and are masked out below
-            if (kk < n) key = kk < nA ? (int64_t)spec : win_lo + (kk - nA);
-            keys[tid] = (int32_t)key;
-        }
-        __syncthreads();
         // every row load of the chunk is issued before any is used
         uint4 kh[kPieces], kl[kPieces], vv[kPieces];
 #pragma unroll
@@ -190,11 +197,11 @@ __global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecode
                 s2 = fmaf(q4.z, k4.z, s2);
                 s3 = fmaf(q4.w, k4.w, s3);
             }
-            const float x = r < nk ? ((s0 + s1) + (s2 + s3)) * a.scale_log2 : -INFINITY;
+            const float x = ((kbits >> r) & 1u) ? ((s0 + s1) + (s2 + s3)) * a.scale_log2 : -INFINITY;
             float mx = x;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
-            const float p = exp2f(x - mx);  // an active chunk holds at least one key: mx is finite
+            const float p = exp2f(x - mx);  // an active chunk keeps at least one key: mx is finite
             float l = p;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, o);
@@ -210,7 +217,7 @@ __global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecode
             float acc[kPer];
 #pragma unroll
             for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
-            for (int r = 0; r < nk; r += 4) {  // ps beyond nk is 0 and vs rows there are finite
+            for (int r = 0; r < kDecodeChunk; r += 4) {  // dropped keys: p = 0, rows finite
                 const float v0 = vs[r][c], v1 = vs[r + 1][c], v2 = vs[r + 2][c], v3 = vs[r + 3][c];
 #pragma unroll
                 for (int e = 0; e < kPer; ++e) {
@@ -326,35 +333,7 @@ __global__ void __launch_bounds__(kCombineWarps * 32) k_decode_combine(const Dec
     }
 }
 
-// rank[m][j] = lower_bound(keys of list m, j) - start, for j = 0 .. t0
-__global__ void k_anchor_rank(const int32_t *keys, const int64_t *off, int32_t n_masks, int64_t t0, int32_t *rank)
-{
-    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= (int64_t)n_masks * (t0 + 1)) return;
-    const int32_t m = (int32_t)(idx / (t0 + 1));
-    const int64_t j = idx - (int64_t)m * (t0 + 1);
-    int64_t lo = off[m], hi = off[m + 1];
-    const int64_t b = lo;
-    while (lo < hi) {
-        const int64_t mid = (lo + hi) >> 1;
-        if ((int64_t)keys[mid] < j)
-            lo = mid + 1;
-        else
-            hi = mid;
-    }
-    rank[idx] = (int32_t)(lo - b);
-}
-
 }  // namespace
-
-cudaError_t launch_anchor_rank(const int32_t *keys, const int64_t *off, int32_t n_masks, int64_t t0, int32_t *rank,
-                               cudaStream_t s)
-{
-    const int64_t n = (int64_t)n_masks * (t0 + 1);
-    k_anchor_rank<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(keys, off, n_masks, t0, rank);
-    note_launch();
-    return cudaGetLastError();
-}
 
 unsigned int read_decode_error()
 {

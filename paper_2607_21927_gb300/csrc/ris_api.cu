@@ -50,7 +50,6 @@ struct ris_anchor_s {
     int32_t heads_keyed = 1, kv_heads = 1;
     int32_t *keys = nullptr;  // device, ascending per mask
     int64_t *off = nullptr;   // device, heads_keyed + 1 offsets
-    int32_t *rank = nullptr;  // device, [heads_keyed][t0 + 1]: keys below j
     int64_t max_keys = 0;     // longest list
     std::vector<int64_t> h_off;
     void *scratch = nullptr;  // decode partials, reused by every step on this anchor
@@ -806,8 +805,6 @@ ris_status ris_decode_anchor(int64_t n_prefill, int32_t kv_heads, int32_t mode, 
     f.row_ptr = an->off;
     f.col = an->keys;
     RIS_CUDA(launch_mask_fill(f, s));
-    RIS_CUDA(cudaMallocAsync((void **)&an->rank, sizeof(int32_t) * (size_t)(hk * (t0 + 1)), s));
-    RIS_CUDA(launch_anchor_rank(an->keys, an->off, hk, t0, an->rank, s));
     for (int32_t m = 0; m < hk; ++m) an->max_keys = std::max(an->max_keys, an->h_off[m + 1] - an->h_off[m]);
     RIS_CUDA(cudaStreamSynchronize(s));
     guard.a = nullptr;
@@ -831,7 +828,7 @@ ris_status ris_anchor_free(ris_anchor_t anchor)
 {
     if (anchor == nullptr) return RIS_OK;
     cudaError_t e = cudaSuccess;
-    for (void *p : {(void *)anchor->keys, (void *)anchor->off, (void *)anchor->rank, anchor->scratch}) {
+    for (void *p : {(void *)anchor->keys, (void *)anchor->off, anchor->scratch}) {
         if (p == nullptr) continue;
         cudaError_t e2 = cudaFreeAsync(p, anchor->stream);
         if (e == cudaSuccess) e = e2;
@@ -905,7 +902,6 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
         a.anchor_base[m] = anchor->h_off[m];
         a.anchor_len[m] = (int32_t)(anchor->h_off[m + 1] - anchor->h_off[m]);
     }
-    a.rank = anchor->rank;
     a.t0 = anchor->t0;
     a.cache_len = cache_len;
     a.heads_keyed = anchor->heads_keyed;
@@ -917,8 +913,9 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     a.advance = advance;
     a.t = t;
     a.t_dev = t_dev;
-    // the grid covers the largest merged set (every anchor key plus a full window), whatever t is
-    const int64_t chunks = (anchor->max_keys + window + kDecodeChunk - 1) / kDecodeChunk;
+    // anchor chunks cover the longest list, window chunks a full window, whatever t is
+    a.n_anchor_chunks = (int32_t)((anchor->max_keys + kDecodeChunk - 1) / kDecodeChunk);
+    const int64_t chunks = a.n_anchor_chunks + ((int64_t)window + kDecodeChunk - 1) / kDecodeChunk;
     a.n_groups = (int32_t)((chunks + kDecodeCluster - 1) / kDecodeCluster);
     a.n_chunks = a.n_groups * kDecodeCluster;
     double ms = 1.0;

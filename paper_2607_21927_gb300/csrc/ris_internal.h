@@ -90,10 +90,10 @@ struct AttnArgs {
 };
 
 // Arguments of the Hybrid Anchor decode kernels (one generated token at position t). The
-// key set of KV head g is its anchor keys below win_lo = max(0, t - W + 1) (their count is
-// rank[min(win_lo, t0)]) followed by the window win_lo .. t; it is cut into chunks of
-// kDecodeChunk keys, one CTA per (chunk, g). The grid covers the largest possible set
-// (anchor size + W), so it does not depend on t, and t may be read from device memory.
+// key set of KV head g is its anchor keys below win_lo = max(0, t - W + 1) plus the window
+// win_lo .. t: chunks of kDecodeChunk anchor entries, then chunks of kDecodeChunk window
+// positions, one CTA per (chunk, g). The grid does not depend on t, so t may be read from
+// device memory.
 constexpr int kDecodeChunk = 32;
 constexpr int kDecodeCluster = 8;  // chunks merged on chip per partial written
 constexpr int kMaxDecodeKvHeads = 64;
@@ -106,7 +106,6 @@ struct DecodeArgs {
     const int32_t *anchor;     // anchor keys, ascending; mask m: anchor[anchor_base[m] ..] (anchor_len[m] keys)
     int64_t anchor_base[kMaxDecodeKvHeads];
     int32_t anchor_len[kMaxDecodeKvHeads];
-    const int32_t *rank;       // [heads_keyed][t0 + 1]: anchor keys of mask m below j
     int64_t t0;                // first generated position (the prefill length)
     int64_t cache_len;
     int32_t heads_keyed;       // 1, or Hkv for per-head anchors
@@ -115,6 +114,7 @@ struct DecodeArgs {
     int32_t G;
     int32_t D;
     int32_t n_chunks;          // chunks per KV head (grid.x), a multiple of kDecodeCluster
+    int32_t n_anchor_chunks;   // the first n_anchor_chunks chunks take anchor entries
     int32_t n_groups;          // n_chunks / kDecodeCluster: partials per KV head
     int32_t window;            // W >= 1
     int32_t advance;           // with t_dev: the combine kernel adds 1 to *t_dev when done
@@ -145,9 +145,6 @@ cudaError_t launch_mask_fill(const MaskFillArgs &a, cudaStream_t s);
 
 // Decode step: partial softmax per (chunk, KV head), then one combine per query head.
 cudaError_t launch_decode(const DecodeArgs &a, int dtype, int out_dtype, cudaStream_t s);
-// rank[m][j] = number of keys of anchor list m below j, j = 0 .. t0
-cudaError_t launch_anchor_rank(const int32_t *keys, const int64_t *off, int32_t n_masks, int64_t t0, int32_t *rank,
-                               cudaStream_t s);
 // Reads and clears the decode error word (bit 1: a step's device-side t was out of range).
 unsigned int read_decode_error();
 
