@@ -711,7 +711,7 @@ def main():
         torch.cuda.synchronize()
         timing[0] = False
     launches = ris.ris_launch_count() - n0
-    k_ms, k_n = ris.ris_kernel_timer_read()
+    k_ms, k_n, k_each = ris.ris_kernel_timer_samples()
     ris.ris_kernel_timer_enable(False)
     barrier(dist)
     elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1), dist)
@@ -731,6 +731,12 @@ def main():
     # algorithmic FLOPs (tiles) per launch / mean launch time
     launches_per_step = len(runs) * L
     mean_launch_ms = k_ms / max(k_n, 1)
+    median_launch_ms = statistics.median(k_each) if k_each else None
+    per_run_ms = {}  # launches are recorded run by run within each step, L per run
+    if len(k_each) == launches_per_step * a.steps:
+        for i, ms_i in enumerate(k_each):
+            per_run_ms.setdefault(runs[(i % launches_per_step) // L][0], []).append(ms_i)
+    median_per_run = {k: statistics.median(v) for k, v in per_run_ms.items()}
     kinds = sorted(set(design.values()))
     hbm, tc = ceil["hbm_gbs"], ceil["tc_tflops"]
     kv_row_bytes = Hkv * 2 * D * e  # K and V rows of one key, all KV heads
@@ -741,7 +747,8 @@ def main():
         roofline = {"bound": "tensor", "achieved": achieved, "peak": tc, "unit": "TFLOP/s", "frac": achieved / tc,
                     "traffic": None, "kernel": "k_attn_tile (tcgen05 masked tiles)", "peak_source": ceil["tc_source"],
                     "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
-                    "mean_launch_ms": mean_launch_ms, "launches_timed": k_n,
+                    "mean_launch_ms": mean_launch_ms, "median_launch_ms": median_launch_ms,
+                    "median_launch_ms_per_run": median_per_run, "launches_timed": k_n,
                     "design_frac": (dense_flops / (tc * 1e12)) / (mean_launch_ms / 1e3),
                     "design_note": "dense-causal tile FLOPs / sustained bf16 peak over the launch time (the "
                                    "kernel issues 2.5x that in hi/lo split products)"}
@@ -754,7 +761,8 @@ def main():
                     "kernel": gather.get(kinds[0], "?") if len(kinds) == 1 else "mixed designs " + str(kinds),
                     "peak_source": ceil["hbm_source"],
                     "bytes": "algorithmic: K and V rows of every sampled pair, all KV heads",
-                    "mean_launch_ms": mean_launch_ms, "launches_timed": k_n}
+                    "mean_launch_ms": mean_launch_ms, "median_launch_ms": median_launch_ms,
+                    "median_launch_ms_per_run": median_per_run, "launches_timed": k_n}
         kv_set = N * Hkv * D * e * (3 if e == 2 else 2)  # rotated K (hi + lo for bf16) and V of a layer
         if "l2_rows_gbs" in ceil and kv_set < ceil["l2_bytes"]:
             # the K/V working set is L2-resident: the gathered rows are served from L2, so L2 is

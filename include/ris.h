@@ -235,6 +235,9 @@ ris_status ris_attention_masked_noalloc(ris_mask_t mask, const void *q, const vo
  * them. Intended for one thread at a time. Errors: RIS_ERR_INVALID (NULL outputs), RIS_ERR_CUDA. */
 ris_status ris_kernel_timer_enable(int32_t enable);
 ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches);
+/* As ris_kernel_timer_read, and also the duration of each of the first `capacity` recorded
+ * launches, in launch order, into the HOST array ms_each (NULL when capacity is 0). */
+ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double *ms_each, int64_t capacity);
 
 /* Attention kernel design a layer call on `mask` uses for this input dtype and head_dim
  * (host-only, no device work): 0 register gather, 1 TMA gather, 2 tcgen05 masked dense tiles,

@@ -649,21 +649,30 @@ ris_status ris_kernel_timer_enable(int32_t enable)
     return RIS_OK;
 }
 
-ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches)
+ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double *ms_each, int64_t capacity)
 {
     if (total_ms == nullptr || launches == nullptr) return fail(RIS_ERR_INVALID, "output pointer is NULL");
+    if (capacity < 0 || (capacity > 0 && ms_each == nullptr)) return fail(RIS_ERR_INVALID, "ms_each / capacity");
     std::lock_guard<std::mutex> lk(g_timer.mu);
     double tot = 0.0;
+    int64_t k = 0;
     for (auto &e : g_timer.used) {
         RIS_CUDA(cudaEventSynchronize(e.second));
         float ms = 0.f;
         RIS_CUDA(cudaEventElapsedTime(&ms, e.first, e.second));
         tot += ms;
+        if (k < capacity) ms_each[k] = ms;
+        ++k;
     }
     *total_ms = tot;
     *launches = (int64_t)g_timer.used.size();
     timer_clear_locked();
     return RIS_OK;
+}
+
+ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches)
+{
+    return ris_kernel_timer_samples(total_ms, launches, nullptr, 0);
 }
 
 int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim)

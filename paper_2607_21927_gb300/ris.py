@@ -99,6 +99,7 @@ _SIGS = {
     "ris_device_status": [ctypes.c_void_p],
     "ris_attention_design": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32],
     "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
+    "ris_kernel_timer_samples": [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64],
     "ris_decode_anchor": [ctypes.c_int64, ctypes.c_int32, ctypes.c_int32, ctypes.c_double, ctypes.c_void_p,
                           ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p],
     "ris_anchor_info": [ctypes.c_void_p] * 6,
@@ -171,6 +172,15 @@ def ris_kernel_timer_read():
     ms, n = ctypes.c_double(), ctypes.c_int64()
     _check("ris_kernel_timer_read", lib().ris_kernel_timer_read(ctypes.byref(ms), ctypes.byref(n)))
     return ms.value, n.value
+
+
+def ris_kernel_timer_samples(capacity: int = 4096):
+    """(summed device ms, launches, [ms of each recorded launch]) since the last read."""
+    ms, n = ctypes.c_double(), ctypes.c_int64()
+    buf = (ctypes.c_double * max(1, int(capacity)))()
+    _check("ris_kernel_timer_samples", lib().ris_kernel_timer_samples(ctypes.byref(ms), ctypes.byref(n), buf,
+                                                                      int(capacity)))
+    return ms.value, n.value, list(buf[:min(n.value, int(capacity))])
 
 
 def ris_probe_l2_read(working_set: int, pattern: int = 0, stream=None) -> float:
