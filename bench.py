@@ -69,6 +69,10 @@ WORKLOADS = {
     "C5": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
                runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)],
                title="Qwen2-1.5B-shaped prefill attention stack, N=65536, 28 layers, YaRN s=2"),
+    # C5 with the index-draw sampler (the torch.randint reading): K = round(dN) draws per row and seed
+    "C5r": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
+                runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)], sampler=1,
+                title="C5 with the index-draw sampler"),
     # C5 with the paper's full geometry: local window 1024 and anchors over the first tokens
     "C6": dict(N=65536, layers=28, Hq=12, Hkv=2, D=128, dtype="bf16", outliers=True, rope=("yarn", 1e6, 32768),
                runs=[("stochastic", 0, 0.01, 10), ("structural", 1, 0.01, 10)], geometry="paper",
@@ -148,6 +152,7 @@ def workload_config(a):
         "runs": [{"name": n, "mode": m, "density": d, "seeds": s} for n, m, d, s in w["runs"]],
         "input_dtype": w["dtype"], "outlier_channels": "1% x8" if w["outliers"] else None,
         "geometry": ("local window 1024 + 4 anchors" if w.get("geometry") == "paper" else "diagonal only"),
+        "sampler": "index draws (K = round(dN) per row and seed)" if w.get("sampler") else "Bernoulli per pair",
         "seed_outputs": "one per seed (per-seed masks)" if w.get("per_seed") else "one (union of the seeds)",
         "l2": (f"inputs larger than L2: each layer has its own q/k/v ({per_layer / 2**20:.0f} MiB), "
                f"{w['layers']} layers = {w['layers'] * per_layer / 2**20:.0f} MiB per run"),
@@ -278,7 +283,8 @@ def oracle_sample(q_host, k_host, v_host, w, run, target_s, rng_seed):
     name, mode, density, n_seeds = run
     paper = w.get("geometry") == "paper"
     spec = oracle.MaskSpec(N=N, mode=mode, density=density, seeds=list(range(n_seeds)),
-                           local_window=1024 if paper else 1, n_anchor=4 if paper else 0)
+                           local_window=1024 if paper else 1, n_anchor=4 if paper else 0,
+                           sampler=int(w.get("sampler", 0)))
     cfg = oracle_rope(w)
     rng = np.random.default_rng(rng_seed)
     nrows, total_ph, total_t, used = 8, 0, 0.0, 0
@@ -653,6 +659,8 @@ def main():
     kind, theta, native = w["rope"]
     rope = ris.rope_cfg(ROPE_KINDS[kind], theta, native)
     geom = ris.paper_geometry() if w.get("geometry") == "paper" else None
+    if w.get("sampler"):
+        geom = ris.mask_opts(sampler=w["sampler"])
 
     # inputs resident in HBM: one (q, k, v) per layer, layer L drawn from seed L
     qs, ks, vs = [], [], []
