@@ -206,6 +206,27 @@ ris_status ris_ensemble_batch(const void *q, const void *k, const void *v, void 
                               int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
                               const ris_mask_opts *opts, float *lse, void *stream);
 
+/* Query rows row_begin .. row_end-1 of ris_attention_masked (same arguments otherwise): the
+ * other rows of out and lse are left untouched, and each computed row equals the same row of
+ * the whole-layer call bit for bit. K and V must still hold every position (any row may
+ * attend to any earlier key). This is how one prefill is split across devices or streams:
+ * query rows are independent given K, V and the counter-based mask (each device can build the
+ * same mask), so each part needs no exchange. Errors: as ris_attention_masked, and
+ * RIS_ERR_INVALID for an empty range or one outside [0, N). */
+ris_status ris_attention_masked_rows(ris_mask_t mask, int64_t row_begin, int64_t row_end, const void *q,
+                                     const void *k, const void *v, void *out, int32_t heads, int32_t kv_heads,
+                                     int32_t head_dim, int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
+                                     float *lse, void *stream);
+
+/* Balanced contiguous row ranges for `parts` workers: bounds[0] = 0 < bounds[1] < ... <
+ * bounds[parts] = N, cut where the running sampled-pair count reaches k/parts of the total
+ * (every part gets at least one row). ris_row_split takes a HOST row_ptr of N + 1 offsets
+ * (no device work); ris_mask_row_split reads the mask's own counts (summed over its per-seed
+ * or per-head masks; row i of a dense mask counts i + 1) and blocks. Errors: RIS_ERR_INVALID
+ * (NULL, parts outside [1, N]), RIS_ERR_CUDA. */
+ris_status ris_row_split(const int64_t *row_ptr, int64_t N, int32_t parts, int64_t *bounds);
+ris_status ris_mask_row_split(ris_mask_t mask, int32_t parts, int64_t *bounds);
+
 /* Allocation-free variant of ris_attention_masked (same arguments, results and errors).
  * The paper has no counterpart: this entry point exists for callers that may not allocate
  * device memory while a layer runs, such as an inference engine's enqueue callback that may

@@ -12,8 +12,8 @@ namespace ris {
 constexpr int kAttnWarps = 4;  // tasks (one per warp) per CTA
 constexpr float kLn2 = 0.69314718055994530942f;
 
-// A task is (output set s, row i, KV head g). Rows are handed out from the last (longest
-// key list) to the first so the short rows fill the tail of the grid.
+// A task is (output set s, row i, KV head g), row0 <= i < row1. Rows are handed out from the
+// last (longest key list) to the first so the short rows fill the tail of the grid.
 struct Task {
     int64_t i;
     int g;
@@ -27,7 +27,7 @@ __device__ __forceinline__ Task decode_task(const AttnArgs &a, int64_t t)
     k.g = (int)(t % a.Hkv);
     const int64_t r = t / a.Hkv;
     k.s = (int)(r % a.n_sets);
-    k.i = a.N - 1 - r / a.n_sets;
+    k.i = a.row1 - 1 - r / a.n_sets;
     k.mask_id = k.s * a.heads_keyed + (a.heads_keyed > 1 ? k.g : 0);
     return k;
 }

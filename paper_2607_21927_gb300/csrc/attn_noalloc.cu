@@ -171,6 +171,8 @@ extern "C" ris_status ris_attention_masked_noalloc(ris_mask_t mask, const void *
     a.heads_keyed = md.heads_keyed;
     a.n_sets = md.per_seed ? md.n_seeds : 1;
     a.scale_log2 = (float)(1.4426950408889634074 / std::sqrt((double)head_dim));
+    a.row0 = 0;
+    a.row1 = N;
     a.n_tasks = (int64_t)a.n_sets * N * kv_heads;
     cudaError_t e = dtype == RIS_BF16
                         ? launch_attention_bf16(a, head_dim, out_dtype, q_split, md.col_bytes, md.dense != 0, s)

@@ -259,17 +259,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t sbase = smem_u32(smem);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    // ---- tile of this CTA: heavier (later) query tiles first
-    const int n_qt = (int)((a.N + BM - 1) / BM);
+    // ---- tile of this CTA (tiles covering rows row0 .. row1-1): heavier (later) tiles first
+    const int qt_end = (int)((a.row1 + BM - 1) / BM);
     const int64_t b = blockIdx.x;
     const int h = (int)(b % a.Hq);
     const int64_t r2 = b / a.Hq;
     const int s = (int)(r2 % a.n_sets);
-    const int qt = n_qt - 1 - (int)(r2 / a.n_sets);
+    const int qt = qt_end - 1 - (int)(r2 / a.n_sets);
     const int64_t q0 = (int64_t)qt * BM;
     const int g = h / a.G;
     const int mask_id = s * a.heads_keyed + (a.heads_keyed > 1 ? g : 0);
-    const int64_t last_row = (q0 + BM - 1 < a.N - 1) ? q0 + BM - 1 : a.N - 1;
+    const int64_t last_row = (q0 + BM - 1 < a.row1 - 1) ? q0 + BM - 1 : a.row1 - 1;
     const int n_kt = (int)(last_row / BN) + 1;  // causal: key tiles 0 .. last_row / BN
 
     if (threadIdx.x == 0) {
@@ -394,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int wq = warp & 3, hf = warp >> 2;
         const int r = wq * 32 + lane;  // TMEM lane
         const int64_t i = q0 + r;
-        const bool row_ok = i < a.N;
+        const bool row_ok = i >= a.row0 && i < a.row1;
         const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
         const uint32_t *bm = DENSE ? nullptr
                                    : a.bitmap + (int64_t)mask_id * a.words_per_mask + (row_ok ? row_word_offset(i) : 0);
@@ -570,7 +570,7 @@ cudaError_t launch_t(const AttnArgs &a, const TileMaps &maps, const void *q_hi, 
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    const int64_t n_qt = (a.N + BM - 1) / BM;
+    const int64_t n_qt = (a.row1 + BM - 1) / BM - a.row0 / BM;  // tiles covering rows row0 .. row1-1
     const unsigned grid = (unsigned)(n_qt * a.Hq * a.n_sets);
     kern<<<grid, kThreads, SMEM_BYTES, s>>>(a, maps, q_hi, q_lo);
     note_launch();

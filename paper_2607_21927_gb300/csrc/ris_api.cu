@@ -537,12 +537,13 @@ ris_status ris_rope_apply(void *x, int32_t dtype, int64_t N, int32_t heads, int3
 
 namespace {
 
-// Attention over an existing mask; arguments already validated.
+// Attention of query rows row0 .. row1-1 over an existing mask; arguments already validated.
 ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, const void *v, void *out,
                          int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t dtype, int32_t out_dtype,
-                         const ris_rope_cfg *rope, float *lse, cudaStream_t s)
+                         const ris_rope_cfg *rope, float *lse, cudaStream_t s, int64_t row0 = 0, int64_t row1 = -1)
 {
     const int64_t N = m->N;
+    if (row1 < 0) row1 = N;
     prepare_pool_once();
     const bool tile = dtype == RIS_BF16 && head_dim == 128 && use_tile_design(m);
     Scratch qt, qtl, kt, ktl;
@@ -601,7 +602,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.heads_keyed = m->heads_keyed;
     a.n_sets = m->per_seed ? m->n_seeds : 1;
     a.scale_log2 = (float)(1.4426950408889634074 / std::sqrt((double)head_dim));
-    a.n_tasks = (int64_t)a.n_sets * N * kv_heads;
+    a.row0 = row0;
+    a.row1 = row1;
+    a.n_tasks = (int64_t)a.n_sets * (row1 - row0) * kv_heads;
     const auto ev = timer_pair();
     if (ev.first) RIS_CUDA(cudaEventRecord(ev.first, s));
     if (tile)
@@ -706,6 +709,68 @@ ris_status ris_attention_masked(ris_mask_t mask, const void *q, const void *k, c
         return fail(RIS_ERR_INVALID, "mask keyed for %d KV heads, call has %d", mask->heads_keyed, kv_heads);
     return run_attention(mask, q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse,
                          reinterpret_cast<cudaStream_t>(stream));
+}
+
+ris_status ris_attention_masked_rows(ris_mask_t mask, int64_t row_begin, int64_t row_end, const void *q,
+                                     const void *k, const void *v, void *out, int32_t heads, int32_t kv_heads,
+                                     int32_t head_dim, int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
+                                     float *lse, void *stream)
+{
+    if (mask == nullptr) return fail(RIS_ERR_INVALID, "mask is NULL");
+    RIS_TRY(validate_attention(q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse));
+    if (mask->heads_keyed > 1 && mask->heads_keyed != kv_heads)
+        return fail(RIS_ERR_INVALID, "mask keyed for %d KV heads, call has %d", mask->heads_keyed, kv_heads);
+    if (row_begin < 0 || row_end > mask->N || row_begin >= row_end)
+        return fail(RIS_ERR_INVALID, "rows [%lld, %lld) not a non-empty range of [0, %lld)", (long long)row_begin,
+                    (long long)row_end, (long long)mask->N);
+    return run_attention(mask, q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse,
+                         reinterpret_cast<cudaStream_t>(stream), row_begin, row_end);
+}
+
+ris_status ris_row_split(const int64_t *row_ptr, int64_t N, int32_t parts, int64_t *bounds)
+{
+    if (row_ptr == nullptr || bounds == nullptr) return fail(RIS_ERR_INVALID, "row_ptr or bounds is NULL");
+    RIS_TRY(check_N(N));
+    if (parts < 1 || parts > N) return fail(RIS_ERR_INVALID, "parts %d outside [1, N]", parts);
+    // cut k: the first row whose prefix of pairs reaches k / parts of the total (each part
+    // gets at least one row)
+    const int64_t total = row_ptr[N] - row_ptr[0];
+    bounds[0] = 0;
+    int64_t r = 0;
+    for (int32_t k = 1; k < parts; ++k) {
+        const double target = (double)total * k / parts;
+        while (r < N && (double)(row_ptr[r] - row_ptr[0]) < target) ++r;
+        int64_t c = r;
+        if (c < bounds[k - 1] + 1) c = bounds[k - 1] + 1;
+        if (c > N - (parts - k)) c = N - (parts - k);
+        bounds[k] = c;
+    }
+    bounds[parts] = N;
+    return RIS_OK;
+}
+
+ris_status ris_mask_row_split(ris_mask_t mask, int32_t parts, int64_t *bounds)
+{
+    if (mask == nullptr || bounds == nullptr) return fail(RIS_ERR_INVALID, "mask or bounds is NULL");
+    const int64_t N = mask->N;
+    if (parts < 1 || parts > N) return fail(RIS_ERR_INVALID, "parts %d outside [1, N]", parts);
+    std::vector<int64_t> rp((size_t)N + 1);
+    RIS_CUDA(cudaStreamSynchronize(mask->stream));
+    if (mask->dense) {
+        for (int64_t i = 0; i <= N; ++i) rp[(size_t)i] = i * (i + 1) / 2;  // row i holds keys 0..i
+    } else {
+        // per-seed or per-head masks: the cost of row i is summed over the masks
+        std::vector<int64_t> all((size_t)(mask->n_masks * N + 1));
+        RIS_CUDA(cudaMemcpy(all.data(), mask->row_ptr, sizeof(int64_t) * all.size(), cudaMemcpyDeviceToHost));
+        rp[0] = 0;
+        for (int64_t i = 0; i < N; ++i) {
+            int64_t c = 0;
+            for (int32_t mm = 0; mm < mask->n_masks; ++mm)
+                c += all[(size_t)(mm * N + i + 1)] - all[(size_t)(mm * N + i)];
+            rp[(size_t)i + 1] = rp[(size_t)i] + c;
+        }
+    }
+    return ris_row_split(rp.data(), N, parts, bounds);
 }
 
 ris_status ris_sparse_attention_fwd(const void *q, const void *k, const void *v, void *out, int64_t N,

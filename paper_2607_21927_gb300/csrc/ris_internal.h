@@ -84,9 +84,11 @@ struct AttnArgs {
     int32_t G;             // Hq / Hkv
     int32_t heads_keyed;   // masks keyed per KV head (1 or Hkv)
     int32_t n_sets;        // output sets: n_seeds for per-seed masks, else 1
+    int64_t row0;          // query rows row0 .. row1-1 are computed (0 and N for a whole layer)
+    int64_t row1;
     int32_t pad_;
     float scale_log2;      // log2(e) / sqrt(D)
-    int64_t n_tasks;       // n_sets * N * Hkv
+    int64_t n_tasks;       // n_sets * (row1 - row0) * Hkv
 };
 
 // Arguments of the Hybrid Anchor decode kernels (one generated token at position t). The

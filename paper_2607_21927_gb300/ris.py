@@ -98,6 +98,10 @@ _SIGS = {
     "ris_kernel_timer_enable": [ctypes.c_int32],
     "ris_device_status": [ctypes.c_void_p],
     "ris_attention_design": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32],
+    "ris_attention_masked_rows": [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64] + [ctypes.c_void_p] * 4 +
+                                 [ctypes.c_int32] * 5 + [ctypes.c_void_p] * 3,
+    "ris_row_split": [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p],
+    "ris_mask_row_split": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p],
     "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
     "ris_kernel_timer_samples": [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64],
     "ris_decode_anchor": [ctypes.c_int64, ctypes.c_int32, ctypes.c_int32, ctypes.c_double, ctypes.c_void_p,
@@ -498,4 +502,33 @@ def ris_decode_step(anchor: Anchor, q: torch.Tensor, k: torch.Tensor, k_lo: Opti
         int(window), int(Hq), int(Hkv), int(D), _dtype(q), _dtype(out), int(n_ctx), _ref(rope), _ptr(out), _ptr(lse),
         _stream(stream)))
     return (out, lse) if return_lse else out
+
+
+# ----------------------------------------------------------------------------- row ranges
+def ris_attention_masked_rows(mask: Mask, row_begin: int, row_end: int, q, k, v, out: torch.Tensor,
+                              rope: Optional[RopeCfg] = None, lse: Optional[torch.Tensor] = None, stream=None):
+    """Rows row_begin .. row_end-1 of ris_attention_masked into `out` (other rows untouched)."""
+    N, Hq, Hkv, D = _shapes(q, k, v)
+    assert out.is_cuda and out.is_contiguous()
+    _check("ris_attention_masked_rows", lib().ris_attention_masked_rows(
+        mask.handle, int(row_begin), int(row_end), _ptr(q), _ptr(k), _ptr(v), _ptr(out), Hq, Hkv, D, _dtype(q),
+        _dtype(out), _ref(rope), _ptr(lse), _stream(stream)))
+    return out
+
+
+def ris_row_split(row_ptr, parts: int):
+    """Balanced row bounds (parts + 1 of them) from a host row_ptr of N + 1 offsets."""
+    import numpy as np
+
+    rp = np.ascontiguousarray(np.asarray(row_ptr, dtype=np.int64))
+    b = np.empty(int(parts) + 1, dtype=np.int64)
+    _check("ris_row_split", lib().ris_row_split(rp.ctypes.data, int(rp.shape[0] - 1), int(parts), b.ctypes.data))
+    return b.tolist()
+
+
+def ris_mask_row_split(mask: Mask, parts: int):
+    """Balanced row bounds (parts + 1 of them) by the mask's sampled-pair counts."""
+    b = (ctypes.c_int64 * (int(parts) + 1))()
+    _check("ris_mask_row_split", lib().ris_mask_row_split(mask.handle, int(parts), b))
+    return list(b)
 

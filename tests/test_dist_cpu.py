@@ -53,3 +53,79 @@ def test_single_process_needs_no_process_group(monkeypatch):
 
     assert bench.dist_init() == (0, 1, None)
     assert bench.max_over_ranks(3.5, None) == 3.5
+
+
+# ----------------------------------------------------------------------------- row sharding
+def _oracle_row_ptr(N, d, S):
+    import numpy as np
+
+    import oracle
+
+    counts = oracle.mask_counts(oracle.MaskSpec(N=N, mode=0, density=d, seeds=list(range(S))))
+    return np.concatenate([[0], np.cumsum(counts)]).astype(np.int64)
+
+
+def test_row_split_balances_pairs():
+    """Balanced cuts of a causal mask's rows: contiguous, non-empty, each part's pair count
+    within one row's count of total / parts (rows near the end cost more)."""
+    import numpy as np
+
+    from paper_2607_21927_gb300 import ris
+
+    rp = _oracle_row_ptr(3000, 0.05, 3)
+    total = int(rp[-1])
+    for parts in (1, 2, 3, 7, 64):
+        b = ris.ris_row_split(rp, parts)
+        assert b[0] == 0 and b[-1] == 3000 and all(b[k] < b[k + 1] for k in range(parts))
+        sizes = [int(rp[b[k + 1]] - rp[b[k]]) for k in range(parts)]
+        biggest_row = int(np.diff(rp).max())
+        assert max(abs(sz - total / parts) for sz in sizes) <= biggest_row + 1
+    b = ris.ris_row_split(np.arange(11, dtype=np.int64), 10)  # ten one-pair rows, ten parts
+    assert b == list(range(11))
+    with pytest.raises(ris.RisError):
+        ris.ris_row_split(rp, 0)
+    with pytest.raises(ris.RisError):
+        ris.ris_row_split(rp, 3001)
+
+
+def _shard_rank(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
+                      LOCAL_RANK=str(rank))
+    sys.path.insert(0, ROOT)
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_21927_gb300 import ris
+
+    dist.init_process_group("gloo")
+    # every rank derives the same counts (the mask is a pure function of its seeds) and takes
+    # its own part: no exchange of mask data between ranks
+    rp = _oracle_row_ptr(2000, 0.03, 2)
+    b = ris.ris_row_split(rp, world)
+    mine = torch.tensor([b[rank], b[rank + 1], int(rp[b[rank + 1]] - rp[b[rank]])], dtype=torch.int64)
+    got = [torch.zeros(3, dtype=torch.int64) for _ in range(world)]
+    dist.all_gather(got, mine)
+    q.put((rank, [g.tolist() for g in got], int(rp[-1])))
+    dist.destroy_process_group()
+
+
+@pytest.mark.timeout(120)
+def test_row_shards_partition_rows_gloo(monkeypatch):
+    """Two gloo ranks take balanced row ranges of the same mask: together they cover every row
+    once and every sampled pair once."""
+    monkeypatch.setenv("CUDA_VISIBLE_DEVICES", "")
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_shard_rank, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(90)
+        assert p.exitcode == 0
+    res = sorted(q.get(timeout=5) for _ in range(2))
+    parts, total = res[0][1], res[0][2]
+    assert res[1][1] == parts
+    assert parts[0][0] == 0 and parts[0][1] == parts[1][0] and parts[1][1] == 2000
+    assert parts[0][2] + parts[1][2] == total and abs(parts[0][2] - parts[1][2]) <= 0.01 * total

@@ -260,3 +260,30 @@ def test_dense_tiles_bf16_output_and_lse():
     ref, ref_lse = run_oracle(qn, kn, vn, 0, 0.5, [1, 2], 3, 1e6, 256)
     check_bf16_path(to_np(out), ref, out_bf16=True)
     np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-2)
+
+
+@pytest.mark.parametrize("d,S,D", [(0.02, 3, 128), (0.5, 2, 128), (1.0, 1, 128), (0.03, 2, 64)],
+                         ids=["gather", "tiles", "dense", "hd64"])
+def test_row_ranges_reassemble_the_layer(d, S, D):
+    """Balanced row ranges computed one call each reassemble the whole-layer output bit for bit
+    (gather and tile designs, ranges that cut through 128-row tiles)."""
+    N, Hq, Hkv = 1500, 6, 2
+    (q, k, v), _ = make_inputs(N, Hq, Hkv, D, seed=17, outliers=True)
+    mode = 2 if d >= 1.0 else 0
+    m = ris.ris_mask_generate(N, Hkv, mode, d, list(range(S)))
+    rope = ris.rope_cfg(3, 1e6, 256)
+    whole = ris.ris_attention_masked(m, q, k, v, rope=rope, out_dtype=torch.float32)
+    bounds = ris.ris_mask_row_split(m, 3)
+    assert bounds[0] == 0 and bounds[-1] == N and sorted(set(bounds)) == bounds
+    parts = torch.full_like(whole, float("nan"))
+    for r0, r1 in zip(bounds[:-1], bounds[1:]):
+        ris.ris_attention_masked_rows(m, r0, r1, q, k, v, parts, rope=rope)
+    torch.cuda.synchronize()
+    assert torch.equal(parts, whole)
+    one = torch.full_like(whole, float("nan"))
+    ris.ris_attention_masked_rows(m, 700, 701, q, k, v, one, rope=rope)
+    torch.cuda.synchronize()
+    assert torch.equal(one[700], whole[700]) and torch.isnan(one[:700]).all() and torch.isnan(one[701:]).all()
+    with pytest.raises(ris.RisError):
+        ris.ris_attention_masked_rows(m, 5, 5, q, k, v, one, rope=rope)
+    m.free()
