@@ -115,6 +115,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle CPU baseline")
     ap.add_argument("--no-probes", action="store_true", help="skip the L2 / FFMA ceiling probes")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle seconds per step")
+    ap.add_argument("--shard", choices=("replicas", "rows"), default="replicas",
+                    help="with several ranks: every rank runs the whole workload (weak scaling), or each "
+                         "rank takes a balanced range of query rows of the same workload (strong scaling)")
     a = ap.parse_args()
     w = dict(WORKLOADS[a.workload])
     w["name"] = a.workload
@@ -154,6 +157,8 @@ def workload_config(a):
         "geometry": ("local window 1024 + 4 anchors" if w.get("geometry") == "paper" else "diagonal only"),
         "sampler": "index draws (K = round(dN) per row and seed)" if w.get("sampler") else "Bernoulli per pair",
         "seed_outputs": "one per seed (per-seed masks)" if w.get("per_seed") else "one (union of the seeds)",
+        "multi_gpu": ("balanced query-row ranges of one workload per rank" if a.shard == "rows"
+                      else "one whole workload per rank"),
         "l2": (f"inputs larger than L2: each layer has its own q/k/v ({per_layer / 2**20:.0f} MiB), "
                f"{w['layers']} layers = {w['layers'] * per_layer / 2**20:.0f} MiB per run"),
     } | ({"decode": {"generated_tokens": w["gen"], "window": w["window"],
@@ -687,8 +692,15 @@ def main():
                 mask_events[-1][2].record(stream)
             pairs[name] = m.info().n_pairs
             design[name] = ris.ris_attention_design(m, tdt, D)
-            for layer in range(L):
-                ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[ri][layer])
+            if a.shard == "rows" and world > 1:
+                # every rank builds the same mask and attends its own balanced range of rows
+                b = ris.ris_mask_row_split(m, world)
+                for layer in range(L):
+                    ris.ris_attention_masked_rows(m, b[rank], b[rank + 1], qs[layer], ks[layer], vs[layer],
+                                                  outs[ri][layer], rope=rope)
+            else:
+                for layer in range(L):
+                    ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[ri][layer])
             if timing[0]:
                 mask_events[-1][3].record(stream)
             m.free()
@@ -732,7 +744,8 @@ def main():
         layers_ms[name] = layers_ms.get(name, 0.0) + e1.elapsed_time(e2) / a.steps
     total_pairs = sum(pairs.values())
     pair_heads_step = total_pairs * L * Hq
-    value = world * pair_heads_step * a.steps / (elapsed_ms / 1e3)
+    strong = a.shard == "rows" and world > 1  # the ranks share one workload
+    value = (1 if strong else world) * pair_heads_step * a.steps / (elapsed_ms / 1e3)
     ms_step = elapsed_ms / a.steps
 
     # roofline of the attention kernel over the timed region: algorithmic bytes (gather) or
@@ -824,8 +837,8 @@ def main():
             "ms_per_step": ms_step, "ms_per_layer": ms_step / (len(runs) * L), "higher_is_better": True,
             "mask_ms_per_step": mask_ms, "layers_ms_per_run": layers_ms,
             "attn_ms_per_layer": (ms_step - mask_ms) / (len(runs) * L),
-            "attn_pair_heads_per_s": world * pair_heads_step / ((ms_step - mask_ms) / 1e3),
-            "scaling": "weak", "vs_baseline": None, "dtype": w["dtype"], "data": "synthetic",
+            "attn_pair_heads_per_s": (1 if strong else world) * pair_heads_step / ((ms_step - mask_ms) / 1e3),
+            "scaling": "strong" if strong else "weak", "vs_baseline": None, "dtype": w["dtype"], "data": "synthetic",
             "config": workload_config(a), "pairs_per_mask": pairs,
             "design_per_run": {k: ris.DESIGNS.get(v, v) for k, v in design.items()}, "roofline": roofline,
             "pair_roofline": {"t_roof_ms_per_step": 1e3 * t_roof, "frac": 1e3 * t_roof / ms_step,
@@ -866,11 +879,17 @@ def main():
                     in_ready[layer].record(h2d_s)
             for ri, (name, mode, dens, ns) in enumerate(runs):
                 m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom, per_seed=per_seed)
+                b = ris.ris_mask_row_split(m, world) if strong else None
                 for layer in range(L):
                     stream.wait_event(in_ready[layer])
                     if not first[0]:
                         stream.wait_event(out_free[ri][layer])
-                    ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope, out=outs[ri][layer])
+                    if strong:
+                        ris.ris_attention_masked_rows(m, b[rank], b[rank + 1], qs[layer], ks[layer], vs[layer],
+                                                      outs[ri][layer], rope=rope)
+                    else:
+                        ris.ris_attention_masked(m, qs[layer], ks[layer], vs[layer], rope=rope,
+                                                 out=outs[ri][layer])
                     out_ready[ri][layer].record(stream)
                     if ri == len(runs) - 1:
                         layer_free[layer].record(stream)
@@ -895,7 +914,7 @@ def main():
         e1.record(stream)
         torch.cuda.synchronize()
         e_ms = max_over_ranks(e0.elapsed_time(e1), dist)
-        line["e2e"] = {"value": world * pair_heads_step * a.steps / (e_ms / 1e3), "unit": UNIT,
+        line["e2e"] = {"value": (1 if strong else world) * pair_heads_step * a.steps / (e_ms / 1e3), "unit": UNIT,
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms / a.steps}
     else:
         line["e2e"] = None
