@@ -766,7 +766,8 @@ def main():
         achieved = flops_per_launch / (mean_launch_ms / 1e3) / 1e12
         dense_flops = sum((4 * D * Hq * N * (N + 1) / 2) * (r[3] if per_seed else 1) for r in runs) * L / launches_per_step
         roofline = {"bound": "tensor", "achieved": achieved, "peak": tc, "unit": "TFLOP/s", "frac": achieved / tc,
-                    "traffic": None, "kernel": "k_attn_tile (tcgen05 masked tiles)", "peak_source": ceil["tc_source"],
+                    "traffic": recorded_traffic("attn_tile.cu") if a.workload == "C4a" else None,
+                    "kernel": "k_attn_tile (tcgen05 masked tiles)", "peak_source": ceil["tc_source"],
                     "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
                     "mean_launch_ms": mean_launch_ms, "median_launch_ms": median_launch_ms,
                     "median_launch_ms_per_run": median_per_run, "launches_timed": k_n,
