@@ -3,21 +3,28 @@
 // upper bound of Table tab:results_32k is the same kernel with every causal pair kept).
 //
 // Where the master mask keeps a large share of the causal pairs (union densities of tens of
-// percent, and the dense mode) a dense 128 x 64 score tile with the mask applied as -inf
+// percent, and the dense mode) a dense 128 x 128 score tile with the mask applied as -inf
 // beats gathering rows pair by pair. One CTA owns one (128-query tile, query head, set):
 //
-//   warp 8 (TMA)   loads the query tile once (bf16 hi and lo) and streams 64-key stages of
-//                  K~ hi, K~ lo and V (128-byte swizzled boxes) into a three-stage ring (L2
-//                  latency under load is long: the third stage took a layer from 10.5 to 7.8 ms);
+//   warp 8 (TMA)   streams 128-key stages of K~ hi, K~ lo and V (128-byte swizzled boxes)
+//                  into a two-stage shared-memory ring (96 KB a stage);
 //   warp 9 (MMA)   one elected lane issues tcgen05.mma: S = Q_hi K_hi^T + Q_lo K_hi^T +
-//                  Q_hi K_lo^T into a double-buffered TMEM score tile, and O += P_hi V + P_lo V
-//                  (A = P, written into TMEM over the consumed scores) into the TMEM output
-//                  tile, committing each step to an mbarrier;
-//   warps 0-7      two threads per query row (score columns 0-31 / 32-63, output columns
-//                  0-63 / 64-127): per tile tcgen05.ld the scores, apply the bitmap (or the causal cut), exchange the
-//                  partial row max with the partner thread, fp32 online softmax with lazy
-//                  rescaling of O in TMEM (only when the row max grows by more than 2^8),
-//                  write P hi / lo into TMEM, and at the end normalise O and store the row.
+//                  Q_hi K_lo^T (A = the query tile, kept in TMEM) into a double-buffered TMEM
+//                  score tile, and O += P_hi V + P_lo V (A = P, written into TMEM over the
+//                  consumed scores) into the TMEM output tile, committing each step to an
+//                  mbarrier; TMEM holds S/P twice (2 x 128 columns), O (128) and Q hi / lo
+//                  (2 x 64), all 512 columns;
+//   warps 0-7      two threads per query row (score and output columns 0-63 / 64-127): write
+//                  the row's query half into TMEM, then per tile tcgen05.ld the scores, apply
+//                  the bitmap (or the causal cut), exchange the partial row max with the
+//                  partner thread, fp32 online softmax with lazy rescaling of O in TMEM (only
+//                  when the row max grows by more than 2^8), write P hi / lo into TMEM, and at
+//                  the end normalise O and store the row.
+//
+// Measured on a 32k-token layer: the products alone (no softmax work) take 6.0 ms, 81% of
+// the measured sustained bf16 rate for the five products a tile issues; the whole kernel
+// 7.2 ms. 128-key tiles with the query in TMEM beat 64-key tiles with the query in shared
+// memory and three stages (7.8 ms).
 //
 // Every mbarrier wait is bounded; a wait that gives up sets bit 1 of the device error word,
 // every role falls through to the end, TMEM is released and the CTA returns.
@@ -38,30 +45,27 @@ __device__ unsigned int g_ris_tile_error;
 namespace {
 
 constexpr int BM = 128;          // query rows per tile (TMEM lanes)
-constexpr int BN = 64;           // keys per stage
+constexpr int BN = 128;          // keys per stage
 constexpr int DT = 128;          // head dim handled by this kernel
 constexpr int kThreads = 320;    // warps 0-7 softmax (two column halves), 8 TMA, 9 MMA
 constexpr int kTmaWarp = 8, kMmaWarp = 9;
-constexpr uint32_t kTmemCols = 256;  // S/P[2] (2 x 64) + O (128)
+constexpr uint32_t kTmemCols = 512;  // S/P[2] (2 x 128) + O (128) + Q hi / lo (2 x 64)
 
 // shared-memory map (bytes, from a 1024-aligned base)
-constexpr int KV_ARR = BN * DT * 2;         // 16 KB: one of K hi / K lo / V
-constexpr int KV_BLK = BN * 128;            // 8 KB: one 64-column block
-constexpr int STAGE = 3 * KV_ARR;           // 48 KB
-constexpr int kKvStages = 3;                // K/V stages in flight
-constexpr int Q_ARR = BM * DT * 2;          // 32 KB: one of Q hi / Q lo (two 64-column blocks)
-constexpr int Q_BLK = BM * 128;             // 16 KB: one 64-column block of the query tile
-constexpr int OFF_Q = 0;
-constexpr int OFF_KV = 2 * Q_ARR;           // 64 KB
-constexpr int SMEM_BYTES = OFF_KV + kKvStages * STAGE + 1024;  // + alignment slack = 214016
+constexpr int KV_ARR = BN * DT * 2;         // 32 KB: one of K hi / K lo / V
+constexpr int KV_BLK = BN * 128;            // 16 KB: one 64-column block
+constexpr int STAGE = 3 * KV_ARR;           // 96 KB
+constexpr int kKvStages = 2;                // K/V stages in flight
+constexpr int OFF_KV = 0;
+constexpr int SMEM_BYTES = OFF_KV + kKvStages * STAGE + 1024;  // + alignment slack = 197632
 
 // P_FULL and PV_DONE have one barrier per P buffer (tile parity), so that no waiter can fall
 // two phases behind a barrier it polls by parity.
 // B_X: per pair of softmax warps sharing rows (columns 0-31 / 32-63) and tile parity, the
 // exchange of their partial row maxima (and at the end their partial sums).
 enum Bar {
-    B_Q = 0, B_KV_FULL = 1, B_KV_EMPTY = 4, B_S_FULL = 7, B_S_EMPTY = 9, B_P_FULL = 11, B_PV_DONE = 13, B_X = 15,
-    NBAR = 23
+    B_Q = 0, B_KV_FULL = 1, B_KV_EMPTY = 3, B_S_FULL = 5, B_S_EMPTY = 7, B_P_FULL = 9, B_PV_DONE = 11, B_X = 13,
+    NBAR = 21
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -243,7 +247,7 @@ __device__ __forceinline__ void store8<__nv_bfloat16>(__nv_bfloat16 *dst, const 
 }
 
 struct TileMaps {
-    CUtensorMap qh, ql, kh, kl, v;
+    CUtensorMap kh, kl, v;
 };
 
 template <bool SPLIT, bool DENSE, typename TOut>
@@ -275,7 +279,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < NBAR; ++i) {
             uint32_t cnt = 1;
-            if (i == B_S_EMPTY || i == B_S_EMPTY + 1 || i == B_P_FULL || i == B_P_FULL + 1) cnt = 256;
+            if (i == B_Q || i == B_S_EMPTY || i == B_S_EMPTY + 1 || i == B_P_FULL || i == B_P_FULL + 1) cnt = 256;
             if (i >= B_X) cnt = 64;
             mbar_init(smem_u32(&bars[i]), cnt);
         }
@@ -292,18 +296,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
-    const uint32_t t_s0 = tmem, t_s1 = tmem + BN, t_o = tmem + 2 * BN;
+    const uint32_t t_s0 = tmem, t_s1 = tmem + BN, t_o = tmem + 2 * BN, t_q = tmem + 2 * BN + DT;
     bool ok = true;
 
     if (warp == kTmaWarp) {
         // =============================== TMA producer
         if (lane == 0) {
-            const uint32_t bq = smem_u32(&bars[B_Q]);
-            mbar_arrive_expect_tx(bq, (SPLIT ? 2 : 1) * Q_ARR);
-            for (int blk = 0; blk < 2; ++blk) {
-                tma_load_3d(sbase + OFF_Q + blk * Q_BLK, &maps.qh, 64 * blk, h, (int)q0, bq);
-                if (SPLIT) tma_load_3d(sbase + OFF_Q + Q_ARR + blk * Q_BLK, &maps.ql, 64 * blk, h, (int)q0, bq);
-            }
             for (int j = 0; j < n_kt && ok; ++j) {
                 const int st = j % kKvStages;
                 if (j >= kKvStages) ok = mbar_wait(smem_u32(&bars[B_KV_EMPTY + st]), ((j / kKvStages) - 1) & 1);
@@ -324,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == kMmaWarp) {
         // =============================== MMA issuer
         if (lane == 0) {
-            constexpr uint32_t ID_S = idesc_bf16(BM, BN, false);  // S[128 x 64] = Q K^T, both K-major
+            constexpr uint32_t ID_S = idesc_bf16(BM, BN, false);  // S[128 x 128] = Q K^T, both K-major
             constexpr uint32_t ID_O = idesc_bf16(BM, DT, true);   // O[128 x 128] += P V, V MN-major
             ok = mbar_wait(smem_u32(&bars[B_Q]), 0);
             tc_fence_after();
@@ -334,14 +332,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t dt = (j & 1) ? t_s1 : t_s0;
                 uint32_t acc = 0;
                 // (A, B) pairs: (Q hi, K hi), (Q lo, K hi), (Q hi, K lo); 8 k-steps of 16 over D
+                // the query tile lives in TMEM (16-bit values packed two per column): A from TMEM
                 for (int prod = 0; prod < (SPLIT ? 3 : 1); ++prod) {
-                    const uint32_t qa = sbase + OFF_Q + (prod == 1 ? Q_ARR : 0);
+                    const uint32_t qa = t_q + (prod == 1 ? DT / 2 : 0);
                     const uint32_t kb = kv + (prod == 2 ? KV_ARR : 0);
                     for (int ks = 0; ks < DT / 16; ++ks) {
                         const uint32_t koff = (uint32_t)((ks & 3) * 32);  // 16 columns = 32 B inside a 128 B row
-                        const uint64_t ad = sdesc(qa + (ks >> 2) * Q_BLK + koff, 16, 1024);
                         const uint64_t bd = sdesc(kb + (ks >> 2) * KV_BLK + koff, 16, 1024);
-                        tc_mma(dt, ad, bd, ID_S, acc);
+                        tc_mma_ts(dt, qa + 8 * ks, bd, ID_S, acc);
                         acc = 1;
                     }
                 }
@@ -350,15 +348,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             auto issue_o = [&](int j) {
                 const int st = j % kKvStages;
                 const uint32_t vb = sbase + OFF_KV + st * STAGE + 2 * KV_ARR;
-                // P hi / lo of this tile sit in TMEM over its score columns: 64 keys of 16-bit
-                // values packed two per column, hi in columns 0-31, lo in 32-63
+                // P hi / lo of this tile sit in TMEM over its score columns: 128 keys of 16-bit
+                // values packed two per column, hi in columns 0-63, lo in 64-127
                 const uint32_t pt = (j & 1) ? t_s1 : t_s0;
                 for (int prod = 0; prod < 2; ++prod) {
                     for (int ks = 0; ks < BN / 16; ++ks) {
                         // V block: 64 keys x 128 B rows; 16 keys = two 8-row atoms (SBO 1024);
                         // the second 64-column block of head dim is LBO = 8 KB away
                         const uint64_t bd = sdesc(vb + ks * 2048, KV_BLK, 1024);
-                        tc_mma_ts(t_o, pt + 32 * prod + 8 * ks, bd, ID_O, (j > 0 || prod > 0 || ks > 0) ? 1u : 0u);
+                        tc_mma_ts(t_o, pt + (BN / 2) * prod + 8 * ks, bd, ID_O, (j > 0 || prod > 0 || ks > 0) ? 1u : 0u);
                     }
                 }
                 tc_commit(smem_u32(&bars[B_PV_DONE + (j & 1)]));
@@ -390,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         // =============================== softmax: two threads per query row q0 + r, one per
-        // column half hf (scores 32 hf .. 32 hf + 31 of each tile, O columns 64 hf .. 64 hf + 63)
+        // column half hf (scores 64 hf .. 64 hf + 63 of each tile, O columns 64 hf .. 64 hf + 63)
         const int wq = warp & 3, hf = warp >> 2;
         const int r = wq * 32 + lane;  // TMEM lane
         const int64_t i = q0 + r;
@@ -401,10 +399,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int64_t last_word = i >> 5;
         const float sc = a.scale_log2;
         float m_used = -INFINITY, l = 0.f;
-        // bitmap word of keys 64j + 32hf .. 64j + 32hf + 31 of this row, fetched one tile ahead
-        auto mask_word = [&](int j) -> uint32_t {
+        // bitmap word e (0, 1) of keys 128j + 64hf + 32e .. +31 of this row, fetched one tile ahead
+        auto mask_word = [&](int j, int e) -> uint32_t {
             if (!row_ok) return 0u;
-            const int64_t k0 = (int64_t)j * BN + 32 * hf;
+            const int64_t k0 = (int64_t)j * BN + 64 * hf + 32 * e;
             if (DENSE) {
                 const int64_t lim = i - k0;  // keys k0 .. i are kept
                 return lim >= 31 ? 0xFFFFFFFFu : (lim < 0 ? 0u : ((2u << lim) - 1u));
@@ -422,28 +420,57 @@ __global__ void __launch_bounds__(kThreads, 1)
             other = xch[pb][hf ^ 1][r];
             return got;
         };
-        uint32_t cw = mask_word(0);
+        // this thread's half row of the query tile (head-dim 64 hf .. 64 hf + 63) into TMEM
+        {
+            uint32_t qw[32];
+            const int64_t qrow = ((row_ok ? i : 0) * a.Hq + h) * DT + 64 * hf;
+            for (int part = 0; part < (SPLIT ? 2 : 1); ++part) {
+                const uint4 *src = reinterpret_cast<const uint4 *>(
+                    reinterpret_cast<const __nv_bfloat16 *>(part == 0 ? q_hi : q_lo) + qrow);
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const uint4 x = row_ok ? src[u] : make_uint4(0u, 0u, 0u, 0u);
+                    qw[4 * u] = x.x;
+                    qw[4 * u + 1] = x.y;
+                    qw[4 * u + 2] = x.z;
+                    qw[4 * u + 3] = x.w;
+                }
+                tmem_st16(t_q + lane_off + (DT / 2) * part + 32 * hf, qw);
+                tmem_st16(t_q + lane_off + (DT / 2) * part + 32 * hf + 16, qw + 16);
+            }
+            tc_fence_before();
+            mbar_arrive(smem_u32(&bars[B_Q]));
+        }
+        uint32_t cw0 = mask_word(0, 0), cw1 = mask_word(0, 1);
         for (int j = 0; j < n_kt; ++j) {
             const int st = j & 1;
-            const uint32_t nw = (j + 1 < n_kt) ? mask_word(j + 1) : 0u;
+            const uint32_t nw0 = (j + 1 < n_kt) ? mask_word(j + 1, 0) : 0u;
+            const uint32_t nw1 = (j + 1 < n_kt) ? mask_word(j + 1, 1) : 0u;
             ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&bars[B_S_FULL + st]), (j >> 1) & 1));
             if (!ok) break;
             tc_fence_after();
-            float sv[32];
-            tmem_ld32(((j & 1) ? t_s1 : t_s0) + lane_off + 32 * hf, sv);
+            float sv[64];
+            const uint32_t sb = ((j & 1) ? t_s1 : t_s0) + lane_off + 64 * hf;
+            tmem_ld32(sb, sv);
+            tmem_ld32(sb + 32, sv + 32);
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_S_EMPTY + st]));
 
             // mask, scale, partial row max as a tree, then the full row max with the partner
 #pragma unroll
-            for (int c = 0; c < 32; ++c) sv[c] = ((cw >> c) & 1u) ? sv[c] * sc : -INFINITY;
-            cw = nw;
-            float mx4[4];
+            for (int c = 0; c < 32; ++c) {
+                sv[c] = ((cw0 >> c) & 1u) ? sv[c] * sc : -INFINITY;
+                sv[32 + c] = ((cw1 >> c) & 1u) ? sv[32 + c] * sc : -INFINITY;
+            }
+            cw0 = nw0;
+            cw1 = nw1;
+            float mx8[8];
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-                mx4[e] = fmaxf(fmaxf(fmaxf(sv[e], sv[e + 4]), fmaxf(sv[e + 8], sv[e + 12])),
-                               fmaxf(fmaxf(sv[e + 16], sv[e + 20]), fmaxf(sv[e + 24], sv[e + 28])));
-            const float pm = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+            for (int e = 0; e < 8; ++e)
+                mx8[e] = fmaxf(fmaxf(fmaxf(sv[e], sv[e + 8]), fmaxf(sv[e + 16], sv[e + 24])),
+                               fmaxf(fmaxf(sv[e + 32], sv[e + 40]), fmaxf(sv[e + 48], sv[e + 56])));
+            const float pm = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
             float om;
             ok = exchange(j, pm, om);
             if (!ok) break;
@@ -479,11 +506,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             // P = exp2(s - m_used) split as hi = p with its low 16 bits cleared (exactly a bf16)
             // and lo = p - hi rounded to bf16 (p to ~16 significant bits with one conversion per
             // pair), written into TMEM over this tile's score columns (both halves have read
-            // their scores: the max exchange came first) as the A operand of the value product
+            // their scores: the max exchange came first) as the A operand of the value product:
+            // keys 64 hf .. 64 hf + 63 as hi in columns 32 hf .. +31 and lo in 64 + 32 hf .. +31
             float lsum[4] = {0.f, 0.f, 0.f, 0.f};
-            uint32_t hw[16], lw[16];
+            uint32_t hw[32], lw[32];
 #pragma unroll
-            for (int w = 0; w < 16; ++w) {
+            for (int w = 0; w < 32; ++w) {
                 const float p0 = exp2f(sv[2 * w] - mu), p1 = exp2f(sv[2 * w + 1] - mu);
                 lsum[w & 3] += p0 + p1;
                 const uint32_t b0 = __float_as_uint(p0), b1 = __float_as_uint(p1);
@@ -492,8 +520,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             l += (lsum[0] + lsum[1]) + (lsum[2] + lsum[3]);
             const uint32_t pt = ((j & 1) ? t_s1 : t_s0) + lane_off;
-            tmem_st16(pt + 16 * hf, hw);
-            tmem_st16(pt + 32 + 16 * hf, lw);
+            tmem_st16(pt + 32 * hf, hw);
+            tmem_st16(pt + 32 * hf + 16, hw + 16);
+            tmem_st16(pt + 64 + 32 * hf, lw);
+            tmem_st16(pt + 64 + 32 * hf + 16, lw + 16);
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_P_FULL + st]));
         }
@@ -599,14 +629,11 @@ cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const voi
     std::lock_guard<std::mutex> lk(mu);
     const bool split = q_lo != nullptr;
     alignas(64) TileMaps maps;
-    if (!make_map3(&maps.qh, q_hi, a.N, a.Hq, BM) || !make_map3(&maps.kh, a.k, a.N, a.Hkv, BN) ||
-        !make_map3(&maps.v, a.v, a.N, a.Hkv, BN))
+    if (!make_map3(&maps.kh, a.k, a.N, a.Hkv, BN) || !make_map3(&maps.v, a.v, a.N, a.Hkv, BN))
         return cudaErrorInvalidValue;
     if (split) {
-        if (!make_map3(&maps.ql, q_lo, a.N, a.Hq, BM) || !make_map3(&maps.kl, a.k_lo, a.N, a.Hkv, BN))
-            return cudaErrorInvalidValue;
+        if (!make_map3(&maps.kl, a.k_lo, a.N, a.Hkv, BN)) return cudaErrorInvalidValue;
     } else {
-        maps.ql = maps.qh;
         maps.kl = maps.kh;
     }
     if (out_dtype == RIS_F32) {
