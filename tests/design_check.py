@@ -20,6 +20,8 @@ CASES = [
     (257, 4, 1, 128, 2, 1.0, [0], None, False),
     (640, 8, 2, 64, 1, 0.1, [3], (2, 1e4, 128), False),
     (400, 6, 2, 128, 0, 0.3, [4, 5, 6], (3, 1e6, 256), True),
+    (3, 6, 2, 128, 0, 0.5, [1], (3, 1e6, 64), False),
+    (1, 2, 1, 64, 1, 0.5, [2], None, False),
 ]
 
 

@@ -70,6 +70,12 @@ SMALL = [
     (300, 12, 2, 128, torch.bfloat16, 2, 1.0, 1, 1, 4096),
     (300, 2, 1, 64, torch.float32, 0, 1.0, 1, 0, 4096),
     (1025, 5, 1, 128, torch.bfloat16, 0, 0.02, 10, 1, 4096),
+    # tiny and ragged sizes on the tile design (their masks keep most causal pairs)
+    (1, 6, 2, 128, torch.bfloat16, 0, 0.05, 1, 3, 64),
+    (2, 6, 2, 128, torch.bfloat16, 1, 0.5, 2, 1, 4096),
+    (129, 12, 2, 128, torch.bfloat16, 0, 0.3, 3, 3, 64),
+    (257, 6, 2, 128, torch.bfloat16, 2, 1.0, 1, 3, 64),
+    (130, 6, 2, 128, torch.bfloat16, 0, 0.01, 1, 1, 4096),
 ]
 
 

@@ -7,6 +7,8 @@ import sys
 
 import pytest
 
+from design_check import CASES
+
 pytestmark = pytest.mark.gpu
 
 HERE = os.path.dirname(os.path.abspath(__file__))
@@ -18,4 +20,5 @@ def test_design_matches_oracle(design):
     r = subprocess.run([sys.executable, os.path.join(HERE, "design_check.py")], env=env, capture_output=True,
                        text=True, timeout=600)
     assert r.returncode == 0, r.stdout + r.stderr
-    assert r.stdout.count("max-abs") == 7
+    expected = sum(len(c[6]) if c[8] else 1 for c in CASES)
+    assert r.stdout.count("max-abs") == expected, r.stdout
