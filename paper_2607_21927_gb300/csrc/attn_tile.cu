@@ -6,8 +6,11 @@
 // percent, and the dense mode) a dense 128 x 128 score tile with the mask applied as -inf
 // beats gathering rows pair by pair. One CTA owns one (128-query tile, query head, set):
 //
-//   warp 8 (TMA)   streams 128-key stages of K~ hi, K~ lo and V (128-byte swizzled boxes)
-//                  into a two-stage shared-memory ring (96 KB a stage);
+//   warp 8 (TMA)   streams 128-key tiles of K~ hi + K~ lo (64 KB) and of V (32 KB) in
+//                  128-byte swizzled boxes into two two-stage shared-memory rings: a key stage
+//                  is refilled as soon as its score products are done, a value stage once its
+//                  value product is, so the next keys load while P and the value product of
+//                  the current tile are still pending;
 //   warp 9 (MMA)   one elected lane issues tcgen05.mma: S = Q_hi K_hi^T + Q_lo K_hi^T +
 //                  Q_hi K_lo^T (A = the query tile, kept in TMEM) into a double-buffered TMEM
 //                  score tile, and O += P_hi V + P_lo V (A = P, written into TMEM over the
@@ -21,10 +24,15 @@
 //                  when the row max grows by more than 2^8), write P hi / lo into TMEM, and at
 //                  the end normalise O and store the row.
 //
-// Measured on a 32k-token layer: the products alone (no softmax work) take 6.0 ms, 81% of
-// the measured sustained bf16 rate for the five products a tile issues; the whole kernel
-// 7.2 ms. 128-key tiles with the query in TMEM beat 64-key tiles with the query in shared
-// memory and three stages (7.8 ms).
+// Precision: the five products keep about 16 significant bits of every operand. Single
+// fp16 keys move outputs by up to 0.1 on inputs with outlier channels, and P rounded to fp16
+// (one value product instead of two: 13% faster) by up to 1.1e-2 at 2k tokens, above the
+// 1e-2 bar, so neither is taken.
+//
+// Measured on a 32k-token layer: 5.7 ms. With one ring of combined K/V stages, released only
+// after the value product, the next tile's keys started loading only then and the tensor
+// pipe waited for them: 7.2 ms (the products alone 6.0 ms). 128-key tiles with the query in
+// TMEM beat 64-key tiles with the query in shared memory and three stages (7.8 ms).
 //
 // Every mbarrier wait is bounded; a wait that gives up sets bit 1 of the device error word,
 // every role falls through to the end, TMEM is released and the CTA returns.
@@ -54,18 +62,20 @@ constexpr uint32_t kTmemCols = 512;  // S/P[2] (2 x 128) + O (128) + Q hi / lo (
 // shared-memory map (bytes, from a 1024-aligned base)
 constexpr int KV_ARR = BN * DT * 2;         // 32 KB: one of K hi / K lo / V
 constexpr int KV_BLK = BN * 128;            // 16 KB: one 64-column block
-constexpr int STAGE = 3 * KV_ARR;           // 96 KB
-constexpr int kKvStages = 2;                // K/V stages in flight
-constexpr int OFF_KV = 0;
-constexpr int SMEM_BYTES = OFF_KV + kKvStages * STAGE + 1024;  // + alignment slack = 197632
+constexpr int K_STAGE = 2 * KV_ARR;         // 64 KB: K hi, K lo
+constexpr int V_STAGE = KV_ARR;             // 32 KB
+constexpr int kStages = 2;                  // stages of each ring
+constexpr int OFF_K = 0;
+constexpr int OFF_V = OFF_K + kStages * K_STAGE;
+constexpr int SMEM_BYTES = OFF_V + kStages * V_STAGE + 1024;  // + alignment slack = 197632
 
 // P_FULL and PV_DONE have one barrier per P buffer (tile parity), so that no waiter can fall
 // two phases behind a barrier it polls by parity.
 // B_X: per pair of softmax warps sharing rows (columns 0-31 / 32-63) and tile parity, the
 // exchange of their partial row maxima (and at the end their partial sums).
 enum Bar {
-    B_Q = 0, B_KV_FULL = 1, B_KV_EMPTY = 3, B_S_FULL = 5, B_S_EMPTY = 7, B_P_FULL = 9, B_PV_DONE = 11, B_X = 13,
-    NBAR = 21
+    B_Q = 0, B_K_FULL = 1, B_K_EMPTY = 3, B_V_FULL = 5, B_V_EMPTY = 7, B_S_FULL = 9, B_S_EMPTY = 11, B_P_FULL = 13,
+    B_PV_DONE = 15, B_X = 17, B_END = 25, NBAR = 26
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -94,6 +104,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
         : "memory");
     return ok != 0;
 }
+// Bounded wait for this CTA's own asynchronous work (copies or products already issued):
+// about 2^31 cycles at most, whatever other CTAs reported.
+__device__ __forceinline__ bool mbar_wait_own(uint32_t bar, uint32_t parity)
+{
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, parity))
+        if (clock64() - t0 > (1LL << 31)) return false;
+    return true;
+}
+
 // Bounded wait (about 2^31 cycles); false if the phase did not complete in time.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
 {
@@ -280,7 +300,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < NBAR; ++i) {
             uint32_t cnt = 1;
             if (i == B_Q || i == B_S_EMPTY || i == B_S_EMPTY + 1 || i == B_P_FULL || i == B_P_FULL + 1) cnt = 256;
-            if (i >= B_X) cnt = 64;
+            if (i >= B_X && i < B_END) cnt = 64;
             mbar_init(smem_u32(&bars[i]), cnt);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -302,22 +322,37 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kTmaWarp) {
         // =============================== TMA producer
         if (lane == 0) {
+            // tile j: keys once the score products of tile j - 2 are done, then values once the
+            // value product of tile j - 2 is (it was issued after the score products of tile
+            // j - 1, whose keys are already in flight: no wait here depends on a later load)
+            int nk = 0, nv = 0;  // tiles whose keys / values were requested
             for (int j = 0; j < n_kt && ok; ++j) {
-                const int st = j % kKvStages;
-                if (j >= kKvStages) ok = mbar_wait(smem_u32(&bars[B_KV_EMPTY + st]), ((j / kKvStages) - 1) & 1);
+                const int st = j % kStages;
+                const uint32_t par = ((j / kStages) - 1) & 1;
+                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_K_EMPTY + st]), par);
                 if (!ok) break;
-                const uint32_t bf = smem_u32(&bars[B_KV_FULL + st]);
-                const uint32_t dst = sbase + OFF_KV + st * STAGE;
-                mbar_arrive_expect_tx(bf, (SPLIT ? 3 : 2) * KV_ARR);
+                const uint32_t bk = smem_u32(&bars[B_K_FULL + st]);
+                const uint32_t dk = sbase + OFF_K + st * K_STAGE;
+                mbar_arrive_expect_tx(bk, (SPLIT ? 2 : 1) * KV_ARR);
                 for (int blk = 0; blk < 2; ++blk) {
-                    tma_load_3d(dst + 0 * KV_ARR + blk * KV_BLK, &maps.kh, 64 * blk, g, j * BN, bf);
-                    if (SPLIT) tma_load_3d(dst + 1 * KV_ARR + blk * KV_BLK, &maps.kl, 64 * blk, g, j * BN, bf);
-                    tma_load_3d(dst + 2 * KV_ARR + blk * KV_BLK, &maps.v, 64 * blk, g, j * BN, bf);
+                    tma_load_3d(dk + blk * KV_BLK, &maps.kh, 64 * blk, g, j * BN, bk);
+                    if (SPLIT) tma_load_3d(dk + KV_ARR + blk * KV_BLK, &maps.kl, 64 * blk, g, j * BN, bk);
                 }
+                nk = j + 1;
+                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_V_EMPTY + st]), par);
+                if (!ok) break;
+                const uint32_t bv = smem_u32(&bars[B_V_FULL + st]);
+                const uint32_t dv = sbase + OFF_V + st * V_STAGE;
+                mbar_arrive_expect_tx(bv, KV_ARR);
+                for (int blk = 0; blk < 2; ++blk) tma_load_3d(dv + blk * KV_BLK, &maps.v, 64 * blk, g, j * BN, bv);
+                nv = j + 1;
             }
-            // let the last stages land before the CTA can leave
-            for (int j = n_kt - kKvStages; j < n_kt; ++j)
-                if (j >= 0) mbar_wait(smem_u32(&bars[B_KV_FULL + j % kKvStages]), (j / kKvStages) & 1);
+            // let the copies requested last into each stage land before the CTA can leave
+            // (earlier ones were consumed before their stage was refilled)
+            for (int j = nk - kStages; j < nk; ++j)
+                if (j >= 0) mbar_wait_own(smem_u32(&bars[B_K_FULL + j % kStages]), (j / kStages) & 1);
+            for (int j = nv - kStages; j < nv; ++j)
+                if (j >= 0) mbar_wait_own(smem_u32(&bars[B_V_FULL + j % kStages]), (j / kStages) & 1);
         }
     } else if (warp == kMmaWarp) {
         // =============================== MMA issuer
@@ -328,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             auto issue_s = [&](int j) {
                 const int st = j & 1;
-                const uint32_t kv = sbase + OFF_KV + (j % kKvStages) * STAGE;
+                const uint32_t kv = sbase + OFF_K + (j % kStages) * K_STAGE;
                 const uint32_t dt = (j & 1) ? t_s1 : t_s0;
                 uint32_t acc = 0;
                 // (A, B) pairs: (Q hi, K hi), (Q lo, K hi), (Q hi, K lo); 8 k-steps of 16 over D
@@ -344,10 +379,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 tc_commit(smem_u32(&bars[B_S_FULL + st]));
+                if (j + kStages < n_kt) tc_commit(smem_u32(&bars[B_K_EMPTY + j % kStages]));  // keys free
             };
             auto issue_o = [&](int j) {
-                const int st = j % kKvStages;
-                const uint32_t vb = sbase + OFF_KV + st * STAGE + 2 * KV_ARR;
+                const int st = j % kStages;
+                const uint32_t vb = sbase + OFF_V + st * V_STAGE;
                 // P hi / lo of this tile sit in TMEM over its score columns: 128 keys of 16-bit
                 // values packed two per column, hi in columns 0-63, lo in 64-127
                 const uint32_t pt = (j & 1) ? t_s1 : t_s0;
@@ -359,18 +395,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tc_mma_ts(t_o, pt + (BN / 2) * prod + 8 * ks, bd, ID_O, (j > 0 || prod > 0 || ks > 0) ? 1u : 0u);
                     }
                 }
+                if (j + kStages < n_kt) tc_commit(smem_u32(&bars[B_V_EMPTY + st]));  // values free
                 tc_commit(smem_u32(&bars[B_PV_DONE + (j & 1)]));
-                tc_commit(smem_u32(&bars[B_KV_EMPTY + st]));
             };
             for (int j = 0; j < n_kt && ok; ++j) {
                 const int st = j & 1;
-                ok = mbar_wait(smem_u32(&bars[B_KV_FULL + j % kKvStages]), (j / kKvStages) & 1);
+                ok = mbar_wait(smem_u32(&bars[B_K_FULL + j % kStages]), (j / kStages) & 1);
                 if (ok && j >= 2) ok = mbar_wait(smem_u32(&bars[B_S_EMPTY + st]), ((j >> 1) - 1) & 1);
                 if (!ok) break;
                 tc_fence_after();
                 issue_s(j);
                 if (j >= 1) {
                     ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((j - 1) & 1)]), ((j - 1) >> 1) & 1);
+                    if (ok) ok = mbar_wait(smem_u32(&bars[B_V_FULL + (j - 1) % kStages]), ((j - 1) / kStages) & 1);
                     if (!ok) break;
                     tc_fence_after();
                     issue_o(j - 1);
@@ -378,13 +415,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (ok) {
                 ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1);
+                if (ok) ok = mbar_wait(smem_u32(&bars[B_V_FULL + (n_kt - 1) % kStages]), ((n_kt - 1) / kStages) & 1);
                 if (ok) {
                     tc_fence_after();
                     issue_o(n_kt - 1);
                 }
             }
-            // the last commit has to land before TMEM is released
-            mbar_wait(smem_u32(&bars[B_PV_DONE + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1);
+            // every product issued has to finish before TMEM is released
+            tc_commit(smem_u32(&bars[B_END]));
+            mbar_wait_own(smem_u32(&bars[B_END]), 0);
         }
     } else {
         // =============================== softmax: two threads per query row q0 + r, one per
@@ -610,6 +649,7 @@ cudaError_t launch_t(const AttnArgs &a, const TileMaps &maps, const void *q_hi, 
 }  // namespace
 
 bool tile_design_available() { return encode_fn() != nullptr; }
+
 
 // Read and clear this kernel's device error word (the caller has synchronised).
 cudaError_t read_tile_error(unsigned int *out)
