@@ -371,14 +371,15 @@ def run_reference(a, rank):
 
 
 # ----------------------------------------------------------------------------- traffic record
-def recorded_traffic(kernel_file: str):
-    """DRAM bytes per launch from the committed ncu summary, if taken on the current kernel source."""
+def recorded_traffic(kernel_file: str, workload: str):
+    """DRAM bytes per launch of `kernel_file`'s kernel at `workload`, from the committed ncu
+    record, if it was taken on the current kernel source."""
     rec = os.path.join(ROOT, "profiles", "traffic.json")
     src = os.path.join(ROOT, "paper_2607_21927_gb300", "csrc", kernel_file)
     try:
         data = json.load(open(rec))
         h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        ent = data.get(kernel_file)
+        ent = data.get(kernel_file, {}).get(workload)
         if ent and ent.get("source_sha256_16") == h:
             return ent.get("dram_bytes_per_launch_full_size")
     except Exception:
@@ -761,70 +762,63 @@ def main():
     kinds = sorted(set(design.values()))
     hbm, tc = ceil["hbm_gbs"], ceil["tc_tflops"]
     kv_row_bytes = Hkv * 2 * D * e  # K and V rows of one key, all KV heads
-    if kinds == [2]:  # every launch on the tensor-core tile kernel
-        flops_per_launch = 4 * D * Hq * total_pairs * L / launches_per_step
-        achieved = flops_per_launch / (mean_launch_ms / 1e3) / 1e12
-        dense_flops = sum((4 * D * Hq * N * (N + 1) / 2) * (r[3] if per_seed else 1) for r in runs) * L / launches_per_step
-        roofline = {"bound": "tensor", "achieved": achieved, "peak": tc, "unit": "TFLOP/s", "frac": achieved / tc,
-                    "traffic": recorded_traffic("attn_tile.cu") if a.workload == "C4a" else None,
-                    "kernel": "k_attn_tile (tcgen05 masked tiles)", "peak_source": ceil["tc_source"],
-                    "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
-                    "mean_launch_ms": mean_launch_ms, "median_launch_ms": median_launch_ms,
-                    "median_launch_ms_per_run": median_per_run, "launches_timed": k_n,
-                    "design_frac": (dense_flops / (tc * 1e12)) / (mean_launch_ms / 1e3),
-                    "design_note": "dense-causal tile FLOPs / sustained bf16 peak over the launch time (the "
-                                   "kernel issues 2.5x that in hi/lo split products)"}
+    kv_set = N * Hkv * D * e * (3 if e == 2 else 2)  # rotated K (hi + lo for bf16) and V of a layer
+    gather_names = {0: "k_attn_bf16 (register gather)", 1: "k_attn_tma (TMA gather4)", 2: "k_attn_tile (tcgen05 masked tiles)",
+                    3: "k_attn_f32 (fp32 gather)"}
+    traffic_file = {0: "attn_bf16.cu", 2: "attn_tile.cu"}
+
+    def design_roofline(kd, names):
+        """Roofline of design kd's kernel over the launches of runs `names`: algorithmic work per
+        launch / that kernel's mean CUDA-event launch time in the timed region."""
+        each = [t for nm in names for t in per_run_ms.get(nm, [])]
+        if each:
+            mean_ms, med_ms, n_l = sum(each) / len(each), statistics.median(each), len(each)
+        else:  # launch times not attributable to runs: all launches
+            mean_ms, med_ms, n_l = mean_launch_ms, median_launch_ms, k_n
+        pairs_launch = sum(pairs[nm] for nm in names) / len(names)
+        traffic = recorded_traffic(traffic_file[kd], a.workload) if kd in traffic_file else None
+        ent = {"kernel": gather_names.get(kd, "?"), "mean_launch_ms": mean_ms, "median_launch_ms": med_ms,
+               "launches_timed": n_l, "traffic": traffic}
+        if kd == 2:
+            achieved = 4 * D * Hq * pairs_launch / (mean_ms / 1e3) / 1e12
+            dense = 4 * D * Hq * N * (N + 1) / 2 * (max(r[3] for r in runs if r[0] in names) if per_seed else 1)
+            ent.update({"bound": "tensor", "achieved": achieved, "peak": tc, "unit": "TFLOP/s", "frac": achieved / tc,
+                        "peak_source": ceil["tc_source"],
+                        "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
+                        "design_frac": (dense / (tc * 1e12)) / (mean_ms / 1e3),
+                        "design_note": "dense-causal tile FLOPs / sustained bf16 peak over the launch time (the "
+                                       "kernel issues 2.5x that in hi/lo split products)"})
+        else:
+            achieved = pairs_launch * kv_row_bytes / (mean_ms / 1e3) / 1e9
+            ent.update({"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                        "peak_source": ceil["hbm_source"],
+                        "bytes": "algorithmic: K and V rows of every sampled pair, all KV heads"})
+            if "l2_rows_gbs" in ceil and kv_set < ceil["l2_bytes"]:
+                # the K/V working set is L2-resident: the gathered rows are served from L2, so L2 is
+                # the bound (HBM carries only the compulsory q/k/v/out traffic, `traffic`)
+                ent.update({"bound": "l2", "peak": ceil["l2_rows_gbs"], "frac": achieved / ceil["l2_rows_gbs"],
+                            "peak_source": "measured in this run by the library's L2 probe: whole 256-byte rows "
+                                           f"at random indices over {ceil['l2_rows_set_bytes'] / 2**20:.0f} MiB "
+                                           "(L2 is not in MEASURED_PEAKS.json)",
+                            "hbm_peak": hbm, "frac_of_hbm": achieved / hbm,
+                            "bytes_read_per_algorithmic_byte": 1.5 if e == 2 else 1.0})
+        ent["device_ms_per_step"] = sum(each) / a.steps if each else None
+        return ent
+
+    by_design = {}
+    for name, kd in design.items():
+        by_design.setdefault(kd, []).append(name)
+    per_design = {kd: design_roofline(kd, names) for kd, names in by_design.items()}
+    if len(kinds) == 1:
+        roofline = per_design[kinds[0]]
+        roofline["median_launch_ms_per_run"] = median_per_run
     else:
-        bytes_per_launch = total_pairs * L * kv_row_bytes / launches_per_step
-        achieved = bytes_per_launch / (mean_launch_ms / 1e3) / 1e9
-        gather = {0: "k_attn_bf16 (register gather)", 1: "k_attn_tma (TMA gather4)", 3: "k_attn_f32 (fp32 gather)"}
-        roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                    "traffic": recorded_traffic("attn_bf16.cu") if kinds == [0] and a.workload == "C5" else None,
-                    "kernel": gather.get(kinds[0], "?") if len(kinds) == 1 else "mixed designs " + str(kinds),
-                    "peak_source": ceil["hbm_source"],
-                    "bytes": "algorithmic: K and V rows of every sampled pair, all KV heads",
-                    "mean_launch_ms": mean_launch_ms, "median_launch_ms": median_launch_ms,
-                    "median_launch_ms_per_run": median_per_run, "launches_timed": k_n}
-        kv_set = N * Hkv * D * e * (3 if e == 2 else 2)  # rotated K (hi + lo for bf16) and V of a layer
-        if "l2_rows_gbs" in ceil and kv_set < ceil["l2_bytes"]:
-            # the K/V working set is L2-resident: the gathered rows are served from L2, so L2 is
-            # the bound (HBM carries only the compulsory q/k/v/out traffic, `traffic`)
-            roofline.update({"bound": "l2", "peak": ceil["l2_rows_gbs"], "frac": achieved / ceil["l2_rows_gbs"],
-                             "peak_source": "measured in this run by the library's L2 probe: whole 256-byte rows "
-                                            f"at random indices over {ceil['l2_rows_set_bytes'] / 2**20:.0f} MiB "
-                                            "(L2 is not in MEASURED_PEAKS.json)",
-                             "hbm_peak": hbm, "frac_of_hbm": achieved / hbm,
-                             "bytes_read_per_algorithmic_byte": 1.5 if e == 2 else 1.0})
-    if len(kinds) > 1:
-        # several designs in one step: each design's work over its runs' layer time (RoPE included)
-        per = {}
-        for name, kd in design.items():
-            t = per.setdefault(kd, [0.0, 0])
-            t[0] += layers_ms[name]
-            t[1] += pairs[name]
-        roofline["per_design"] = {}
-        for kd, (ms, pr) in per.items():
-            if kd == 2:
-                ach = 4 * D * Hq * pr * L / (ms / 1e3) / 1e12
-                roofline["per_design"][ris.DESIGNS[kd]] = {"bound": "tensor", "achieved": ach, "peak": tc,
-                                                           "unit": "TFLOP/s", "frac": ach / tc, "ms_per_step": ms}
-            else:
-                ach = pr * L * kv_row_bytes / (ms / 1e3) / 1e9
-                ent = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
-                       "ms_per_step": ms}
-                kv_set = N * Hkv * D * e * (3 if e == 2 else 2)
-                if "l2_rows_gbs" in ceil and kv_set < ceil["l2_bytes"]:
-                    ent.update({"bound": "l2", "peak": ceil["l2_rows_gbs"], "frac": ach / ceil["l2_rows_gbs"],
-                                "frac_of_hbm": ach / hbm})
-                roofline["per_design"][ris.DESIGNS[kd]] = ent
-        dom = max(per, key=lambda kd: per[kd][0])
-        top = roofline["per_design"][ris.DESIGNS[dom]]
-        roofline.update({k: top[k] for k in ("bound", "achieved", "peak", "unit", "frac")})
-        for k in ("hbm_peak", "frac_of_hbm", "bytes_read_per_algorithmic_byte", "peak_source"):
-            roofline.pop(k, None)
-        roofline["peak_source"] = "per design, see per_design"
-        roofline["kernel"] = "mixed designs; headline = " + ris.DESIGNS[dom] + " (most device time)"
-        roofline["note"] = "per design: its runs' layer time per step (RoPE included), not the kernel alone"
+        # several designs in one step: the headline is the design with the most kernel time
+        dom = max(per_design, key=lambda kd: per_design[kd]["device_ms_per_step"] or 0.0)
+        roofline = dict(per_design[dom])
+        roofline["kernel"] = "mixed designs; headline = " + per_design[dom]["kernel"] + " (most kernel time)"
+        roofline["median_launch_ms_per_run"] = median_per_run
+        roofline["per_design"] = {ris.DESIGNS[kd]: ent for kd, ent in per_design.items()}
     # the sampled-pair roofline: max(sampled FLOPs / tensor peak, min(row, tile) K/V bytes / bandwidth)
     flops = 4 * D * Hq * total_pairs * L
     b_row = total_pairs * L * kv_row_bytes

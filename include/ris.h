@@ -263,7 +263,7 @@ ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double 
 /* Attention kernel design a layer call on `mask` uses for this input dtype and head_dim
  * (host-only, no device work): 0 register gather, 1 TMA gather, 2 tcgen05 masked dense tiles,
  * 3 fp32 gather; -1 for invalid arguments. bf16 calls with head_dim 128 use tiles when the
- * mask is dense or keeps at least 9.7% of the causal pairs, the register gather otherwise;
+ * mask is dense or keeps at least 8.5% of the causal pairs, the register gather otherwise;
  * RIS_FORCE_DESIGN = gather | tma | tile in the environment overrides (benchmarking). */
 int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim);
 

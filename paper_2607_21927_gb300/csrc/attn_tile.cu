@@ -162,16 +162,6 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major)
            | ((uint32_t)(M >> 4) << 24);
 }
 
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc)
-{
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a), "l"(b), "r"(idesc), "r"(acc)
-        : "memory");
-}
-
 // A operand from TMEM (rows in lanes, 16-bit values packed two per column), B from shared memory.
 __device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc)
 {
@@ -206,6 +196,34 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v)
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 32 lanes x 64 consecutive 32-bit columns, loaded and waited for in one statement (the
+// registers are defined only once the wait has passed).
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float *v)
+{
+    uint32_t r[64];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x64.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%64];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Two 32-column stores (32 lanes each) and one wait for both.
+__device__ __forceinline__ void tmem_st32x2(uint32_t ta, const uint32_t *a, uint32_t tb, const uint32_t *b)
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33};\n\t"
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%1], {%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63,%64,%65};\n\t"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(ta), "r"(tb),
+        "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(a[4]), "r"(a[5]), "r"(a[6]), "r"(a[7]), "r"(a[8]), "r"(a[9]), "r"(a[10]), "r"(a[11]), "r"(a[12]), "r"(a[13]), "r"(a[14]), "r"(a[15]), "r"(a[16]), "r"(a[17]), "r"(a[18]), "r"(a[19]), "r"(a[20]), "r"(a[21]), "r"(a[22]), "r"(a[23]), "r"(a[24]), "r"(a[25]), "r"(a[26]), "r"(a[27]), "r"(a[28]), "r"(a[29]), "r"(a[30]), "r"(a[31]),
+        "r"(b[0]), "r"(b[1]), "r"(b[2]), "r"(b[3]), "r"(b[4]), "r"(b[5]), "r"(b[6]), "r"(b[7]), "r"(b[8]), "r"(b[9]), "r"(b[10]), "r"(b[11]), "r"(b[12]), "r"(b[13]), "r"(b[14]), "r"(b[15]), "r"(b[16]), "r"(b[17]), "r"(b[18]), "r"(b[19]), "r"(b[20]), "r"(b[21]), "r"(b[22]), "r"(b[23]), "r"(b[24]), "r"(b[25]), "r"(b[26]), "r"(b[27]), "r"(b[28]), "r"(b[29]), "r"(b[30]), "r"(b[31])
+        : "memory");
+}
+
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float *v)
 {
     asm volatile(
@@ -233,6 +251,15 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *v)
         "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
         : "memory");
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// 2^x by the SFU (ex2.approx, relative error about 2^-22, subnormal results flushed to 0);
+// 2^-inf = 0.
+__device__ __forceinline__ float ex2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
@@ -490,16 +517,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             float sv[64];
             const uint32_t sb = ((j & 1) ? t_s1 : t_s0) + lane_off + 64 * hf;
-            tmem_ld32(sb, sv);
-            tmem_ld32(sb + 32, sv + 32);
+            tmem_ld64(sb, sv);
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_S_EMPTY + st]));
 
-            // mask, scale, partial row max as a tree, then the full row max with the partner
+            // mask, partial row max as a tree (the scale is positive: it is applied to the max
+            // and folded into the exponent of P), then the full row max with the partner
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
-                sv[c] = ((cw0 >> c) & 1u) ? sv[c] * sc : -INFINITY;
-                sv[32 + c] = ((cw1 >> c) & 1u) ? sv[32 + c] * sc : -INFINITY;
+                sv[c] = ((cw0 >> c) & 1u) ? sv[c] : -INFINITY;
+                sv[32 + c] = ((cw1 >> c) & 1u) ? sv[32 + c] : -INFINITY;
             }
             cw0 = nw0;
             cw1 = nw1;
@@ -509,7 +536,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mx8[e] = fmaxf(fmaxf(fmaxf(sv[e], sv[e + 8]), fmaxf(sv[e + 16], sv[e + 24])),
                                fmaxf(fmaxf(sv[e + 32], sv[e + 40]), fmaxf(sv[e + 48], sv[e + 56])));
             const float pm = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * sc;
             float om;
             ok = exchange(j, pm, om);
             if (!ok) break;
@@ -551,7 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t hw[32], lw[32];
 #pragma unroll
             for (int w = 0; w < 32; ++w) {
-                const float p0 = exp2f(sv[2 * w] - mu), p1 = exp2f(sv[2 * w + 1] - mu);
+                const float p0 = ex2(fmaf(sv[2 * w], sc, -mu)), p1 = ex2(fmaf(sv[2 * w + 1], sc, -mu));
                 lsum[w & 3] += p0 + p1;
                 const uint32_t b0 = __float_as_uint(p0), b1 = __float_as_uint(p1);
                 hw[w] = __byte_perm(b0, b1, 0x7632);
@@ -559,10 +586,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             l += (lsum[0] + lsum[1]) + (lsum[2] + lsum[3]);
             const uint32_t pt = ((j & 1) ? t_s1 : t_s0) + lane_off;
-            tmem_st16(pt + 32 * hf, hw);
-            tmem_st16(pt + 32 * hf + 16, hw + 16);
-            tmem_st16(pt + 64 + 32 * hf, lw);
-            tmem_st16(pt + 64 + 32 * hf + 16, lw + 16);
+            tmem_st32x2(pt + 32 * hf, hw, pt + 64 + 32 * hf, lw);
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_P_FULL + st]));
         }

@@ -165,8 +165,8 @@ bool use_tma_gather() { return std::string(forced_design()) == "tma" && tma_gath
 // Union density at and above which masked dense tiles beat gathering pair by pair (bf16,
 // head dim 128): a tile costs the dense causal products (x2.5 for the precision splits)
 // whatever the mask, a gathered pair 1.5 KB of K/V rows. Measured crossover on Qwen2-shaped
-// layers: 9.9% of the causal pairs at N = 32768 and 9.7% at N = 65536.
-constexpr double kTileDensity = 0.097;
+// layers: 8.6% of the causal pairs at N = 32768 and 8.4% at N = 65536.
+constexpr double kTileDensity = 0.085;
 
 bool use_tile_design(const ris_mask_s *m)
 {
