@@ -371,16 +371,17 @@ def run_reference(a, rank):
 
 
 # ----------------------------------------------------------------------------- traffic record
-def recorded_traffic(kernel_file: str, workload: str):
-    """DRAM bytes per launch of `kernel_file`'s kernel at `workload`, from the committed ncu
-    record, if it was taken on the current kernel source."""
+def recorded_traffic(kernel_files, workload: str):
+    """DRAM bytes per launch (per layer call, summed over its launches) of the kernels of
+    `kernel_files` at `workload`, from the committed ncu record, if it was taken on the
+    current sources."""
     rec = os.path.join(ROOT, "profiles", "traffic.json")
-    src = os.path.join(ROOT, "paper_2607_21927_gb300", "csrc", kernel_file)
     try:
         data = json.load(open(rec))
-        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        ent = data.get(kernel_file, {}).get(workload)
-        if ent and ent.get("source_sha256_16") == h:
+        hs = [hashlib.sha256(open(os.path.join(ROOT, "paper_2607_21927_gb300", "csrc", f), "rb").read()).hexdigest()[:16]
+              for f in kernel_files]
+        ent = data.get("+".join(kernel_files), {}).get(workload)
+        if ent and ent.get("source_sha256_16") == (hs[0] if len(hs) == 1 else hs):
             return ent.get("dram_bytes_per_launch_full_size")
     except Exception:
         pass
@@ -679,7 +680,7 @@ def main():
     oshape = lambda ns: (ns, N, Hq, D) if per_seed else (N, Hq, D)  # noqa: E731
     outs = [[torch.empty(oshape(ns), dtype=tdt, device=dev) for _ in range(L)] for (_, _, _, ns) in runs]
     stream = torch.cuda.current_stream()
-    pairs, design = {}, {}
+    pairs, design, cliques = {}, {}, {}
     mask_events = []  # (run, start, mask built, layers done) events of each run while `timing` is set
     timing = [False]
 
@@ -691,8 +692,11 @@ def main():
             m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom, per_seed=per_seed)
             if timing[0]:
                 mask_events[-1][2].record(stream)
-            pairs[name] = m.info().n_pairs
+            mi = m.info()
+            pairs[name] = mi.n_pairs
             design[name] = ris.ris_attention_design(m, tdt, D)
+            # the Structural split attends the in-block clique pairs on the tiles, not by gathering
+            cliques[name] = mi.params.clique_pairs * mi.n_masks if design[name] == 4 else 0
             if a.shard == "rows" and world > 1:
                 # every rank builds the same mask and attends its own balanced range of rows
                 b = ris.ris_mask_row_split(m, world)
@@ -764,8 +768,9 @@ def main():
     kv_row_bytes = Hkv * 2 * D * e  # K and V rows of one key, all KV heads
     kv_set = N * Hkv * D * e * (3 if e == 2 else 2)  # rotated K (hi + lo for bf16) and V of a layer
     gather_names = {0: "k_attn_bf16 (register gather)", 1: "k_attn_tma (TMA gather4)", 2: "k_attn_tile (tcgen05 masked tiles)",
-                    3: "k_attn_f32 (fp32 gather)"}
-    traffic_file = {0: "attn_bf16.cu", 2: "attn_tile.cu"}
+                    3: "k_attn_f32 (fp32 gather)",
+                    4: "k_attn_tile clique pass + k_attn_bf16 (Structural split: cliques on the tiles, the rest gathered)"}
+    traffic_file = {0: ("attn_bf16.cu",), 2: ("attn_tile.cu",), 4: ("attn_tile.cu", "attn_bf16.cu")}
 
     def design_roofline(kd, names):
         """Roofline of design kd's kernel over the launches of runs `names`: algorithmic work per
@@ -789,10 +794,17 @@ def main():
                         "design_note": "dense-causal tile FLOPs / sustained bf16 peak over the launch time (the "
                                        "kernel issues 2.5x that in hi/lo split products)"})
         else:
-            achieved = pairs_launch * kv_row_bytes / (mean_ms / 1e3) / 1e9
+            # gathered pairs: all of them, or with the Structural split all but the cliques (whose
+            # tile pass is inside the launch time: the split's two launches are timed as one)
+            gathered = pairs_launch - sum(cliques[nm] for nm in names) / len(names)
+            achieved = gathered * kv_row_bytes / (mean_ms / 1e3) / 1e9
             ent.update({"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
                         "peak_source": ceil["hbm_source"],
-                        "bytes": "algorithmic: K and V rows of every sampled pair, all KV heads"})
+                        "bytes": "algorithmic: K and V rows of every gathered sampled pair, all KV heads"})
+            if kd == 4:
+                ent["clique_pairs_per_launch"] = sum(cliques[nm] for nm in names) / len(names)
+                ent["note"] = ("time of both launches (clique pass on the tiles, then the gather); bytes of the "
+                               "gathered pairs only")
             if "l2_rows_gbs" in ceil and kv_set < ceil["l2_bytes"]:
                 # the K/V working set is L2-resident: the gathered rows are served from L2, so L2 is
                 # the bound (HBM carries only the compulsory q/k/v/out traffic, `traffic`)

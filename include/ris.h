@@ -262,9 +262,15 @@ ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double 
 
 /* Attention kernel design a layer call on `mask` uses for this input dtype and head_dim
  * (host-only, no device work): 0 register gather, 1 TMA gather, 2 tcgen05 masked dense tiles,
- * 3 fp32 gather; -1 for invalid arguments. bf16 calls with head_dim 128 use tiles when the
- * mask is dense or keeps at least 8.5% of the causal pairs, the register gather otherwise;
- * RIS_FORCE_DESIGN = gather | tma | tile in the environment overrides (benchmarking). */
+ * 3 fp32 gather, 4 Structural split; -1 for invalid arguments. bf16 calls with head_dim 128
+ * use tiles when the mask is dense or keeps at least 8.5% of the causal pairs in what a
+ * gather would fetch. The Structural split applies to Structural masks (not per seed) whose
+ * blocks hold at least 256 tokens: a first launch attends every row to its own block's clique
+ * on the tiles (Methods, "Sampling Modes": the in-block pairs are all kept) and the register
+ * gather continues that softmax over the row's other keys, so the clique pairs are never
+ * gathered; the result is the same single softmax over the row's whole key set.
+ * RIS_FORCE_DESIGN = gather | tma | tile | cliques in the environment overrides
+ * (benchmarking). */
 int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim);
 
 /* Synchronise `stream` and report (then clear) the device error words: RIS_ERR_DEVICE_TIMEOUT

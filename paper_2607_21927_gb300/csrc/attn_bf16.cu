@@ -154,6 +154,13 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     const Task t = decode_task(a, tid);
     int64_t beg, n;
     key_range<DENSE>(a, t, beg, n);
+    // Structural split: the keys of the row's own block (its clique, i - b0 + 1 keys up to the
+    // row) end the ascending list and were attended by the tile kernel's clique pass
+    const bool cliques = a.clique_B > 0;
+    if (cliques) {
+        n -= t.i - (t.i / a.clique_B) * a.clique_B + 1;
+        if (n < 0) n = 0;
+    }
     const TIdx *cols = DENSE ? nullptr : reinterpret_cast<const TIdx *>(a.col) + beg;
 
     // ---- query fragments (B operand of the score product), head p of this KV group
@@ -164,7 +171,16 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
             const int d0 = kelem<D, WIDE>(ks, q);
-            if (QSPLIT) {
+            if (QSPLIT && a.q_lo != nullptr) {  // the split given as a bf16 pair
+                const uint2 wh = hv ? *reinterpret_cast<const uint2 *>(reinterpret_cast<const __nv_bfloat16 *>(a.q) + qrow + d0)
+                                    : make_uint2(0u, 0u);
+                const uint2 wl = hv ? *reinterpret_cast<const uint2 *>(reinterpret_cast<const __nv_bfloat16 *>(a.q_lo) + qrow + d0)
+                                    : make_uint2(0u, 0u);
+                qh[ks][0] = wh.x;
+                qh[ks][1] = wh.y;
+                ql[ks][0] = wl.x;
+                ql[ks][1] = wl.y;
+            } else if (QSPLIT) {
                 float4 x = hv ? *reinterpret_cast<const float4 *>(reinterpret_cast<const float *>(a.q) + qrow + d0)
                               : make_float4(0.f, 0.f, 0.f, 0.f);
                 const float h0 = __bfloat162float(__float2bfloat16_rn(x.x));
@@ -196,6 +212,32 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     for (int mt = 0; mt < MT; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
     const float sc = a.scale_log2;
+    if (cliques) {
+        // start from the clique pass's softmax: maximum = its log-sum-exp, sum 1 (on one lane
+        // of the eight that share heads 2q, 2q+1), O = its normalised output, laid out as the
+        // epilogue stores it
+        const int hh0 = 2 * q, hh1 = 2 * q + 1;
+        const float *po = a.part_o + (t.i * a.Hq + (int64_t)t.g * a.G) * D;
+        const float *pl = a.part_lse + t.i * a.Hq + (int64_t)t.g * a.G;
+#pragma unroll
+        for (int hs = 0; hs < 2; ++hs) {
+            const int hh = hs ? hh1 : hh0;
+            if (hh >= a.G) continue;
+            (hs ? m1 : m0) = pl[hh];
+            (hs ? l1 : l0) = p == 0 ? 1.f : 0.f;
+#pragma unroll
+            for (int r = 0; r < MT / 4; ++r) {
+                const float4 *src = reinterpret_cast<const float4 *>(po + (int64_t)hh * D + velem<D, WIDE>(4 * r, p));
+                const float4 x0 = src[0], x1 = src[1];
+                const float run[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    o[4 * r + j][hs] = run[2 * j];
+                    o[4 * r + j][2 + hs] = run[2 * j + 1];
+                }
+            }
+        }
+    }
 
     // ---- key indices, prefetched 64 keys (4 groups) ahead: lane holds positions
     //      64c + lane and 64c + 32 + lane of chunk c; slots past the row read the row itself

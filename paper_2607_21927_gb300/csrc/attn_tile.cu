@@ -34,6 +34,11 @@
 // pipe waited for them: 7.2 ms (the products alone 6.0 ms). 128-key tiles with the query in
 // TMEM beat 64-key tiles with the query in shared memory and three stages (7.8 ms).
 //
+// The clique pass of the Structural split (CLIQUE) runs the same pipeline over the key tiles
+// of each row's own Structural block only (every key of the block up to the row is kept: no
+// bitmap), and writes the normalised partial output and its log-sum-exp for the register
+// gather to continue from.
+//
 // Every mbarrier wait is bounded; a wait that gives up sets bit 1 of the device error word,
 // every role falls through to the end, TMEM is released and the CTA returns.
 #include <cuda.h>
@@ -297,7 +302,7 @@ struct TileMaps {
     CUtensorMap kh, kl, v;
 };
 
-template <bool SPLIT, bool DENSE, typename TOut>
+template <bool SPLIT, bool DENSE, bool CLIQUE, typename TOut>
 __global__ void __launch_bounds__(kThreads, 1)
     k_attn_tile(const AttnArgs a, const __grid_constant__ TileMaps maps, const void *q_hi, const void *q_lo)
 {
@@ -321,7 +326,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int g = h / a.G;
     const int mask_id = s * a.heads_keyed + (a.heads_keyed > 1 ? g : 0);
     const int64_t last_row = (q0 + BM - 1 < a.row1 - 1) ? q0 + BM - 1 : a.row1 - 1;
-    const int n_kt = (int)(last_row / BN) + 1;  // causal: key tiles 0 .. last_row / BN
+    // causal: key tiles kt0 .. last_row / BN (kt0 = 0, or the tile of the first block start)
+    const int kt0 = CLIQUE ? (int)(((q0 / a.clique_B) * a.clique_B) / BN) : 0;
+    const int n_kt = (int)(last_row / BN) + 1 - kt0;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < NBAR; ++i) {
@@ -362,8 +369,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t dk = sbase + OFF_K + st * K_STAGE;
                 mbar_arrive_expect_tx(bk, (SPLIT ? 2 : 1) * KV_ARR);
                 for (int blk = 0; blk < 2; ++blk) {
-                    tma_load_3d(dk + blk * KV_BLK, &maps.kh, 64 * blk, g, j * BN, bk);
-                    if (SPLIT) tma_load_3d(dk + KV_ARR + blk * KV_BLK, &maps.kl, 64 * blk, g, j * BN, bk);
+                    tma_load_3d(dk + blk * KV_BLK, &maps.kh, 64 * blk, g, (kt0 + j) * BN, bk);
+                    if (SPLIT) tma_load_3d(dk + KV_ARR + blk * KV_BLK, &maps.kl, 64 * blk, g, (kt0 + j) * BN, bk);
                 }
                 nk = j + 1;
                 if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_V_EMPTY + st]), par);
@@ -371,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t bv = smem_u32(&bars[B_V_FULL + st]);
                 const uint32_t dv = sbase + OFF_V + st * V_STAGE;
                 mbar_arrive_expect_tx(bv, KV_ARR);
-                for (int blk = 0; blk < 2; ++blk) tma_load_3d(dv + blk * KV_BLK, &maps.v, 64 * blk, g, j * BN, bv);
+                for (int blk = 0; blk < 2; ++blk) tma_load_3d(dv + blk * KV_BLK, &maps.v, 64 * blk, g, (kt0 + j) * BN, bv);
                 nv = j + 1;
             }
             // let the copies requested last into each stage land before the CTA can leave
@@ -460,15 +467,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int64_t i = q0 + r;
         const bool row_ok = i >= a.row0 && i < a.row1;
         const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
-        const uint32_t *bm = DENSE ? nullptr
-                                   : a.bitmap + (int64_t)mask_id * a.words_per_mask + (row_ok ? row_word_offset(i) : 0);
+        const uint32_t *bm = (DENSE || CLIQUE) ? nullptr
+                                               : a.bitmap + (int64_t)mask_id * a.words_per_mask + (row_ok ? row_word_offset(i) : 0);
         const int64_t last_word = i >> 5;
         const float sc = a.scale_log2;
         float m_used = -INFINITY, l = 0.f;
-        // bitmap word e (0, 1) of keys 128j + 64hf + 32e .. +31 of this row, fetched one tile ahead
+        // bitmap word e (0, 1) of keys 128 (kt0 + j) + 64hf + 32e .. +31 of this row, fetched
+        // one tile ahead
         auto mask_word = [&](int j, int e) -> uint32_t {
             if (!row_ok) return 0u;
-            const int64_t k0 = (int64_t)j * BN + 64 * hf + 32 * e;
+            const int64_t k0 = (int64_t)(kt0 + j) * BN + 64 * hf + 32 * e;
+            if (CLIQUE) {  // keys of the row's block up to the row: offsets lo .. hi of the word
+                const int64_t lo = (i / a.clique_B) * a.clique_B - k0, hi = i - k0;
+                if (hi < 0 || lo > 31) return 0u;
+                uint32_t w = hi >= 31 ? 0xFFFFFFFFu : ((2u << hi) - 1u);
+                if (lo > 0) w &= ~((1u << lo) - 1u);
+                return w;
+            }
             if (DENSE) {
                 const int64_t lim = i - k0;  // keys k0 .. i are kept
                 return lim >= 31 ? 0xFFFFFFFFu : (lim < 0 ? 0u : ((2u << lim) - 1u));
@@ -599,7 +614,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const float lt = l + ol;
             const float inv = lt > 0.f ? 1.f / lt : 0.f;
-            TOut *out = reinterpret_cast<TOut *>(a.out) + (((int64_t)s * a.N + (row_ok ? i : 0)) * a.Hq + h) * DT + 64 * hf;
+            TOut *out = CLIQUE ? reinterpret_cast<TOut *>(a.part_o + ((row_ok ? i : 0) * a.Hq + h) * DT + 64 * hf)
+                               : reinterpret_cast<TOut *>(a.out) + (((int64_t)s * a.N + (row_ok ? i : 0)) * a.Hq + h) * DT +
+                                     64 * hf;
             float ov[32];
 #pragma unroll
             for (int c4 = 0; c4 < 2; ++c4) {
@@ -611,8 +628,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int e = 0; e < 4; ++e) store8<TOut>(out + 32 * c4 + 8 * e, ov + 8 * e);
                 }
             }
-            if (row_ok && hf == 0 && a.lse != nullptr)
+            if (CLIQUE) {
+                if (row_ok && hf == 0) a.part_lse[i * a.Hq + h] = m_used + __log2f(lt);
+            } else if (row_ok && hf == 0 && a.lse != nullptr) {
                 a.lse[((int64_t)s * a.Hq + h) * a.N + i] = (m_used + __log2f(lt)) * kLn2;
+            }
         }
     }
 
@@ -653,10 +673,10 @@ bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows)
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool SPLIT, bool DENSE, typename TOut>
+template <bool SPLIT, bool DENSE, typename TOut, bool CLIQUE = false>
 cudaError_t launch_t(const AttnArgs &a, const TileMaps &maps, const void *q_hi, const void *q_lo, cudaStream_t s)
 {
-    auto kern = k_attn_tile<SPLIT, DENSE, TOut>;
+    auto kern = k_attn_tile<SPLIT, DENSE, CLIQUE, TOut>;
     static bool attr = false;
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
@@ -684,6 +704,15 @@ cudaError_t read_tile_error(unsigned int *out)
     return cudaMemcpyToSymbol(g_ris_tile_error, &zero, sizeof(unsigned int));
 }
 
+// K / V tensor maps of a call (the key low part only with split queries and keys).
+bool make_maps(TileMaps &maps, const AttnArgs &a, bool split)
+{
+    if (!make_map3(&maps.kh, a.k, a.N, a.Hkv, BN) || !make_map3(&maps.v, a.v, a.N, a.Hkv, BN)) return false;
+    if (split) return make_map3(&maps.kl, a.k_lo, a.N, a.Hkv, BN);
+    maps.kl = maps.kh;
+    return true;
+}
+
 // q_hi / q_lo: queries as a bf16 pair [N][Hq][128] (q_lo null: exact bf16 queries and keys,
 // one score product); a.k / a.k_lo: keys as a pair; a.v: values. Head dim 128 only.
 cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const void *q_lo, int out_dtype, bool dense,
@@ -693,13 +722,7 @@ cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const voi
     std::lock_guard<std::mutex> lk(mu);
     const bool split = q_lo != nullptr;
     alignas(64) TileMaps maps;
-    if (!make_map3(&maps.kh, a.k, a.N, a.Hkv, BN) || !make_map3(&maps.v, a.v, a.N, a.Hkv, BN))
-        return cudaErrorInvalidValue;
-    if (split) {
-        if (!make_map3(&maps.kl, a.k_lo, a.N, a.Hkv, BN)) return cudaErrorInvalidValue;
-    } else {
-        maps.kl = maps.kh;
-    }
+    if (!make_maps(maps, a, split)) return cudaErrorInvalidValue;
     if (out_dtype == RIS_F32) {
         if (split) return dense ? launch_t<true, true, float>(a, maps, q_hi, q_lo, s) : launch_t<true, false, float>(a, maps, q_hi, q_lo, s);
         return dense ? launch_t<false, true, float>(a, maps, q_hi, q_lo, s) : launch_t<false, false, float>(a, maps, q_hi, q_lo, s);
@@ -707,6 +730,18 @@ cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const voi
     if (split)
         return dense ? launch_t<true, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s) : launch_t<true, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
     return dense ? launch_t<false, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s) : launch_t<false, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
+}
+
+cudaError_t launch_attention_tile_cliques(const AttnArgs &a, const void *q_hi, const void *q_lo, cudaStream_t s)
+{
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lk(mu);
+    if (a.clique_B < 1 || a.part_o == nullptr || a.part_lse == nullptr || a.n_sets != 1) return cudaErrorInvalidValue;
+    const bool split = q_lo != nullptr;
+    alignas(64) TileMaps maps;
+    if (!make_maps(maps, a, split)) return cudaErrorInvalidValue;
+    return split ? launch_t<true, false, float, true>(a, maps, q_hi, q_lo, s)
+                 : launch_t<false, false, float, true>(a, maps, q_hi, q_lo, s);
 }
 
 }  // namespace ris

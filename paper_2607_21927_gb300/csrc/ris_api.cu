@@ -35,6 +35,7 @@ using namespace ris;
 
 struct ris_mask_s {
     int64_t N = 0;
+    int32_t mode = 0;  // ris_mode of the call that built it
     int32_t n_masks = 0, heads_keyed = 1, kv_heads = 1, n_seeds = 0, per_seed = 0;
     int32_t col_bytes = 2, dense = 0;
     int64_t n_pairs = 0, words_per_mask = 0;
@@ -150,7 +151,8 @@ std::pair<cudaEvent_t, cudaEvent_t> timer_pair()
 }
 
 // Kernel design override for benchmarking the designs against each other:
-// RIS_FORCE_DESIGN = gather (register gather), tma (TMA gather) or tile (masked dense tiles).
+// RIS_FORCE_DESIGN = gather (register gather), tma (TMA gather), tile (masked dense tiles) or
+// cliques (the Structural split, where the mask allows it).
 const char *forced_design()
 {
     static const std::string d = [] {
@@ -160,7 +162,6 @@ const char *forced_design()
     return d.c_str();
 }
 
-bool use_tma_gather() { return std::string(forced_design()) == "tma" && tma_gather_available(); }
 
 // Union density at and above which masked dense tiles beat gathering pair by pair (bf16,
 // head dim 128): a tile costs the dense causal products (x2.5 for the precision splits)
@@ -168,13 +169,30 @@ bool use_tma_gather() { return std::string(forced_design()) == "tma" && tma_gath
 // layers: 8.6% of the causal pairs at N = 32768 and 8.4% at N = 65536.
 constexpr double kTileDensity = 0.085;
 
-bool use_tile_design(const ris_mask_s *m)
+// Smallest Structural block for which the cliques go to the tile kernel (a block then fills
+// at least two 128 x 128 tiles' worth of pairs).
+constexpr int64_t kCliqueMinBlock = 256;
+
+// Design of a layer call: 0 register gather, 1 TMA gather, 2 masked dense tiles, 3 fp32
+// gather, 4 Structural split (the in-block cliques on the tile kernel, the remaining keys on
+// the register gather, one softmax). The gather's cost grows with the pairs it gathers (with
+// the split: all but the cliques), a tile's does not, hence the density threshold.
+int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim)
 {
+    if (dtype == RIS_F32) return 3;
     const std::string f = forced_design();
-    if (!tile_design_available() || f == "gather" || f == "tma") return false;
-    if (f == "tile" || m->dense) return true;
-    const double causal = (double)m->n_masks * ((double)m->N * (double)(m->N + 1) / 2.0);
-    return (double)m->n_pairs >= kTileDensity * causal;
+    if (f == "tma" && tma_gather_available()) return 1;
+    if (f == "gather") return 0;
+    const bool tiles = head_dim == 128 && tile_design_available();
+    if (tiles && (f == "tile" || m->dense)) return 2;
+    const bool split = tiles && m->mode == RIS_MODE_STRUCTURAL && !m->per_seed && m->params.block >= kCliqueMinBlock;
+    if (split && f == "cliques") return 4;
+    if (tiles) {
+        const double causal = (double)m->n_masks * ((double)m->N * (double)(m->N + 1) / 2.0);
+        const double gathered = (double)m->n_pairs - (split ? (double)m->n_masks * (double)m->params.clique_pairs : 0.0);
+        if (gathered >= kTileDensity * causal) return 2;
+    }
+    return split ? 4 : 0;
 }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -396,6 +414,7 @@ ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double d
     mk->n_seeds = n_seeds;
     mk->per_seed = per_seed;
     mk->col_bytes = N <= 65536 ? 2 : 4;
+    mk->mode = mode;
     mk->params = p;
     mk->stream = s;
     if (p.dense) {
@@ -546,8 +565,10 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     const int64_t N = m->N;
     if (row1 < 0) row1 = N;
     prepare_pool_once();
-    const bool tile = dtype == RIS_BF16 && head_dim == 128 && use_tile_design(m);
-    Scratch qt, qtl, kt, ktl;
+    const int design = design_of(m, dtype, head_dim);
+    const bool tile = design == 2, cliques = design == 4;
+    const bool q_pair = tile || cliques;  // queries as a bf16 hi + lo pair
+    Scratch qt, qtl, kt, ktl, po, pl;
     const void *qu = q, *ku = k, *kl = nullptr, *q_lo = nullptr;
     bool q_split = false;
     if (rope != nullptr && rope->kind != RIS_ROPE_NONE) {
@@ -558,10 +579,10 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         ra.D = head_dim;
         ra.mscale = (float)ms;
         const size_t nq = (size_t)N * heads * head_dim, nk = (size_t)N * kv_heads * head_dim;
-        // rotated queries: fp32 (split into bf16 hi + lo by the gather kernels) or, for the
-        // tile kernel, a bf16 hi + lo pair; rotated keys in fp32, or for bf16 inputs a bf16
-        // hi + lo pair
-        if (tile) {
+        // rotated queries: fp32 (split into bf16 hi + lo by the gather kernels) or, when the
+        // tile kernel runs, a bf16 hi + lo pair; rotated keys in fp32, or for bf16 inputs a
+        // bf16 hi + lo pair
+        if (q_pair) {
             RIS_CUDA(qt.alloc(nq * 2, s));
             RIS_CUDA(qtl.alloc(nq * 2, s));
         } else {
@@ -571,9 +592,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         if (dtype == RIS_BF16) RIS_CUDA(ktl.alloc(nk * 2, s));
         ra.x_in = q;
         ra.x_out = qt.p;
-        ra.x_out_lo = tile ? qtl.p : nullptr;
+        ra.x_out_lo = q_pair ? qtl.p : nullptr;
         ra.H = heads;
-        RIS_CUDA(launch_rope(ra, dtype, tile ? RIS_BF16 : RIS_F32, s));
+        RIS_CUDA(launch_rope(ra, dtype, q_pair ? RIS_BF16 : RIS_F32, s));
         ra.x_in = k;
         ra.x_out = kt.p;
         ra.x_out_lo = ktl.p;
@@ -587,6 +608,7 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     }
     AttnArgs a{};
     a.q = qu;
+    a.q_lo = q_pair ? q_lo : nullptr;
     a.k = ku;
     a.k_lo = kl;
     a.v = v;
@@ -606,11 +628,21 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.row0 = row0;
     a.row1 = row1;
     a.n_tasks = (int64_t)a.n_sets * (row1 - row0) * kv_heads;
+    if (cliques) {
+        RIS_CUDA(po.alloc((size_t)N * heads * head_dim * sizeof(float), s));
+        RIS_CUDA(pl.alloc((size_t)N * heads * sizeof(float), s));
+        a.clique_B = m->params.block;
+        a.part_o = (float *)po.p;
+        a.part_lse = (float *)pl.p;
+    }
     const auto ev = timer_pair();
     if (ev.first) RIS_CUDA(cudaEventRecord(ev.first, s));
-    if (tile)
+    if (tile) {
         RIS_CUDA(launch_attention_tile(a, qu, q_lo, out_dtype, m->dense != 0, s));
-    else if (dtype == RIS_BF16 && use_tma_gather())
+    } else if (cliques) {  // the cliques on the tiles, then the gather continues their softmax
+        RIS_CUDA(launch_attention_tile_cliques(a, qu, a.q_lo, s));
+        RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, false, s));
+    } else if (design == 1)
         RIS_CUDA(launch_attention_tma(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
     else if (dtype == RIS_BF16)
         RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
@@ -682,9 +714,7 @@ ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches)
 int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim)
 {
     if (mask == nullptr || (dtype != RIS_F32 && dtype != RIS_BF16) || (head_dim != 64 && head_dim != 128)) return -1;
-    if (dtype == RIS_F32) return 3;
-    if (head_dim == 128 && use_tile_design(mask)) return 2;
-    return use_tma_gather() ? 1 : 0;
+    return design_of(mask, dtype, head_dim);
 }
 
 ris_status ris_device_status(void *stream)

@@ -68,7 +68,9 @@ struct RopeArgs {
 
 // Arguments of the attention kernels. One warp handles one task = (set s, row i, KV head g).
 struct AttnArgs {
-    const void *q;         // [N][Hq][D]: fp32 rotated queries (split path) or dtype as given
+    const void *q;         // [N][Hq][D]: fp32 rotated queries (split path) or dtype as given;
+                           // with q_lo set, the bf16 high part of the rotated queries
+    const void *q_lo;      // split path: bf16 low part of the rotated queries (q~ = q + q_lo), or null
     const void *k;         // [N][Hkv][D]
     const void *k_lo;      // bf16 path: low part of the rotated keys (k~ = k + k_lo), or null
     const void *v;         // [N][Hkv][D]
@@ -86,6 +88,14 @@ struct AttnArgs {
     int32_t n_sets;        // output sets: n_seeds for per-seed masks, else 1
     int64_t row0;          // query rows row0 .. row1-1 are computed (0 and N for a whole layer)
     int64_t row1;
+    // Structural cliques on the tiles (0: off): rows are split into blocks of clique_B tokens,
+    // and every key of a row's own block up to the row is kept. The tile kernel's clique pass
+    // attends each row to those keys only and writes part_o / part_lse; the register gather
+    // then starts from that partial softmax and skips the same keys, which are the tail of the
+    // row's ascending key list.
+    int64_t clique_B;
+    float *part_o;         // [N][Hq][D] normalised partial outputs
+    float *part_lse;       // [N][Hq] their log2-domain log-sum-exp
     int32_t pad_;
     float scale_log2;      // log2(e) / sqrt(D)
     int64_t n_tasks;       // n_sets * (row1 - row0) * Hkv
@@ -171,6 +181,8 @@ cudaError_t read_device_error(unsigned int *out, cudaStream_t s);
 bool tile_design_available();
 cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const void *q_lo, int out_dtype, bool dense,
                                   cudaStream_t s);
+// The clique pass of the Structural split (a.clique_B > 0): writes a.part_o / a.part_lse.
+cudaError_t launch_attention_tile_cliques(const AttnArgs &a, const void *q_hi, const void *q_lo, cudaStream_t s);
 cudaError_t read_tile_error(unsigned int *out);
 
 }  // namespace ris

@@ -154,7 +154,8 @@ def ris_version() -> str:
     return lib().ris_version().decode()
 
 
-DESIGNS = {0: "register gather", 1: "TMA gather", 2: "tcgen05 masked tiles", 3: "fp32 gather"}
+DESIGNS = {0: "register gather", 1: "TMA gather", 2: "tcgen05 masked tiles", 3: "fp32 gather",
+           4: "cliques on tiles + register gather"}
 
 
 def ris_attention_design(mask: "Mask", dtype=torch.bfloat16, head_dim: int = 128) -> int:

@@ -293,3 +293,60 @@ def test_row_ranges_reassemble_the_layer(d, S, D):
     with pytest.raises(ris.RisError):
         ris.ris_attention_masked_rows(m, 5, 5, q, k, v, one, rope=rope)
     m.free()
+
+
+def test_structural_split_design_choice():
+    """C5's Structural mask (blocks of 655) takes the split: cliques on the tiles, the rest
+    gathered; Structural masks with small blocks, per-seed masks and head_dim 64 do not."""
+    m = ris.ris_mask_generate(65536, 2, 1, 0.01, list(range(10)))
+    assert ris.ris_attention_design(m, torch.bfloat16, 128) == 4
+    assert ris.ris_attention_design(m, torch.bfloat16, 64) == 0
+    m.free()
+    m = ris.ris_mask_generate(2000, 2, 1, 0.05, [1])  # B = min(200, 100) = 100 < 256
+    assert ris.ris_attention_design(m, torch.bfloat16, 128) in (0, 2)
+    m.free()
+    m = ris.ris_mask_generate(65536, 2, 1, 0.01, list(range(10)), per_seed=True)
+    assert ris.ris_attention_design(m, torch.bfloat16, 128) != 4
+    m.free()
+
+
+@pytest.mark.parametrize("N,d,S,kind,window,anchors", [(3000, 0.1, 1, 3, 1, 0), (2700, 0.11, 1, 0, 1, 0),
+                                                     (4100, 0.08, 1, 3, 40, 3)],
+                         ids=["yarn", "pre_rotated", "window_anchors"])
+def test_structural_split_full(N, d, S, kind, window, anchors):
+    """The Structural split (blocks of >= 256 tokens) against the oracle on every row: fp32 and
+    bf16 outputs and the log-sum-exp, with and without RoPE, with a local window and anchors
+    reaching outside the block."""
+    Hq, Hkv, D = 12, 2, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=N, outliers=True)
+    seeds = list(range(5, 5 + S))
+    opts = ris.mask_opts(local_window=window, n_anchor=anchors)
+    m = ris.ris_mask_generate(N, Hkv, 1, d, seeds, opts=opts)
+    assert ris.ris_attention_design(m, torch.bfloat16, D) == 4
+    rope = ris.rope_cfg(kind, 1e6, 256) if kind else None
+    out32, lse = ris.ris_attention_masked(m, q, k, v, rope=rope, out_dtype=torch.float32, return_lse=True)
+    out16 = ris.ris_attention_masked(m, q, k, v, rope=rope)
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    m.free()
+    ref, ref_lse = run_oracle(qn, kn, vn, 1, d, seeds, kind, 1e6, 256, W=window, A=anchors)
+    check_bf16_path(to_np(out32), ref)
+    check_bf16_path(to_np(out16), ref, out_bf16=True)
+    np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
+
+
+def test_structural_split_row_ranges():
+    """Row ranges through the Structural split reassemble the whole layer bit for bit."""
+    N, Hq, Hkv, D = 3000, 6, 2, 128
+    (q, k, v), _ = make_inputs(N, Hq, Hkv, D, seed=29, outliers=True)
+    m = ris.ris_mask_generate(N, Hkv, 1, 0.1, [4])
+    assert ris.ris_attention_design(m, torch.bfloat16, D) == 4
+    rope = ris.rope_cfg(3, 1e6, 256)
+    whole = ris.ris_attention_masked(m, q, k, v, rope=rope, out_dtype=torch.float32)
+    bounds = ris.ris_mask_row_split(m, 4)
+    parts = torch.full_like(whole, float("nan"))
+    for r0, r1 in zip(bounds[:-1], bounds[1:]):
+        ris.ris_attention_masked_rows(m, r0, r1, q, k, v, parts, rope=rope)
+    torch.cuda.synchronize()
+    assert torch.equal(parts, whole)
+    m.free()
