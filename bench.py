@@ -680,7 +680,7 @@ def main():
     oshape = lambda ns: (ns, N, Hq, D) if per_seed else (N, Hq, D)  # noqa: E731
     outs = [[torch.empty(oshape(ns), dtype=tdt, device=dev) for _ in range(L)] for (_, _, _, ns) in runs]
     stream = torch.cuda.current_stream()
-    pairs, design, cliques = {}, {}, {}
+    pairs, design, suffix = {}, {}, {}
     mask_events = []  # (run, start, mask built, layers done) events of each run while `timing` is set
     timing = [False]
 
@@ -695,8 +695,9 @@ def main():
             mi = m.info()
             pairs[name] = mi.n_pairs
             design[name] = ris.ris_attention_design(m, tdt, D)
-            # the Structural split attends the in-block clique pairs on the tiles, not by gathering
-            cliques[name] = mi.params.clique_pairs * mi.n_masks if design[name] == 4 else 0
+            # the dense-suffix split attends the rows' dense suffixes (Structural blocks, local
+            # window) on the tiles, not by gathering
+            suffix[name] = mi.suffix_pairs * mi.n_masks if design[name] == 4 else 0
             if a.shard == "rows" and world > 1:
                 # every rank builds the same mask and attends its own balanced range of rows
                 b = ris.ris_mask_row_split(m, world)
@@ -769,7 +770,8 @@ def main():
     kv_set = N * Hkv * D * e * (3 if e == 2 else 2)  # rotated K (hi + lo for bf16) and V of a layer
     gather_names = {0: "k_attn_bf16 (register gather)", 1: "k_attn_tma (TMA gather4)", 2: "k_attn_tile (tcgen05 masked tiles)",
                     3: "k_attn_f32 (fp32 gather)",
-                    4: "k_attn_tile clique pass + k_attn_bf16 (Structural split: cliques on the tiles, the rest gathered)"}
+                    4: "k_attn_tile suffix pass + k_attn_bf16 (dense-suffix split: Structural blocks / local window "
+                       "on the tiles, the rest gathered)"}
     traffic_file = {0: ("attn_bf16.cu",), 2: ("attn_tile.cu",), 4: ("attn_tile.cu", "attn_bf16.cu")}
 
     def design_roofline(kd, names):
@@ -794,16 +796,16 @@ def main():
                         "design_note": "dense-causal tile FLOPs / sustained bf16 peak over the launch time (the "
                                        "kernel issues 2.5x that in hi/lo split products)"})
         else:
-            # gathered pairs: all of them, or with the Structural split all but the cliques (whose
-            # tile pass is inside the launch time: the split's two launches are timed as one)
-            gathered = pairs_launch - sum(cliques[nm] for nm in names) / len(names)
+            # gathered pairs: all of them, or with the dense-suffix split all but the suffixes
+            # (whose tile pass is inside the launch time: the split's two launches are timed as one)
+            gathered = pairs_launch - sum(suffix[nm] for nm in names) / len(names)
             achieved = gathered * kv_row_bytes / (mean_ms / 1e3) / 1e9
             ent.update({"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
                         "peak_source": ceil["hbm_source"],
                         "bytes": "algorithmic: K and V rows of every gathered sampled pair, all KV heads"})
             if kd == 4:
-                ent["clique_pairs_per_launch"] = sum(cliques[nm] for nm in names) / len(names)
-                ent["note"] = ("time of both launches (clique pass on the tiles, then the gather); bytes of the "
+                ent["suffix_pairs_per_launch"] = sum(suffix[nm] for nm in names) / len(names)
+                ent["note"] = ("time of both launches (suffix pass on the tiles, then the gather); bytes of the "
                                "gathered pairs only")
             if "l2_rows_gbs" in ceil and kv_set < ceil["l2_bytes"]:
                 # the K/V working set is L2-resident: the gathered rows are served from L2, so L2 is

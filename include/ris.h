@@ -124,6 +124,11 @@ typedef struct {
     const void *col;
     const uint32_t *bitmap;
     ris_params params;
+    int64_t suffix_pairs;  /* pairs per mask in the rows' dense suffixes: keys lo(i) .. i of row i,
+                              all kept, lo(i) the earlier of the row's Structural block start
+                              (blocks of >= 256 tokens) and its local window start (0 when the
+                              mask is dense, per seed, or has neither span of >= 256); the
+                              dense-suffix split attends these on the tiles */
 } ris_mask_desc;
 
 /* Resolve the scalars of a call on the host (no device work, usable without a GPU).
@@ -262,15 +267,16 @@ ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double 
 
 /* Attention kernel design a layer call on `mask` uses for this input dtype and head_dim
  * (host-only, no device work): 0 register gather, 1 TMA gather, 2 tcgen05 masked dense tiles,
- * 3 fp32 gather, 4 Structural split; -1 for invalid arguments. bf16 calls with head_dim 128
- * use tiles when the mask is dense or keeps at least 8.5% of the causal pairs in what a
- * gather would fetch. The Structural split applies to Structural masks (not per seed) whose
- * blocks hold at least 256 tokens: a first launch attends every row to its own block's clique
- * on the tiles (Methods, "Sampling Modes": the in-block pairs are all kept) and the register
- * gather continues that softmax over the row's other keys, so the clique pairs are never
- * gathered; the result is the same single softmax over the row's whole key set.
- * RIS_FORCE_DESIGN = gather | tma | tile | cliques in the environment overrides
- * (benchmarking). */
+ * 3 fp32 gather, 4 dense-suffix split; -1 for invalid arguments. bf16 calls with head_dim
+ * 128 use tiles when the mask is dense or keeps at least 8.5% of the causal pairs in what a
+ * gather would fetch. The dense-suffix split applies to masks (not per seed) with Structural
+ * blocks of at least 256 tokens or a local window of at least 256 keys: every key of row i
+ * from the earlier of its block start and its window start up to i is kept (Methods,
+ * "Sampling Modes": in-block pairs are cliques; the window is forced), so a first launch
+ * attends every row to that suffix on the tiles and the register gather continues that
+ * softmax over the row's other keys; the result is the same single softmax over the row's
+ * whole key set. RIS_FORCE_DESIGN = gather | tma | tile | suffix in the environment
+ * overrides (benchmarking). */
 int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim);
 
 /* Synchronise `stream` and report (then clear) the device error words: RIS_ERR_DEVICE_TIMEOUT

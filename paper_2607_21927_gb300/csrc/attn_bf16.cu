@@ -154,11 +154,12 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     const Task t = decode_task(a, tid);
     int64_t beg, n;
     key_range<DENSE>(a, t, beg, n);
-    // Structural split: the keys of the row's own block (its clique, i - b0 + 1 keys up to the
-    // row) end the ascending list and were attended by the tile kernel's clique pass
-    const bool cliques = a.clique_B > 0;
-    if (cliques) {
-        n -= t.i - (t.i / a.clique_B) * a.clique_B + 1;
+    // dense-suffix split: the row's dense suffix (its Structural block and / or local window,
+    // i - lo + 1 keys up to the row) ends the ascending list and was attended by the tile
+    // kernel's suffix pass
+    const bool split = a.part_o != nullptr;
+    if (split) {
+        n -= t.i - dense_suffix_start(a, t.i) + 1;
         if (n < 0) n = 0;
     }
     const TIdx *cols = DENSE ? nullptr : reinterpret_cast<const TIdx *>(a.col) + beg;
@@ -212,8 +213,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     for (int mt = 0; mt < MT; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
     const float sc = a.scale_log2;
-    if (cliques) {
-        // start from the clique pass's softmax: maximum = its log-sum-exp, sum 1 (on one lane
+    if (split) {
+        // start from the suffix pass's softmax: maximum = its log-sum-exp, sum 1 (on one lane
         // of the eight that share heads 2q, 2q+1), O = its normalised output, laid out as the
         // epilogue stores it
         const int hh0 = 2 * q, hh1 = 2 * q + 1;

@@ -46,6 +46,16 @@ __device__ __forceinline__ void key_range(const AttnArgs &a, const Task &t, int6
     }
 }
 
+// First key of row i's dense suffix (AttnArgs::part_o): the earlier of its Structural block
+// start and its local window start.
+__device__ __forceinline__ int64_t dense_suffix_start(const AttnArgs &a, int64_t i)
+{
+    int64_t lo = i;
+    if (a.clique_B > 0) lo = min(lo, (i / a.clique_B) * a.clique_B);
+    if (a.window > 1) lo = min(lo, max((int64_t)0, i - (int64_t)a.window + 1));
+    return lo;
+}
+
 template <bool DENSE, typename TIdx>
 __device__ __forceinline__ int key_at(const TIdx *cols, int64_t pos)
 {

@@ -34,10 +34,10 @@
 // pipe waited for them: 7.2 ms (the products alone 6.0 ms). 128-key tiles with the query in
 // TMEM beat 64-key tiles with the query in shared memory and three stages (7.8 ms).
 //
-// The clique pass of the Structural split (CLIQUE) runs the same pipeline over the key tiles
-// of each row's own Structural block only (every key of the block up to the row is kept: no
-// bitmap), and writes the normalised partial output and its log-sum-exp for the register
-// gather to continue from.
+// The suffix pass of the dense-suffix split (SUFFIX) runs the same pipeline over the key
+// tiles of each row's dense suffix only (its Structural block and / or local window: every key
+// kept, no bitmap), and writes the normalised partial output and its log-sum-exp for the
+// register gather to continue from.
 //
 // Every mbarrier wait is bounded; a wait that gives up sets bit 1 of the device error word,
 // every role falls through to the end, TMEM is released and the CTA returns.
@@ -302,7 +302,7 @@ struct TileMaps {
     CUtensorMap kh, kl, v;
 };
 
-template <bool SPLIT, bool DENSE, bool CLIQUE, typename TOut>
+template <bool SPLIT, bool DENSE, bool SUFFIX, typename TOut>
 __global__ void __launch_bounds__(kThreads, 1)
     k_attn_tile(const AttnArgs a, const __grid_constant__ TileMaps maps, const void *q_hi, const void *q_lo)
 {
@@ -326,8 +326,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int g = h / a.G;
     const int mask_id = s * a.heads_keyed + (a.heads_keyed > 1 ? g : 0);
     const int64_t last_row = (q0 + BM - 1 < a.row1 - 1) ? q0 + BM - 1 : a.row1 - 1;
-    // causal: key tiles kt0 .. last_row / BN (kt0 = 0, or the tile of the first block start)
-    const int kt0 = CLIQUE ? (int)(((q0 / a.clique_B) * a.clique_B) / BN) : 0;
+    // causal: key tiles kt0 .. last_row / BN (kt0 = 0, or the tile of the first row's dense
+    // suffix start, the earliest of the tile's rows)
+    const int kt0 = SUFFIX ? (int)(dense_suffix_start(a, q0) / BN) : 0;
     const int n_kt = (int)(last_row / BN) + 1 - kt0;
 
     if (threadIdx.x == 0) {
@@ -467,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int64_t i = q0 + r;
         const bool row_ok = i >= a.row0 && i < a.row1;
         const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
-        const uint32_t *bm = (DENSE || CLIQUE) ? nullptr
+        const uint32_t *bm = (DENSE || SUFFIX) ? nullptr
                                                : a.bitmap + (int64_t)mask_id * a.words_per_mask + (row_ok ? row_word_offset(i) : 0);
         const int64_t last_word = i >> 5;
         const float sc = a.scale_log2;
@@ -477,8 +478,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         auto mask_word = [&](int j, int e) -> uint32_t {
             if (!row_ok) return 0u;
             const int64_t k0 = (int64_t)(kt0 + j) * BN + 64 * hf + 32 * e;
-            if (CLIQUE) {  // keys of the row's block up to the row: offsets lo .. hi of the word
-                const int64_t lo = (i / a.clique_B) * a.clique_B - k0, hi = i - k0;
+            if (SUFFIX) {  // the row's dense suffix: offsets lo .. hi of the word
+                const int64_t lo = dense_suffix_start(a, i) - k0, hi = i - k0;
                 if (hi < 0 || lo > 31) return 0u;
                 uint32_t w = hi >= 31 ? 0xFFFFFFFFu : ((2u << hi) - 1u);
                 if (lo > 0) w &= ~((1u << lo) - 1u);
@@ -614,7 +615,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const float lt = l + ol;
             const float inv = lt > 0.f ? 1.f / lt : 0.f;
-            TOut *out = CLIQUE ? reinterpret_cast<TOut *>(a.part_o + ((row_ok ? i : 0) * a.Hq + h) * DT + 64 * hf)
+            TOut *out = SUFFIX ? reinterpret_cast<TOut *>(a.part_o + ((row_ok ? i : 0) * a.Hq + h) * DT + 64 * hf)
                                : reinterpret_cast<TOut *>(a.out) + (((int64_t)s * a.N + (row_ok ? i : 0)) * a.Hq + h) * DT +
                                      64 * hf;
             float ov[32];
@@ -628,7 +629,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int e = 0; e < 4; ++e) store8<TOut>(out + 32 * c4 + 8 * e, ov + 8 * e);
                 }
             }
-            if (CLIQUE) {
+            if (SUFFIX) {
                 if (row_ok && hf == 0) a.part_lse[i * a.Hq + h] = m_used + __log2f(lt);
             } else if (row_ok && hf == 0 && a.lse != nullptr) {
                 a.lse[((int64_t)s * a.Hq + h) * a.N + i] = (m_used + __log2f(lt)) * kLn2;
@@ -673,10 +674,10 @@ bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows)
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool SPLIT, bool DENSE, typename TOut, bool CLIQUE = false>
+template <bool SPLIT, bool DENSE, typename TOut, bool SUFFIX = false>
 cudaError_t launch_t(const AttnArgs &a, const TileMaps &maps, const void *q_hi, const void *q_lo, cudaStream_t s)
 {
-    auto kern = k_attn_tile<SPLIT, DENSE, CLIQUE, TOut>;
+    auto kern = k_attn_tile<SPLIT, DENSE, SUFFIX, TOut>;
     static bool attr = false;
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
@@ -732,11 +733,11 @@ cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const voi
     return dense ? launch_t<false, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s) : launch_t<false, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
 }
 
-cudaError_t launch_attention_tile_cliques(const AttnArgs &a, const void *q_hi, const void *q_lo, cudaStream_t s)
+cudaError_t launch_attention_tile_suffix(const AttnArgs &a, const void *q_hi, const void *q_lo, cudaStream_t s)
 {
     static std::mutex mu;
     std::lock_guard<std::mutex> lk(mu);
-    if (a.clique_B < 1 || a.part_o == nullptr || a.part_lse == nullptr || a.n_sets != 1) return cudaErrorInvalidValue;
+    if (a.part_o == nullptr || a.part_lse == nullptr || a.n_sets != 1) return cudaErrorInvalidValue;
     const bool split = q_lo != nullptr;
     alignas(64) TileMaps maps;
     if (!make_maps(maps, a, split)) return cudaErrorInvalidValue;

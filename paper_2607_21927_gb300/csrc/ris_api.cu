@@ -35,7 +35,9 @@ using namespace ris;
 
 struct ris_mask_s {
     int64_t N = 0;
-    int32_t mode = 0;  // ris_mode of the call that built it
+    int32_t mode = 0;    // ris_mode of the call that built it
+    int32_t window = 1;  // forced local window
+    int64_t suffix_pairs = 0;  // pairs in the rows' dense suffixes (dense-suffix split), per mask
     int32_t n_masks = 0, heads_keyed = 1, kv_heads = 1, n_seeds = 0, per_seed = 0;
     int32_t col_bytes = 2, dense = 0;
     int64_t n_pairs = 0, words_per_mask = 0;
@@ -152,7 +154,7 @@ std::pair<cudaEvent_t, cudaEvent_t> timer_pair()
 
 // Kernel design override for benchmarking the designs against each other:
 // RIS_FORCE_DESIGN = gather (register gather), tma (TMA gather), tile (masked dense tiles) or
-// cliques (the Structural split, where the mask allows it).
+// suffix (the dense-suffix split, where the mask allows it).
 const char *forced_design()
 {
     static const std::string d = [] {
@@ -169,14 +171,48 @@ const char *forced_design()
 // layers: 8.6% of the causal pairs at N = 32768 and 8.4% at N = 65536.
 constexpr double kTileDensity = 0.085;
 
-// Smallest Structural block for which the cliques go to the tile kernel (a block then fills
-// at least two 128 x 128 tiles' worth of pairs).
-constexpr int64_t kCliqueMinBlock = 256;
+// Shortest dense span (Structural block or local window) for which the split pays: two
+// 128-key tiles.
+constexpr int64_t kSuffixMin = 256;
+
+// Dense suffix of row i: every key in [lo(i), i] is kept, where lo(i) is the start of the
+// row's own Structural block (a causal clique; blocks shorter than kSuffixMin are not used)
+// and / or of its forced local window, whichever reaches further back. Those keys end the
+// row's ascending key list.
+int64_t suffix_block(const ris_mask_s *m)
+{
+    return (m->mode == RIS_MODE_STRUCTURAL && m->params.block >= kSuffixMin) ? m->params.block : 0;
+}
+
+bool suffix_split_allowed(const ris_mask_s *m)
+{
+    return !m->dense && !m->per_seed && (suffix_block(m) > 0 || m->window >= kSuffixMin);
+}
+
+// sum of x over a <= x < b
+int64_t range_sum(int64_t a, int64_t b) { return b > a ? (a + b - 1) * (b - a) / 2 : 0; }
+
+// Pairs in all rows' dense suffixes: the suffix of row i holds i - lo(i) + 1 keys, which is
+// min(i + 1, W) without blocks, and with blocks i + 1 for i < W, else max(W, i - b0 + 1).
+int64_t suffix_pairs_of(int64_t N, int64_t block, int64_t W)
+{
+    if (W < 1) W = 1;
+    if (block <= 0) return N <= W ? range_sum(1, N + 1) : range_sum(1, W + 1) + (N - W) * W;
+    int64_t total = 0;
+    for (int64_t b0 = 0; b0 < N; b0 += block) {
+        const int64_t b1 = std::min(N, b0 + block);
+        total += range_sum(b0 + 1, std::min(b1, W) + 1);                  // i < W: i + 1 keys
+        const int64_t s = std::max(b0, W);                                // i >= W:
+        total += std::max<int64_t>(0, std::min(b1, b0 + W) - s) * W;     //   i - b0 < W: W keys
+        total += range_sum(W + 1, b1 - b0 + 1);                           //   else i - b0 + 1 keys
+    }
+    return total;
+}
 
 // Design of a layer call: 0 register gather, 1 TMA gather, 2 masked dense tiles, 3 fp32
-// gather, 4 Structural split (the in-block cliques on the tile kernel, the remaining keys on
+// gather, 4 dense-suffix split (each row's dense suffix on the tile kernel, its other keys on
 // the register gather, one softmax). The gather's cost grows with the pairs it gathers (with
-// the split: all but the cliques), a tile's does not, hence the density threshold.
+// the split: all but the suffixes), a tile's does not, hence the density threshold.
 int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim)
 {
     if (dtype == RIS_F32) return 3;
@@ -185,11 +221,11 @@ int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim)
     if (f == "gather") return 0;
     const bool tiles = head_dim == 128 && tile_design_available();
     if (tiles && (f == "tile" || m->dense)) return 2;
-    const bool split = tiles && m->mode == RIS_MODE_STRUCTURAL && !m->per_seed && m->params.block >= kCliqueMinBlock;
-    if (split && f == "cliques") return 4;
+    const bool split = tiles && suffix_split_allowed(m);
+    if (split && f == "suffix") return 4;
     if (tiles) {
         const double causal = (double)m->n_masks * ((double)m->N * (double)(m->N + 1) / 2.0);
-        const double gathered = (double)m->n_pairs - (split ? (double)m->n_masks * (double)m->params.clique_pairs : 0.0);
+        const double gathered = (double)m->n_pairs - (split ? (double)m->n_masks * (double)m->suffix_pairs : 0.0);
         if (gathered >= kTileDensity * causal) return 2;
     }
     return split ? 4 : 0;
@@ -415,8 +451,10 @@ ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double d
     mk->per_seed = per_seed;
     mk->col_bytes = N <= 65536 ? 2 : 4;
     mk->mode = mode;
+    mk->window = o.local_window;
     mk->params = p;
     mk->stream = s;
+    mk->suffix_pairs = suffix_pairs_of(N, suffix_block(mk), o.local_window);
     if (p.dense) {
         mk->dense = 1;
         mk->n_pairs = n_masks * (N * (N + 1) / 2);
@@ -509,6 +547,7 @@ ris_status ris_mask_info(ris_mask_t m, ris_mask_desc *out)
     d.col = m->col;
     d.bitmap = m->bitmap;
     d.params = m->params;
+    d.suffix_pairs = suffix_split_allowed(m) ? m->suffix_pairs : 0;
     *out = d;
     return RIS_OK;
 }
@@ -566,8 +605,8 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     if (row1 < 0) row1 = N;
     prepare_pool_once();
     const int design = design_of(m, dtype, head_dim);
-    const bool tile = design == 2, cliques = design == 4;
-    const bool q_pair = tile || cliques;  // queries as a bf16 hi + lo pair
+    const bool tile = design == 2, suffix = design == 4;
+    const bool q_pair = tile || suffix;  // queries as a bf16 hi + lo pair
     Scratch qt, qtl, kt, ktl, po, pl;
     const void *qu = q, *ku = k, *kl = nullptr, *q_lo = nullptr;
     bool q_split = false;
@@ -628,10 +667,11 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.row0 = row0;
     a.row1 = row1;
     a.n_tasks = (int64_t)a.n_sets * (row1 - row0) * kv_heads;
-    if (cliques) {
+    if (suffix) {
         RIS_CUDA(po.alloc((size_t)N * heads * head_dim * sizeof(float), s));
         RIS_CUDA(pl.alloc((size_t)N * heads * sizeof(float), s));
-        a.clique_B = m->params.block;
+        a.clique_B = suffix_block(m);
+        a.window = m->window;
         a.part_o = (float *)po.p;
         a.part_lse = (float *)pl.p;
     }
@@ -639,8 +679,8 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     if (ev.first) RIS_CUDA(cudaEventRecord(ev.first, s));
     if (tile) {
         RIS_CUDA(launch_attention_tile(a, qu, q_lo, out_dtype, m->dense != 0, s));
-    } else if (cliques) {  // the cliques on the tiles, then the gather continues their softmax
-        RIS_CUDA(launch_attention_tile_cliques(a, qu, a.q_lo, s));
+    } else if (suffix) {  // the dense suffixes on the tiles, then the gather continues their softmax
+        RIS_CUDA(launch_attention_tile_suffix(a, qu, a.q_lo, s));
         RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, false, s));
     } else if (design == 1)
         RIS_CUDA(launch_attention_tma(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));

@@ -88,15 +88,16 @@ struct AttnArgs {
     int32_t n_sets;        // output sets: n_seeds for per-seed masks, else 1
     int64_t row0;          // query rows row0 .. row1-1 are computed (0 and N for a whole layer)
     int64_t row1;
-    // Structural cliques on the tiles (0: off): rows are split into blocks of clique_B tokens,
-    // and every key of a row's own block up to the row is kept. The tile kernel's clique pass
-    // attends each row to those keys only and writes part_o / part_lse; the register gather
-    // then starts from that partial softmax and skips the same keys, which are the tail of the
-    // row's ascending key list.
+    // Dense-suffix split (part_o set): every key in [lo(i), i] of row i is kept, lo(i) being
+    // the start of the row's Structural block of clique_B tokens (0: no blocks) and / or of its
+    // forced local window of `window` keys, whichever reaches further back. The tile kernel's
+    // suffix pass attends each row to those keys only and writes part_o / part_lse; the
+    // register gather then starts from that partial softmax and skips the same keys, which
+    // are the tail of the row's ascending key list.
     int64_t clique_B;
-    float *part_o;         // [N][Hq][D] normalised partial outputs
+    float *part_o;         // [N][Hq][D] normalised partial outputs, or null
     float *part_lse;       // [N][Hq] their log2-domain log-sum-exp
-    int32_t pad_;
+    int32_t window;
     float scale_log2;      // log2(e) / sqrt(D)
     int64_t n_tasks;       // n_sets * (row1 - row0) * Hkv
 };
@@ -181,8 +182,8 @@ cudaError_t read_device_error(unsigned int *out, cudaStream_t s);
 bool tile_design_available();
 cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const void *q_lo, int out_dtype, bool dense,
                                   cudaStream_t s);
-// The clique pass of the Structural split (a.clique_B > 0): writes a.part_o / a.part_lse.
-cudaError_t launch_attention_tile_cliques(const AttnArgs &a, const void *q_hi, const void *q_lo, cudaStream_t s);
+// The suffix pass of the dense-suffix split (a.part_o set): writes a.part_o / a.part_lse.
+cudaError_t launch_attention_tile_suffix(const AttnArgs &a, const void *q_hi, const void *q_lo, cudaStream_t s);
 cudaError_t read_tile_error(unsigned int *out);
 
 }  // namespace ris

@@ -53,7 +53,7 @@ class MaskDesc(ctypes.Structure):
                 ("n_seeds", ctypes.c_int32), ("per_seed", ctypes.c_int32), ("col_bytes", ctypes.c_int32),
                 ("dense", ctypes.c_int32), ("n_pairs", ctypes.c_int64), ("words_per_mask", ctypes.c_int64),
                 ("row_ptr", ctypes.c_void_p), ("col", ctypes.c_void_p), ("bitmap", ctypes.c_void_p),
-                ("params", Params)]
+                ("params", Params), ("suffix_pairs", ctypes.c_int64)]
 
 
 def rope_cfg(kind: int = ROPE_PLAIN, theta: float = 1e6, native_len: int = 32768, factor: float = 0.0,
@@ -155,7 +155,7 @@ def ris_version() -> str:
 
 
 DESIGNS = {0: "register gather", 1: "TMA gather", 2: "tcgen05 masked tiles", 3: "fp32 gather",
-           4: "cliques on tiles + register gather"}
+           4: "dense suffix on tiles + register gather"}
 
 
 def ris_attention_design(mask: "Mask", dtype=torch.bfloat16, head_dim: int = 128) -> int:

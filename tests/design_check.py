@@ -22,7 +22,7 @@ CASES = [
     (400, 6, 2, 128, 0, 0.3, [4, 5, 6], (3, 1e6, 256), True),
     (3, 6, 2, 128, 0, 0.5, [1], (3, 1e6, 64), False),
     (1, 2, 1, 64, 1, 0.5, [2], None, False),
-    # Structural blocks of 300 and 260 tokens: the split (cliques on the tiles) where allowed
+    # Structural blocks of 300 and 260 tokens: the dense-suffix split (blocks on the tiles) where allowed
     (3000, 6, 2, 128, 1, 0.1, [1], (3, 1e6, 256), False),
     (2600, 4, 1, 128, 1, 0.12, [3], None, False),
 ]

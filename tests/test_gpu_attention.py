@@ -296,8 +296,9 @@ def test_row_ranges_reassemble_the_layer(d, S, D):
 
 
 def test_structural_split_design_choice():
-    """C5's Structural mask (blocks of 655) takes the split: cliques on the tiles, the rest
-    gathered; Structural masks with small blocks, per-seed masks and head_dim 64 do not."""
+    """C5's Structural mask (blocks of 655) takes the dense-suffix split: cliques on the tiles,
+    the rest gathered; Structural masks with small blocks and no wide window, per-seed masks
+    and head_dim 64 do not; a Stochastic mask with a 1024-key window does."""
     m = ris.ris_mask_generate(65536, 2, 1, 0.01, list(range(10)))
     assert ris.ris_attention_design(m, torch.bfloat16, 128) == 4
     assert ris.ris_attention_design(m, torch.bfloat16, 64) == 0
@@ -308,20 +309,26 @@ def test_structural_split_design_choice():
     m = ris.ris_mask_generate(65536, 2, 1, 0.01, list(range(10)), per_seed=True)
     assert ris.ris_attention_design(m, torch.bfloat16, 128) != 4
     m.free()
+    m = ris.ris_mask_generate(65536, 2, 0, 0.005, list(range(4)), opts=ris.paper_geometry())
+    assert ris.ris_attention_design(m, torch.bfloat16, 128) == 4
+    m.free()
 
 
-@pytest.mark.parametrize("N,d,S,kind,window,anchors", [(3000, 0.1, 1, 3, 1, 0), (2700, 0.11, 1, 0, 1, 0),
-                                                     (4100, 0.08, 1, 3, 40, 3)],
-                         ids=["yarn", "pre_rotated", "window_anchors"])
-def test_structural_split_full(N, d, S, kind, window, anchors):
-    """The Structural split (blocks of >= 256 tokens) against the oracle on every row: fp32 and
-    bf16 outputs and the log-sum-exp, with and without RoPE, with a local window and anchors
-    reaching outside the block."""
+@pytest.mark.parametrize("N,mode,d,S,kind,window,anchors", [
+    (3000, 1, 0.1, 1, 3, 1, 0), (2700, 1, 0.11, 1, 0, 1, 0), (4100, 1, 0.08, 1, 3, 40, 3),
+    (3300, 1, 0.1, 1, 3, 700, 2), (2900, 0, 0.01, 2, 3, 300, 4), (1500, 1, 0.002, 1, 3, 600, 0)],
+    ids=["blocks", "blocks_pre_rotated", "blocks_small_window_anchors", "blocks_in_wider_window",
+         "stochastic_window", "structural_small_blocks_window"])
+def test_dense_suffix_split_full(N, mode, d, S, kind, window, anchors):
+    """The dense-suffix split (Structural blocks of >= 256 tokens and / or a local window of
+    >= 256 keys on the tiles, the other keys gathered) against the oracle on every row: fp32
+    and bf16 outputs and the log-sum-exp, with and without RoPE, with anchors and with windows
+    shorter and longer than the blocks."""
     Hq, Hkv, D = 12, 2, 128
     (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=N, outliers=True)
     seeds = list(range(5, 5 + S))
     opts = ris.mask_opts(local_window=window, n_anchor=anchors)
-    m = ris.ris_mask_generate(N, Hkv, 1, d, seeds, opts=opts)
+    m = ris.ris_mask_generate(N, Hkv, mode, d, seeds, opts=opts)
     assert ris.ris_attention_design(m, torch.bfloat16, D) == 4
     rope = ris.rope_cfg(kind, 1e6, 256) if kind else None
     out32, lse = ris.ris_attention_masked(m, q, k, v, rope=rope, out_dtype=torch.float32, return_lse=True)
@@ -329,14 +336,14 @@ def test_structural_split_full(N, d, S, kind, window, anchors):
     torch.cuda.synchronize()
     ris.ris_device_status()
     m.free()
-    ref, ref_lse = run_oracle(qn, kn, vn, 1, d, seeds, kind, 1e6, 256, W=window, A=anchors)
+    ref, ref_lse = run_oracle(qn, kn, vn, mode, d, seeds, kind, 1e6, 256, W=window, A=anchors)
     check_bf16_path(to_np(out32), ref)
     check_bf16_path(to_np(out16), ref, out_bf16=True)
     np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
 
 
 def test_structural_split_row_ranges():
-    """Row ranges through the Structural split reassemble the whole layer bit for bit."""
+    """Row ranges through the dense-suffix split reassemble the whole layer bit for bit."""
     N, Hq, Hkv, D = 3000, 6, 2, 128
     (q, k, v), _ = make_inputs(N, Hq, Hkv, D, seed=29, outliers=True)
     m = ris.ris_mask_generate(N, Hkv, 1, 0.1, [4])
