@@ -184,3 +184,11 @@ def test_decode_device_position_and_graph_replay():
         ris.ris_device_status()
     ris.ris_device_status()  # the report cleared the flag
     an.free()
+
+
+def test_decode_long_anchor_fold_beyond_shared_memory():
+    """An anchor list long enough (about 42k keys, 167 cluster partials x 8 heads) that the
+    final fold takes its fallback path (more partials than the shared memory holds)."""
+    N = 65536
+    _decode_case(N, N + 4, 16, 2, 64, torch.bfloat16, 0, 0.1, list(range(10)), [N, N + 3], 256, native=32768,
+                 theta=1e6, out_dtype=torch.float32, seed=8)
