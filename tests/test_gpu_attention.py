@@ -357,3 +357,36 @@ def test_structural_split_row_ranges():
     torch.cuda.synchronize()
     assert torch.equal(parts, whole)
     m.free()
+
+
+def test_dense_suffix_split_per_head_masks():
+    """Per-head masks (keyed per KV head) take the dense-suffix split too: each KV head
+    gathers from its own key lists after the shared suffix pass."""
+    N, Hq, Hkv, D = 2800, 6, 2, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=31, outliers=True)
+    opts = ris.mask_opts(per_head=True, local_window=300)
+    m = ris.ris_mask_generate(N, Hkv, 1, 0.1, [2], opts=opts)
+    assert ris.ris_attention_design(m, torch.bfloat16, D) == 4
+    out = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e6, 256), out_dtype=torch.float32)
+    torch.cuda.synchronize()
+    m.free()
+    G = Hq // Hkv
+    for g in range(Hkv):
+        spec = ora.MaskSpec(N=N, mode=1, density=0.1, seeds=[2], local_window=300, head_key=g)
+        ref, _, _, _ = ora.sparse_attention(qn[:, g * G:(g + 1) * G], kn[:, g:g + 1], vn[:, g:g + 1], spec,
+                                            oracle_rope(3, 1e6, 256))
+        check_bf16_path(to_np(out[:, g * G:(g + 1) * G]), ref)
+
+
+def test_dense_suffix_split_u32_keys_beyond_65536():
+    """N > 65536 (32-bit key lists) with Structural blocks of 656 tokens: the split on sampled rows."""
+    N, Hq, Hkv, D = 65600, 2, 1, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=19, outliers=True)
+    m = ris.ris_mask_generate(N, Hkv, 1, 0.01, [1, 2])
+    assert ris.ris_attention_design(m, torch.bfloat16, D) == 4
+    out = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e6, 32768), out_dtype=torch.float32)
+    torch.cuda.synchronize()
+    m.free()
+    rows = sample_rows(N, 24, seed=7)
+    ref, _ = run_oracle(qn, kn, vn, 1, 0.01, [1, 2], 3, 1e6, 32768, rows=rows)
+    check_bf16_path(to_np(out[rows]), ref)
