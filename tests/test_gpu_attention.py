@@ -390,3 +390,23 @@ def test_dense_suffix_split_u32_keys_beyond_65536():
     rows = sample_rows(N, 24, seed=7)
     ref, _ = run_oracle(qn, kn, vn, 1, 0.01, [1, 2], 3, 1e6, 32768, rows=rows)
     check_bf16_path(to_np(out[rows]), ref)
+
+
+@pytest.mark.parametrize("mode,d,S", [(0, 0.01, 4), (1, 0.01, 2), (0, 0.01, 12)], ids=["stochastic_gather", "structural_split", "stochastic_tiles"])
+def test_quarter_million_tokens_sampled(mode, d, S):
+    """N = 262144 (bitmap of 4.3 GB, byte offsets past 2^32, 32-bit key lists; 256 K keys per
+    row at most): sampled rows of the gather, the dense-suffix split and the tile design."""
+    N, Hq, Hkv, D = 262144, 2, 1, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=41, outliers=True)
+    seeds = list(range(S))
+    m = ris.ris_mask_generate(N, Hkv, mode, d, seeds)
+    design = ris.ris_attention_design(m, torch.bfloat16, D)
+    assert design == {"stochastic_gather": 0, "structural_split": 4, "stochastic_tiles": 2}[
+        {(0, 4): "stochastic_gather", (1, 2): "structural_split", (0, 12): "stochastic_tiles"}[(mode, S)]]
+    out = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e6, 32768), out_dtype=torch.float32)
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    m.free()
+    rows = sample_rows(N, 12, seed=3)
+    ref, _ = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e6, 32768, rows=rows)
+    check_bf16_path(to_np(out[rows]), ref)
