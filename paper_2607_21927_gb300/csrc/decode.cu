@@ -26,6 +26,7 @@
 // so it runs on the FP32 pipes (no tensor-core tile to fill) and is bound by the K/V row
 // reads; fp32 scores and probabilities keep it well inside the bf16 tolerance.
 #include <cooperative_groups.h>
+#include <utility>
 #include <cuda_bf16.h>
 
 #include <cmath>
@@ -122,6 +123,12 @@ __global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecode
     int32_t spec = -1;
     if (from_anchor && tid < kDecodeChunk && k0 + tid < a.anchor_len[m])
         spec = __ldg(a.anchor + a.anchor_base[m] + k0 + tid);
+    // Launched as a programmatic dependent of the kernel before it (the previous step's
+    // combine): everything above only reads the anchor list, built before the first step.
+    // Wait for that kernel (the position, q and the partials' buffer come after it), then let
+    // the next kernel be scheduled while this one runs.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int64_t t = a.t_dev != nullptr ? *a.t_dev : a.t;
     const bool valid = t >= a.t0 && t < a.cache_len;  // only a device-side t can be outside
     if (!valid && tid == 0 && chunk == 0 && g == 0) atomicOr(&g_ris_decode_error, 2u);
@@ -286,6 +293,9 @@ constexpr int kCombineWarps = 8;
 template <typename TO>
 __global__ void __launch_bounds__(kCombineWarps * 32) k_decode_combine(const DecodeArgs a)
 {
+    // a programmatic dependent of the partial kernel: wait for its partials
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     __shared__ float wm[kCombineWarps], wl[kCombineWarps], wacc[kCombineWarps][32];
     const int h = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int c = blockIdx.y * 32 + lane;
@@ -343,31 +353,44 @@ unsigned int read_decode_error()
     return v;
 }
 
-template <int D>
-void launch_partial(const DecodeArgs &a, int dtype, dim3 grid, cudaStream_t s)
+// Launch as a programmatic dependent of the previous kernel in the stream: it may be scheduled
+// while that kernel runs and waits for it (griddepcontrol.wait) before touching its results.
+template <typename... P, typename... A>
+cudaError_t launch_pdl(void (*kern)(P...), dim3 grid, dim3 block, cudaStream_t s, A &&...args)
 {
-    if (dtype == RIS_F32)
-        k_decode_partial<float, false, D><<<grid, kDecodeThreads, 0, s>>>(a);
-    else if (a.k_lo != nullptr)
-        k_decode_partial<__nv_bfloat16, true, D><<<grid, kDecodeThreads, 0, s>>>(a);
-    else
-        k_decode_partial<__nv_bfloat16, false, D><<<grid, kDecodeThreads, 0, s>>>(a);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<A>(args)...);
+}
+
+template <int D>
+cudaError_t launch_partial(const DecodeArgs &a, int dtype, dim3 grid, cudaStream_t s)
+{
+    if (dtype == RIS_F32) return launch_pdl(k_decode_partial<float, false, D>, grid, dim3(kDecodeThreads), s, a);
+    if (a.k_lo != nullptr)
+        return launch_pdl(k_decode_partial<__nv_bfloat16, true, D>, grid, dim3(kDecodeThreads), s, a);
+    return launch_pdl(k_decode_partial<__nv_bfloat16, false, D>, grid, dim3(kDecodeThreads), s, a);
 }
 
 cudaError_t launch_decode(const DecodeArgs &a, int dtype, int out_dtype, cudaStream_t s)
 {
     // n_chunks is a multiple of the cluster size (the host rounds it up)
     const dim3 grid_p((unsigned)a.n_chunks, (unsigned)a.Hkv);
-    if (a.D == 128)
-        launch_partial<128>(a, dtype, grid_p, s);
-    else
-        launch_partial<64>(a, dtype, grid_p, s);
+    cudaError_t e = a.D == 128 ? launch_partial<128>(a, dtype, grid_p, s) : launch_partial<64>(a, dtype, grid_p, s);
+    if (e != cudaSuccess) return e;
     const dim3 grid_c((unsigned)a.Hq, (unsigned)(a.D / 32));
-    if (out_dtype == RIS_F32)
-        k_decode_combine<float><<<grid_c, kCombineWarps * 32, 0, s>>>(a);
-    else
-        k_decode_combine<__nv_bfloat16><<<grid_c, kCombineWarps * 32, 0, s>>>(a);
+    e = out_dtype == RIS_F32 ? launch_pdl(k_decode_combine<float>, grid_c, dim3(kCombineWarps * 32), s, a)
+                             : launch_pdl(k_decode_combine<__nv_bfloat16>, grid_c, dim3(kCombineWarps * 32), s, a);
     note_launch(2);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
