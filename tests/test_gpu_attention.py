@@ -316,9 +316,11 @@ def test_structural_split_design_choice():
 
 @pytest.mark.parametrize("N,mode,d,S,kind,window,anchors", [
     (3000, 1, 0.1, 1, 3, 1, 0), (2700, 1, 0.11, 1, 0, 1, 0), (4100, 1, 0.08, 1, 3, 40, 3),
-    (3300, 1, 0.1, 1, 3, 700, 2), (2900, 0, 0.01, 2, 3, 300, 4), (1500, 1, 0.002, 1, 3, 600, 0)],
+    (3300, 1, 0.1, 1, 3, 700, 2), (2900, 0, 0.01, 2, 3, 300, 4), (1500, 1, 0.002, 1, 3, 600, 0),
+    (2560, 1, 0.1, 1, 3, 1, 0), (1000, 0, 0.02, 1, 3, 256, 0), (700, 0, 0.02, 1, 0, 900, 0)],
     ids=["blocks", "blocks_pre_rotated", "blocks_small_window_anchors", "blocks_in_wider_window",
-         "stochastic_window", "structural_small_blocks_window"])
+         "stochastic_window", "structural_small_blocks_window", "blocks_of_exactly_256",
+         "window_of_exactly_256", "window_longer_than_the_sequence"])
 def test_dense_suffix_split_full(N, mode, d, S, kind, window, anchors):
     """The dense-suffix split (Structural blocks of >= 256 tokens and / or a local window of
     >= 256 keys on the tiles, the other keys gathered) against the oracle on every row: fp32
