@@ -138,7 +138,11 @@ constexpr float kLazyLog2 = 8.f;  // rescale O only when the row maximum grows b
 // D: head dim (64 or 128). QSPLIT: q is fp32 (split hi + lo); else q is bf16.
 // KSPLIT: keys come as a bf16 hi (a.k) + lo (a.k_lo) pair. WIDE: 32-byte loads (K, K lo and
 // V pointers 32-byte aligned).
-template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut>
+// SEEDS (per-seed masks, n_sets > 1): a warp owns (row i, KV head g) and walks the sets one
+// after the other, requesting the next set's key range and first keys while the current set
+// runs and its first K/V rows during the current set's last group, so the load pipeline
+// never drains between sets; a.n_tasks counts (row, KV head) pairs.
+template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut, bool SEEDS>
 __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
 {
     constexpr int KSTEPS = D / 16;  // k-steps of the score product
@@ -151,7 +155,15 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     const int64_t tid = (int64_t)blockIdx.x * kAttnWarps + (threadIdx.x >> 5);
     if (tid >= a.n_tasks) return;
     const int p = lane >> 2, q = lane & 3;
-    const Task t = decode_task(a, tid);
+    Task t;
+    if (SEEDS) {
+        t.g = (int)(tid % a.Hkv);
+        t.i = a.row1 - 1 - tid / a.Hkv;
+        t.s = 0;
+        t.mask_id = a.heads_keyed > 1 ? t.g : 0;
+    } else {
+        t = decode_task(a, tid);
+    }
     int64_t beg, n;
     key_range<DENSE>(a, t, beg, n);
     // dense-suffix split: the row's dense suffix (its Structural block and / or local window,
@@ -163,6 +175,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         if (n < 0) n = 0;
     }
     const TIdx *cols = DENSE ? nullptr : reinterpret_cast<const TIdx *>(a.col) + beg;
+    int64_t set_n = n;  // keys of the current set (SEEDS: reloaded per set)
 
     // ---- query fragments (B operand of the score product), head p of this KV group
     uint32_t qh[KSTEPS][2], ql[KSTEPS][2];
@@ -243,13 +256,14 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     // ---- key indices, prefetched 64 keys (4 groups) ahead: lane holds positions
     //      64c + lane and 64c + 32 + lane of chunk c; slots past the row read the row itself
     int cur[2], nxt[2];
-    auto load_chunk = [&](int64_t cbase, int (&dst)[2]) {
+    auto load_chunk_at = [&](const TIdx *cl, int64_t nk, int64_t cbase, int (&dst)[2]) {
 #pragma unroll
         for (int w = 0; w < 2; ++w) {
             const int64_t pos = cbase + 32 * w + lane;
-            dst[w] = pos < n ? key_at<DENSE, TIdx>(cols, pos) : (int)t.i;
+            dst[w] = pos < nk ? key_at<DENSE, TIdx>(cl, pos) : (int)t.i;
         }
     };
+    auto load_chunk = [&](int64_t cbase, int (&dst)[2]) { load_chunk_at(cols, set_n, cbase, dst); };
     load_chunk(0, cur);
     load_chunk(64, nxt);
     // index of slot r (0..15) of group slot gs (0..3) of a chunk held in (c0, c1)
@@ -290,11 +304,28 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     // scores are formed, its V rows as soon as this group's values are accumulated.
     issue_k(cur[0], cur[1], 0);
     issue_v(cur[0], cur[1], 0);
+    const int n_sets = SEEDS ? a.n_sets : 1;
+    for (int set = 0; set < n_sets; ++set) {
+    // SEEDS: the next set's key range and first 64 keys, requested now
+    const TIdx *ncols = cols;
+    int64_t nn = 0;
+    int ncur[2] = {0, 0};
+    if (SEEDS && set + 1 < n_sets) {
+        Task tn = t;
+        tn.s = set + 1;
+        tn.mask_id = tn.s * a.heads_keyed + (a.heads_keyed > 1 ? t.g : 0);
+        int64_t nbeg;
+        key_range<DENSE>(a, tn, nbeg, nn);
+        ncols = DENSE ? nullptr : reinterpret_cast<const TIdx *>(a.col) + nbeg;
+        load_chunk_at(ncols, nn, 0, ncur);
+    }
+    n = set_n;
     const int64_t ngroups = (n + 15) / 16;
     for (int64_t g = 0; g < ngroups; ++g) {
         const int64_t base = 16 * g;
         const int gs = (int)(g & 3), gs1 = (gs + 1) & 3;
         const bool more = g + 1 < ngroups;
+        const bool cross = SEEDS && !more && set + 1 < n_sets;  // the next set's first group
         const int n0 = gs1 == 0 ? nxt[0] : cur[0], n1 = gs1 == 0 ? nxt[1] : cur[1];
         const bool val0 = base + p < n, val1 = base + p + 8 < n;
 
@@ -319,7 +350,10 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         float s[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) s[e] = ((sa[0][e] + sa[1][e]) + (sb[0][e] + sb[1][e])) + (sl[0][e] + sl[1][e]);
-        if (more) issue_k(n0, n1, gs1);
+        if (more)
+            issue_k(n0, n1, gs1);
+        else if (cross)
+            issue_k(ncur[0], ncur[1], 0);
 
         // ---- online softmax; lane holds keys p, p+8 x heads 2q, 2q+1
         float s0 = val0 ? s[0] * sc : -INFINITY, s1 = val0 ? s[1] * sc : -INFINITY;
@@ -372,7 +406,10 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
             mma16816(o[mt], a0, a1, a2, a3, pb0, pb1);
             mma16816(o[mt], a0, a1, a2, a3, pl0, pl1);
         }
-        if (more) issue_v(n0, n1, gs1);
+        if (more)
+            issue_v(n0, n1, gs1);
+        else if (cross)
+            issue_v(ncur[0], ncur[1], 0);
         if (gs == 3) {  // the next group starts the prefetched chunk; fetch the one after it
             cur[0] = nxt[0];
             cur[1] = nxt[1];
@@ -417,6 +454,21 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         if (h0 < a.G) lse[(int64_t)h0 * a.N] = (m0 + __log2f(l0)) * kLn2;
         if (h1 < a.G) lse[(int64_t)h1 * a.N] = (m1 + __log2f(l1)) * kLn2;
     }
+    if (SEEDS && set + 1 < n_sets) {
+        // on to the next set: its first group's rows are in flight
+        t.s = set + 1;
+        t.mask_id = t.s * a.heads_keyed + (a.heads_keyed > 1 ? t.g : 0);
+        cols = ncols;
+        set_n = nn;
+        cur[0] = ncur[0];
+        cur[1] = ncur[1];
+        load_chunk(64, nxt);
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+        m0 = m1 = -INFINITY;
+        l0 = l1 = 0.f;
+    }
+    }  // sets
 }
 
 template <int D, bool QSPLIT, bool WIDE, typename TOut>
@@ -424,14 +476,25 @@ cudaError_t launch_w(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t 
 {
     // rotated inputs: fp32 queries and hi + lo keys; as given: bf16 queries and keys
     constexpr bool KSPLIT = QSPLIT;
-    const unsigned grid = (unsigned)((a.n_tasks + kAttnWarps - 1) / kAttnWarps);
     const dim3 block(kAttnWarps * 32);
+    if (!dense && a.n_sets > 1) {  // per-seed sets: one warp per (row, KV head) walks them all
+        AttnArgs b = a;
+        b.n_tasks = (a.row1 - a.row0) * a.Hkv;
+        const unsigned grid = (unsigned)((b.n_tasks + kAttnWarps - 1) / kAttnWarps);
+        if (col_bytes == 2)
+            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, true><<<grid, block, 0, s>>>(b);
+        else
+            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, true><<<grid, block, 0, s>>>(b);
+        note_launch();
+        return cudaGetLastError();
+    }
+    const unsigned grid = (unsigned)((a.n_tasks + kAttnWarps - 1) / kAttnWarps);
     if (dense)
-        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, true, TOut><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, true, TOut, false><<<grid, block, 0, s>>>(a);
     else if (col_bytes == 2)
-        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, false><<<grid, block, 0, s>>>(a);
     else
-        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, false><<<grid, block, 0, s>>>(a);
     note_launch();
     return cudaGetLastError();
 }
