@@ -2,7 +2,8 @@
 // Pre-Fusion Unified Softmax (PFUS)": one softmax over each row's whole sampled key set).
 //
 // One warp owns one task (row i, KV head g, output set s) and walks the row's ascending key
-// list 16 keys at a time. The G query heads that share KV head g (GQA) ride in the N
+// list 16 keys at a time (per-seed outputs: one warp walks the sets of (i, g) one after the
+// other, see SEEDS below). The G query heads that share KV head g (GQA) ride in the N
 // dimension of the tensor-core tile, so every gathered K/V row is fetched once and used by
 // all of them:
 //
