@@ -412,3 +412,24 @@ def test_quarter_million_tokens_sampled(mode, d, S):
     rows = sample_rows(N, 12, seed=3)
     ref, _ = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e6, 32768, rows=rows)
     check_bf16_path(to_np(out[rows]), ref)
+
+
+def test_row_ranges_per_seed_sets():
+    """Row ranges of a per-seed mask (one output set per seed, walked by the gather's set loop)
+    reassemble the whole per-seed output bit for bit."""
+    N, Hq, Hkv, D, seeds = 1400, 6, 2, 128, [3, 4, 5]
+    (q, k, v), _ = make_inputs(N, Hq, Hkv, D, seed=37, outliers=True)
+    m = ris.ris_mask_generate(N, Hkv, 0, 0.03, seeds, per_seed=True)
+    assert ris.ris_attention_design(m, torch.bfloat16, D) == 0
+    rope = ris.rope_cfg(3, 1e6, 256)
+    whole = torch.empty(len(seeds), N, Hq, D, dtype=torch.float32, device="cuda")
+    ris.ris_attention_masked_rows(m, 0, N, q, k, v, whole, rope=rope)
+    parts = torch.full_like(whole, float("nan"))
+    for r0, r1 in ((0, 333), (333, 900), (900, 1399), (1399, 1400)):
+        ris.ris_attention_masked_rows(m, r0, r1, q, k, v, parts, rope=rope)
+    torch.cuda.synchronize()
+    assert torch.equal(parts, whole)
+    ref = ris.ris_ensemble_batch(q, k, v, 0, 0.03, seeds, rope=rope, out_dtype=torch.float32)
+    torch.cuda.synchronize()
+    assert torch.equal(ref, whole)
+    m.free()
