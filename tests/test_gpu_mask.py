@@ -165,3 +165,39 @@ def test_mask_sub1pct_structural_sweep(d, S):
     p = m.info().params
     assert p.bmax == int(np.floor(d * N + 0.5)) and p.block == min(N // 10, p.bmax)
     check_rows(m, [oracle_spec(N, 1, d, seeds)], sample_rows(N, 16, seed=int(d * 1e4) + S))
+
+
+@pytest.mark.parametrize("N,mode,d,S,W,per_head", [
+    (3000, 1, 0.1, 2, 1, False), (4100, 1, 0.08, 1, 40, False), (3300, 1, 0.1, 1, 700, True),
+    (2900, 0, 0.01, 3, 300, False), (1500, 1, 0.002, 1, 600, False), (2000, 1, 0.05, 1, 1, False),
+    (700, 0, 0.02, 1, 900, False)])
+def test_dense_suffix_is_the_tail_of_every_row(N, mode, d, S, W, per_head):
+    """The dense-suffix split's premise on real masks: every key from lo(i) (the earlier of the
+    row's Structural block start, for blocks of >= 256 tokens, and its local window start,
+    for windows of >= 256) up to i is kept, so those keys end the row's ascending list; and
+    the mask description's suffix pair count is the brute-force sum of their lengths."""
+    m = gpu_mask(N, mode, d, list(range(S)), kv_heads=2, W=W, per_head=per_head)
+    info = m.info()
+    block = info.params.block if (mode == 1 and info.params.block >= 256) else 0
+    allowed = block > 0 or W >= 256
+
+    def lo(i):
+        v = i
+        if block:
+            v = min(v, (i // block) * block)
+        if W > 1:
+            v = min(v, max(0, i - W + 1))
+        return v
+
+    expect = sum(i - lo(i) + 1 for i in range(N)) if allowed else 0
+    assert info.suffix_pairs == expect
+    if allowed:
+        row_ptr = m.row_ptr().cpu().numpy()
+        cols = m.cols().cpu().numpy().astype(np.int64)
+        for mid in range(info.n_masks):
+            for i in range(N):
+                a, b = row_ptr[mid * N + i], row_ptr[mid * N + i + 1]
+                tail = i - lo(i) + 1
+                assert b - a >= tail
+                np.testing.assert_array_equal(cols[b - tail:b], np.arange(lo(i), i + 1), err_msg=f"row {i}")
+    m.free()
