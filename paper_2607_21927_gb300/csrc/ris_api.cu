@@ -213,9 +213,10 @@ int64_t suffix_pairs_of(int64_t N, int64_t block, int64_t W)
 // gather, 4 dense-suffix split (each row's dense suffix on the tile kernel, its other keys on
 // the register gather, one softmax). The gather's cost grows with the pairs it gathers (with
 // the split: all but the suffixes), a tile's does not, hence the density threshold.
-int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim)
+int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim, int32_t group = 1)
 {
     if (dtype == RIS_F32) return 3;
+    if (group > 8) return 2;  // only the tiles take more than 8 query heads per KV head
     const std::string f = forced_design();
     if (f == "tma" && tma_gather_available()) return 1;
     if (f == "gather") return 0;
@@ -284,12 +285,16 @@ ris_status check_seeds(const uint32_t *seeds, int32_t n_seeds)
     return RIS_OK;
 }
 
-ris_status check_shape(int32_t heads, int32_t kv_heads, int32_t head_dim)
+// wide_groups: more than 8 query heads per KV head are allowed (the tile design, which runs
+// one CTA per query head, takes them; the gathers carry at most 8 heads in a tensor-core tile)
+ris_status check_shape(int32_t heads, int32_t kv_heads, int32_t head_dim, bool wide_groups = false)
 {
     if (heads < 1 || kv_heads < 1) return fail(RIS_ERR_INVALID, "heads and kv_heads must be >= 1");
     if (heads % kv_heads != 0) return fail(RIS_ERR_INVALID, "heads %d not a multiple of kv_heads %d", heads, kv_heads);
     if (head_dim != 64 && head_dim != 128) return fail(RIS_ERR_INVALID, "head_dim %d not in {64, 128}", head_dim);
-    if (heads / kv_heads > 8) return fail(RIS_ERR_UNSUPPORTED, "heads/kv_heads = %d > 8 is not built", heads / kv_heads);
+    if (heads / kv_heads > 8 && !wide_groups)
+        return fail(RIS_ERR_UNSUPPORTED, "heads/kv_heads = %d > 8 needs bf16 inputs with head_dim 128 (tile design)",
+                    heads / kv_heads);
     return RIS_OK;
 }
 
@@ -329,14 +334,15 @@ double resolve_factor(const ris_rope_cfg *r, int64_t N)
 
 ris_status validate_attention(const void *q, const void *k, const void *v, void *out, int32_t heads,
                               int32_t kv_heads, int32_t head_dim, int32_t dtype, int32_t out_dtype,
-                              const ris_rope_cfg *rope, const float *lse)
+                              const ris_rope_cfg *rope, const float *lse, bool prefill = true)
 {
     RIS_TRY(check_ptr(q, "q"));
     RIS_TRY(check_ptr(k, "k"));
     RIS_TRY(check_ptr(v, "v"));
     RIS_TRY(check_ptr(out, "out"));
     if (lse != nullptr && !aligned16(lse)) return fail(RIS_ERR_INVALID, "lse is not 16-byte aligned");
-    RIS_TRY(check_shape(heads, kv_heads, head_dim));
+    RIS_TRY(check_shape(heads, kv_heads, head_dim,
+                        prefill && dtype == RIS_BF16 && head_dim == 128 && tile_design_available()));
     RIS_TRY(check_dtype(dtype, "dtype"));
     RIS_TRY(check_dtype(out_dtype, "out_dtype"));
     RIS_TRY(check_rope(rope));
@@ -604,7 +610,7 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     const int64_t N = m->N;
     if (row1 < 0) row1 = N;
     prepare_pool_once();
-    const int design = design_of(m, dtype, head_dim);
+    const int design = design_of(m, dtype, head_dim, heads / kv_heads);
     const bool tile = design == 2, suffix = design == 4;
     const bool q_pair = tile || suffix;  // queries as a bf16 hi + lo pair
     Scratch qt, qtl, kt, ktl, po, pl;
@@ -1019,7 +1025,7 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
                            int64_t n_ctx, const ris_rope_cfg *rope, void *out, float *lse, void *stream)
 {
     if (anchor == nullptr) return fail(RIS_ERR_INVALID, "anchor is NULL");
-    RIS_TRY(validate_attention(q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse));
+    RIS_TRY(validate_attention(q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse, false));
     if (k_lo != nullptr && (dtype != RIS_BF16 || !aligned16(k_lo)))
         return fail(RIS_ERR_INVALID, "k_lo must be NULL for fp32 and 16-byte aligned for bf16");
     if (kv_heads > kMaxDecodeKvHeads) return fail(RIS_ERR_UNSUPPORTED, "kv_heads %d > %d", kv_heads, kMaxDecodeKvHeads);

@@ -56,7 +56,9 @@ def test_invalid_arguments_launch_nothing(ris):
     for c in cases:
         assert call(**c) == ris.RIS_ERR_INVALID, (c, ris.ris_last_error())
         assert ris.ris_last_error() != ""
-    assert call(heads=32, kv_heads=2) == ris.RIS_ERR_UNSUPPORTED
+    # more than 8 query heads per KV head: only bf16 with head_dim 128 (the tile design)
+    assert call(heads=32, kv_heads=2, D=64) == ris.RIS_ERR_UNSUPPORTED
+    assert call(heads=32, kv_heads=2, dt=0) == ris.RIS_ERR_UNSUPPORTED
     bad_rope = ris.rope_cfg(3, 1e6, 32768)
     bad_rope.yarn_beta = 0.5
     st = L.ris_sparse_attention_fwd(p16, p16, p16, p16, 64, 4, 2, 128, 0, 0.05, seeds, 2, 1, 0,

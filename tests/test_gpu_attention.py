@@ -433,3 +433,24 @@ def test_row_ranges_per_seed_sets():
     torch.cuda.synchronize()
     assert torch.equal(ref, whole)
     m.free()
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,S", [(16, 1, 0.02, 2), (24, 2, 0.3, 1)], ids=["mqa_16_sparse", "group_12"])
+def test_groups_wider_than_eight_on_tiles(Hq, Hkv, d, S):
+    """More than 8 query heads per KV head (multi-query attention): bf16 with head_dim 128 runs
+    on the tile design whatever the density; fp32 and head_dim 64 report RIS_ERR_UNSUPPORTED."""
+    N, D = 700, 128
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=43, outliers=True)
+    seeds = list(range(S))
+    out, lse = ris.ris_sparse_attention_fwd(q, k, v, 0, d, seeds, rope=ris.rope_cfg(3, 1e6, 256),
+                                            out_dtype=torch.float32, return_lse=True)
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    ref, ref_lse = run_oracle(qn, kn, vn, 0, d, seeds, 3, 1e6, 256)
+    check_bf16_path(to_np(out), ref)
+    np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
+    with pytest.raises(ris.RisError):
+        ris.ris_sparse_attention_fwd(q.float(), k.float(), v.float(), 0, d, seeds, out_dtype=torch.float32)
+    (q6, k6, v6), _ = make_inputs(N, Hq, Hkv, 64, seed=44)
+    with pytest.raises(ris.RisError):
+        ris.ris_sparse_attention_fwd(q6, k6, v6, 0, d, seeds, out_dtype=torch.float32)
