@@ -182,9 +182,9 @@ ris_status ris_rope_apply(void *x, int32_t dtype, int64_t N, int32_t heads, int3
  * dtype: q, k, v element type; out_dtype: out element type (F32 or BF16). lse: optional
  * [heads][N] fp32 natural-log sum of exp of the scaled scores (NULL to skip).
  * head_dim in {64, 128}; heads a multiple of kv_heads; heads/kv_heads <= 8, or any group size
- * with bf16 inputs and head_dim 128, which then always run on the tile design (the gathers
- * carry at most 8 query heads per KV head; otherwise RIS_ERR_UNSUPPORTED; the decode step
- * keeps the limit of 8).
+ * with bf16 inputs, which then always run on the tile design (the gathers carry at most 8
+ * query heads per KV head; otherwise RIS_ERR_UNSUPPORTED; the decode step keeps the limit
+ * of 8).
  * Errors: RIS_ERR_INVALID, RIS_ERR_UNSUPPORTED, RIS_ERR_OOM, RIS_ERR_CUDA. */
 ris_status ris_sparse_attention_fwd(const void *q, const void *k, const void *v, void *out,
                                     int64_t N, int32_t heads, int32_t kv_heads, int32_t head_dim,
@@ -269,9 +269,9 @@ ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double 
 
 /* Attention kernel design a layer call on `mask` uses for this input dtype and head_dim
  * (host-only, no device work): 0 register gather, 1 TMA gather, 2 tcgen05 masked dense tiles,
- * 3 fp32 gather, 4 dense-suffix split; -1 for invalid arguments. bf16 calls with head_dim
- * 128 use tiles when the mask is dense or keeps at least 8.5% of the causal pairs in what a
- * gather would fetch (and always when heads/kv_heads > 8, which this call does not see). The dense-suffix split applies to masks (not per seed) with Structural
+ * 3 fp32 gather, 4 dense-suffix split; -1 for invalid arguments. bf16 calls use tiles when
+ * the mask is dense or keeps at least 8.5% of the causal pairs in what a gather would fetch
+ * (and always when heads/kv_heads > 8, which this call does not see). The dense-suffix split applies to masks (not per seed) with Structural
  * blocks of at least 256 tokens or a local window of at least 256 keys: every key of row i
  * from the earlier of its block start and its window start up to i is kept (Methods,
  * "Sampling Modes": in-block pairs are cliques; the window is forced), so a first launch

@@ -59,20 +59,23 @@ namespace {
 
 constexpr int BM = 128;          // query rows per tile (TMEM lanes)
 constexpr int BN = 128;          // keys per stage
-constexpr int DT = 128;          // head dim handled by this kernel
 constexpr int kThreads = 320;    // warps 0-7 softmax (two column halves), 8 TMA, 9 MMA
 constexpr int kTmaWarp = 8, kMmaWarp = 9;
 constexpr uint32_t kTmemCols = 512;  // S/P[2] (2 x 128) + O (128) + Q hi / lo (2 x 64)
 
-// shared-memory map (bytes, from a 1024-aligned base)
-constexpr int KV_ARR = BN * DT * 2;         // 32 KB: one of K hi / K lo / V
+// shared-memory map (bytes, from a 1024-aligned base) for head dim DT (128 or 64)
+template <int DT>
+struct Smem {
+    static constexpr int KV_ARR = BN * DT * 2;  // 32 KB at DT = 128: one of K hi / K lo / V
+    static constexpr int K_STAGE = 2 * KV_ARR;  // K hi, K lo
+    static constexpr int V_STAGE = KV_ARR;
+};
 constexpr int KV_BLK = BN * 128;            // 16 KB: one 64-column block
-constexpr int K_STAGE = 2 * KV_ARR;         // 64 KB: K hi, K lo
-constexpr int V_STAGE = KV_ARR;             // 32 KB
 constexpr int kStages = 2;                  // stages of each ring
 constexpr int OFF_K = 0;
-constexpr int OFF_V = OFF_K + kStages * K_STAGE;
-constexpr int SMEM_BYTES = OFF_V + kStages * V_STAGE + 1024;  // + alignment slack = 197632
+// the head-dim-128 layout (197632 bytes with the alignment slack) is requested at either
+// head dim: it keeps one CTA per SM, as the CTA holds all 512 TMEM columns
+constexpr int SMEM_BYTES = OFF_K + kStages * (Smem<128>::K_STAGE + Smem<128>::V_STAGE) + 1024;
 
 // P_FULL and PV_DONE have one barrier per P buffer (tile parity), so that no waiter can fall
 // two phases behind a barrier it polls by parity.
@@ -302,10 +305,15 @@ struct TileMaps {
     CUtensorMap kh, kl, v;
 };
 
-template <bool SPLIT, bool DENSE, bool SUFFIX, typename TOut>
+template <int DT, bool SPLIT, bool DENSE, bool SUFFIX, typename TOut>
 __global__ void __launch_bounds__(kThreads, 1)
     k_attn_tile(const AttnArgs a, const __grid_constant__ TileMaps maps, const void *q_hi, const void *q_lo)
 {
+    static_assert(DT == 128 || DT == 64, "head dim 64 or 128");
+    constexpr int KV_ARR = Smem<DT>::KV_ARR, K_STAGE = Smem<DT>::K_STAGE, V_STAGE = Smem<DT>::V_STAGE;
+    constexpr int OFF_V = OFF_K + kStages * K_STAGE;
+    constexpr int NB = DT / 64;  // 64-column blocks of a row
+    constexpr int HALF = DT / 2; // head-dim columns of one softmax thread (one of two per row)
     extern __shared__ unsigned char smem_raw[];
     __shared__ __align__(8) uint64_t bars[NBAR];
     __shared__ uint32_t tmem_base_sh;
@@ -369,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t bk = smem_u32(&bars[B_K_FULL + st]);
                 const uint32_t dk = sbase + OFF_K + st * K_STAGE;
                 mbar_arrive_expect_tx(bk, (SPLIT ? 2 : 1) * KV_ARR);
-                for (int blk = 0; blk < 2; ++blk) {
+                for (int blk = 0; blk < NB; ++blk) {
                     tma_load_3d(dk + blk * KV_BLK, &maps.kh, 64 * blk, g, (kt0 + j) * BN, bk);
                     if (SPLIT) tma_load_3d(dk + KV_ARR + blk * KV_BLK, &maps.kl, 64 * blk, g, (kt0 + j) * BN, bk);
                 }
@@ -379,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t bv = smem_u32(&bars[B_V_FULL + st]);
                 const uint32_t dv = sbase + OFF_V + st * V_STAGE;
                 mbar_arrive_expect_tx(bv, KV_ARR);
-                for (int blk = 0; blk < 2; ++blk) tma_load_3d(dv + blk * KV_BLK, &maps.v, 64 * blk, g, (kt0 + j) * BN, bv);
+                for (int blk = 0; blk < NB; ++blk) tma_load_3d(dv + blk * KV_BLK, &maps.v, 64 * blk, g, (kt0 + j) * BN, bv);
                 nv = j + 1;
             }
             // let the copies requested last into each stage land before the CTA can leave
@@ -502,23 +510,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             other = xch[pb][hf ^ 1][r];
             return got;
         };
-        // this thread's half row of the query tile (head-dim 64 hf .. 64 hf + 63) into TMEM
+        // this thread's half row of the query tile (head-dim HALF hf .. HALF hf + HALF - 1,
+        // DT / 4 packed columns) into TMEM
         {
-            uint32_t qw[32];
-            const int64_t qrow = ((row_ok ? i : 0) * a.Hq + h) * DT + 64 * hf;
+            uint32_t qw[DT / 4];
+            const int64_t qrow = ((row_ok ? i : 0) * a.Hq + h) * DT + HALF * hf;
             for (int part = 0; part < (SPLIT ? 2 : 1); ++part) {
                 const uint4 *src = reinterpret_cast<const uint4 *>(
                     reinterpret_cast<const __nv_bfloat16 *>(part == 0 ? q_hi : q_lo) + qrow);
 #pragma unroll
-                for (int u = 0; u < 8; ++u) {
+                for (int u = 0; u < DT / 16; ++u) {
                     const uint4 x = row_ok ? src[u] : make_uint4(0u, 0u, 0u, 0u);
                     qw[4 * u] = x.x;
                     qw[4 * u + 1] = x.y;
                     qw[4 * u + 2] = x.z;
                     qw[4 * u + 3] = x.w;
                 }
-                tmem_st16(t_q + lane_off + (DT / 2) * part + 32 * hf, qw);
-                tmem_st16(t_q + lane_off + (DT / 2) * part + 32 * hf + 16, qw + 16);
+#pragma unroll
+                for (int w16 = 0; w16 < DT / 64; ++w16)
+                    tmem_st16(t_q + lane_off + (DT / 2) * part + (DT / 4) * hf + 16 * w16, qw + 16 * w16);
             }
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_Q]));
@@ -577,11 +587,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 float ov[32];
 #pragma unroll
-                for (int c4 = 0; c4 < 2; ++c4) {
-                    tmem_ld32(t_o + lane_off + 64 * hf + 32 * c4, ov);
+                for (int c4 = 0; c4 < HALF / 32; ++c4) {
+                    tmem_ld32(t_o + lane_off + HALF * hf + 32 * c4, ov);
 #pragma unroll
                     for (int c = 0; c < 32; ++c) ov[c] *= al;
-                    tmem_st32(t_o + lane_off + 64 * hf + 32 * c4, ov);
+                    tmem_st32(t_o + lane_off + HALF * hf + 32 * c4, ov);
                 }
             }
             const float mu = (m_used == -INFINITY) ? 0.f : m_used;
@@ -615,13 +625,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const float lt = l + ol;
             const float inv = lt > 0.f ? 1.f / lt : 0.f;
-            TOut *out = SUFFIX ? reinterpret_cast<TOut *>(a.part_o + ((row_ok ? i : 0) * a.Hq + h) * DT + 64 * hf)
+            TOut *out = SUFFIX ? reinterpret_cast<TOut *>(a.part_o + ((row_ok ? i : 0) * a.Hq + h) * DT + HALF * hf)
                                : reinterpret_cast<TOut *>(a.out) + (((int64_t)s * a.N + (row_ok ? i : 0)) * a.Hq + h) * DT +
-                                     64 * hf;
+                                     HALF * hf;
             float ov[32];
 #pragma unroll
-            for (int c4 = 0; c4 < 2; ++c4) {
-                tmem_ld32(t_o + lane_off + 64 * hf + 32 * c4, ov);
+            for (int c4 = 0; c4 < HALF / 32; ++c4) {
+                tmem_ld32(t_o + lane_off + HALF * hf + 32 * c4, ov);
                 if (row_ok) {
 #pragma unroll
                     for (int c = 0; c < 32; ++c) ov[c] *= inv;
@@ -660,8 +670,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-// [N][H][128] bf16 viewed as 3D (d, head, token); box = 64 d x 1 head x `rows` tokens.
-bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows)
+// [N][H][DT] bf16 viewed as 3D (d, head, token); box = 64 d x 1 head x `rows` tokens.
+bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows, int DT)
 {
     auto fn = encode_fn();
     if (fn == nullptr) return false;
@@ -674,10 +684,10 @@ bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows)
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool SPLIT, bool DENSE, typename TOut, bool SUFFIX = false>
+template <int DT, bool SPLIT, bool DENSE, typename TOut, bool SUFFIX = false>
 cudaError_t launch_t(const AttnArgs &a, const TileMaps &maps, const void *q_hi, const void *q_lo, cudaStream_t s)
 {
-    auto kern = k_attn_tile<SPLIT, DENSE, SUFFIX, TOut>;
+    auto kern = k_attn_tile<DT, SPLIT, DENSE, SUFFIX, TOut>;
     static bool attr = false;
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
@@ -706,43 +716,58 @@ cudaError_t read_tile_error(unsigned int *out)
 }
 
 // K / V tensor maps of a call (the key low part only with split queries and keys).
-bool make_maps(TileMaps &maps, const AttnArgs &a, bool split)
+bool make_maps(TileMaps &maps, const AttnArgs &a, bool split, int D)
 {
-    if (!make_map3(&maps.kh, a.k, a.N, a.Hkv, BN) || !make_map3(&maps.v, a.v, a.N, a.Hkv, BN)) return false;
-    if (split) return make_map3(&maps.kl, a.k_lo, a.N, a.Hkv, BN);
+    if (!make_map3(&maps.kh, a.k, a.N, a.Hkv, BN, D) || !make_map3(&maps.v, a.v, a.N, a.Hkv, BN, D)) return false;
+    if (split) return make_map3(&maps.kl, a.k_lo, a.N, a.Hkv, BN, D);
     maps.kl = maps.kh;
     return true;
 }
 
-// q_hi / q_lo: queries as a bf16 pair [N][Hq][128] (q_lo null: exact bf16 queries and keys,
-// one score product); a.k / a.k_lo: keys as a pair; a.v: values. Head dim 128 only.
-cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const void *q_lo, int out_dtype, bool dense,
-                                  cudaStream_t s)
+template <int DT>
+cudaError_t launch_tile_d(const AttnArgs &a, const TileMaps &maps, const void *q_hi, const void *q_lo, int out_dtype,
+                          bool dense, cudaStream_t s)
 {
-    static std::mutex mu;
-    std::lock_guard<std::mutex> lk(mu);
     const bool split = q_lo != nullptr;
-    alignas(64) TileMaps maps;
-    if (!make_maps(maps, a, split)) return cudaErrorInvalidValue;
     if (out_dtype == RIS_F32) {
-        if (split) return dense ? launch_t<true, true, float>(a, maps, q_hi, q_lo, s) : launch_t<true, false, float>(a, maps, q_hi, q_lo, s);
-        return dense ? launch_t<false, true, float>(a, maps, q_hi, q_lo, s) : launch_t<false, false, float>(a, maps, q_hi, q_lo, s);
+        if (split) return dense ? launch_t<DT, true, true, float>(a, maps, q_hi, q_lo, s) : launch_t<DT, true, false, float>(a, maps, q_hi, q_lo, s);
+        return dense ? launch_t<DT, false, true, float>(a, maps, q_hi, q_lo, s) : launch_t<DT, false, false, float>(a, maps, q_hi, q_lo, s);
     }
     if (split)
-        return dense ? launch_t<true, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s) : launch_t<true, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
-    return dense ? launch_t<false, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s) : launch_t<false, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
+        return dense ? launch_t<DT, true, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s)
+                     : launch_t<DT, true, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
+    return dense ? launch_t<DT, false, true, __nv_bfloat16>(a, maps, q_hi, q_lo, s)
+                 : launch_t<DT, false, false, __nv_bfloat16>(a, maps, q_hi, q_lo, s);
 }
 
-cudaError_t launch_attention_tile_suffix(const AttnArgs &a, const void *q_hi, const void *q_lo, cudaStream_t s)
+// q_hi / q_lo: queries as a bf16 pair [N][Hq][D] (q_lo null: exact bf16 queries and keys,
+// one score product); a.k / a.k_lo: keys as a pair; a.v: values. Head dim 128 or 64.
+cudaError_t launch_attention_tile(const AttnArgs &a, int D, const void *q_hi, const void *q_lo, int out_dtype,
+                                  bool dense, cudaStream_t s)
 {
     static std::mutex mu;
     std::lock_guard<std::mutex> lk(mu);
-    if (a.part_o == nullptr || a.part_lse == nullptr || a.n_sets != 1) return cudaErrorInvalidValue;
+    if (D != 128 && D != 64) return cudaErrorInvalidValue;
+    alignas(64) TileMaps maps;
+    if (!make_maps(maps, a, q_lo != nullptr, D)) return cudaErrorInvalidValue;
+    return D == 128 ? launch_tile_d<128>(a, maps, q_hi, q_lo, out_dtype, dense, s)
+                    : launch_tile_d<64>(a, maps, q_hi, q_lo, out_dtype, dense, s);
+}
+
+cudaError_t launch_attention_tile_suffix(const AttnArgs &a, int D, const void *q_hi, const void *q_lo, cudaStream_t s)
+{
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lk(mu);
+    if (a.part_o == nullptr || a.part_lse == nullptr || a.n_sets != 1 || (D != 128 && D != 64))
+        return cudaErrorInvalidValue;
     const bool split = q_lo != nullptr;
     alignas(64) TileMaps maps;
-    if (!make_maps(maps, a, split)) return cudaErrorInvalidValue;
-    return split ? launch_t<true, false, float, true>(a, maps, q_hi, q_lo, s)
-                 : launch_t<false, false, float, true>(a, maps, q_hi, q_lo, s);
+    if (!make_maps(maps, a, split, D)) return cudaErrorInvalidValue;
+    if (D == 128)
+        return split ? launch_t<128, true, false, float, true>(a, maps, q_hi, q_lo, s)
+                     : launch_t<128, false, false, float, true>(a, maps, q_hi, q_lo, s);
+    return split ? launch_t<64, true, false, float, true>(a, maps, q_hi, q_lo, s)
+                 : launch_t<64, false, false, float, true>(a, maps, q_hi, q_lo, s);
 }
 
 }  // namespace ris

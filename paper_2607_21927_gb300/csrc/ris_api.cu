@@ -220,7 +220,7 @@ int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim, int32_t grou
     const std::string f = forced_design();
     if (f == "tma" && tma_gather_available()) return 1;
     if (f == "gather") return 0;
-    const bool tiles = head_dim == 128 && tile_design_available();
+    const bool tiles = (head_dim == 128 || head_dim == 64) && tile_design_available();
     if (tiles && (f == "tile" || m->dense)) return 2;
     const bool split = tiles && suffix_split_allowed(m);
     if (split && f == "suffix") return 4;
@@ -293,7 +293,7 @@ ris_status check_shape(int32_t heads, int32_t kv_heads, int32_t head_dim, bool w
     if (heads % kv_heads != 0) return fail(RIS_ERR_INVALID, "heads %d not a multiple of kv_heads %d", heads, kv_heads);
     if (head_dim != 64 && head_dim != 128) return fail(RIS_ERR_INVALID, "head_dim %d not in {64, 128}", head_dim);
     if (heads / kv_heads > 8 && !wide_groups)
-        return fail(RIS_ERR_UNSUPPORTED, "heads/kv_heads = %d > 8 needs bf16 inputs with head_dim 128 (tile design)",
+        return fail(RIS_ERR_UNSUPPORTED, "heads/kv_heads = %d > 8 needs bf16 inputs (tile design)",
                     heads / kv_heads);
     return RIS_OK;
 }
@@ -341,8 +341,7 @@ ris_status validate_attention(const void *q, const void *k, const void *v, void 
     RIS_TRY(check_ptr(v, "v"));
     RIS_TRY(check_ptr(out, "out"));
     if (lse != nullptr && !aligned16(lse)) return fail(RIS_ERR_INVALID, "lse is not 16-byte aligned");
-    RIS_TRY(check_shape(heads, kv_heads, head_dim,
-                        prefill && dtype == RIS_BF16 && head_dim == 128 && tile_design_available()));
+    RIS_TRY(check_shape(heads, kv_heads, head_dim, prefill && dtype == RIS_BF16 && tile_design_available()));
     RIS_TRY(check_dtype(dtype, "dtype"));
     RIS_TRY(check_dtype(out_dtype, "out_dtype"));
     RIS_TRY(check_rope(rope));
@@ -684,9 +683,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     const auto ev = timer_pair();
     if (ev.first) RIS_CUDA(cudaEventRecord(ev.first, s));
     if (tile) {
-        RIS_CUDA(launch_attention_tile(a, qu, q_lo, out_dtype, m->dense != 0, s));
+        RIS_CUDA(launch_attention_tile(a, head_dim, qu, q_lo, out_dtype, m->dense != 0, s));
     } else if (suffix) {  // the dense suffixes on the tiles, then the gather continues their softmax
-        RIS_CUDA(launch_attention_tile_suffix(a, qu, a.q_lo, s));
+        RIS_CUDA(launch_attention_tile_suffix(a, head_dim, qu, a.q_lo, s));
         RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, false, s));
     } else if (design == 1)
         RIS_CUDA(launch_attention_tma(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));

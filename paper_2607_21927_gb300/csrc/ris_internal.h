@@ -177,13 +177,13 @@ cudaError_t launch_attention_tma(const AttnArgs &a, int D, int out_dtype, bool s
                                  cudaStream_t s);
 cudaError_t read_device_error(unsigned int *out, cudaStream_t s);
 
-// Masked dense-tile design (tcgen05, head dim 128): q_hi / q_lo bf16 query pair (q_lo null
-// for exact bf16 inputs).
+// Masked dense-tile design (tcgen05, head dim 128 or 64): q_hi / q_lo bf16 query pair (q_lo
+// null for exact bf16 inputs).
 bool tile_design_available();
-cudaError_t launch_attention_tile(const AttnArgs &a, const void *q_hi, const void *q_lo, int out_dtype, bool dense,
-                                  cudaStream_t s);
+cudaError_t launch_attention_tile(const AttnArgs &a, int D, const void *q_hi, const void *q_lo, int out_dtype,
+                                  bool dense, cudaStream_t s);
 // The suffix pass of the dense-suffix split (a.part_o set): writes a.part_o / a.part_lse.
-cudaError_t launch_attention_tile_suffix(const AttnArgs &a, const void *q_hi, const void *q_lo, cudaStream_t s);
+cudaError_t launch_attention_tile_suffix(const AttnArgs &a, int D, const void *q_hi, const void *q_lo, cudaStream_t s);
 cudaError_t read_tile_error(unsigned int *out);
 
 }  // namespace ris

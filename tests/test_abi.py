@@ -56,8 +56,7 @@ def test_invalid_arguments_launch_nothing(ris):
     for c in cases:
         assert call(**c) == ris.RIS_ERR_INVALID, (c, ris.ris_last_error())
         assert ris.ris_last_error() != ""
-    # more than 8 query heads per KV head: only bf16 with head_dim 128 (the tile design)
-    assert call(heads=32, kv_heads=2, D=64) == ris.RIS_ERR_UNSUPPORTED
+    # more than 8 query heads per KV head: bf16 only (the tile design)
     assert call(heads=32, kv_heads=2, dt=0) == ris.RIS_ERR_UNSUPPORTED
     bad_rope = ris.rope_cfg(3, 1e6, 32768)
     bad_rope.yarn_beta = 0.5

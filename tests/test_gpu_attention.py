@@ -297,11 +297,11 @@ def test_row_ranges_reassemble_the_layer(d, S, D):
 
 def test_structural_split_design_choice():
     """C5's Structural mask (blocks of 655) takes the dense-suffix split: cliques on the tiles,
-    the rest gathered; Structural masks with small blocks and no wide window, per-seed masks
-    and head_dim 64 do not; a Stochastic mask with a 1024-key window does."""
+    the rest gathered, at head_dim 128 and 64; Structural masks with small blocks and no wide
+    window, and per-seed masks, do not; a Stochastic mask with a 1024-key window does."""
     m = ris.ris_mask_generate(65536, 2, 1, 0.01, list(range(10)))
     assert ris.ris_attention_design(m, torch.bfloat16, 128) == 4
-    assert ris.ris_attention_design(m, torch.bfloat16, 64) == 0
+    assert ris.ris_attention_design(m, torch.bfloat16, 64) == 4
     m.free()
     m = ris.ris_mask_generate(2000, 2, 1, 0.05, [1])  # B = min(200, 100) = 100 < 256
     assert ris.ris_attention_design(m, torch.bfloat16, 128) in (0, 2)
@@ -435,11 +435,12 @@ def test_row_ranges_per_seed_sets():
     m.free()
 
 
-@pytest.mark.parametrize("Hq,Hkv,d,S", [(16, 1, 0.02, 2), (24, 2, 0.3, 1)], ids=["mqa_16_sparse", "group_12"])
-def test_groups_wider_than_eight_on_tiles(Hq, Hkv, d, S):
-    """More than 8 query heads per KV head (multi-query attention): bf16 with head_dim 128 runs
-    on the tile design whatever the density; fp32 and head_dim 64 report RIS_ERR_UNSUPPORTED."""
-    N, D = 700, 128
+@pytest.mark.parametrize("Hq,Hkv,D,d,S", [(16, 1, 128, 0.02, 2), (24, 2, 128, 0.3, 1), (16, 1, 64, 0.05, 1)],
+                         ids=["mqa_16_sparse", "group_12", "mqa_16_hd64"])
+def test_groups_wider_than_eight_on_tiles(Hq, Hkv, D, d, S):
+    """More than 8 query heads per KV head (multi-query attention): bf16 runs on the tile
+    design whatever the density; fp32 reports RIS_ERR_UNSUPPORTED."""
+    N = 700
     (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=43, outliers=True)
     seeds = list(range(S))
     out, lse = ris.ris_sparse_attention_fwd(q, k, v, 0, d, seeds, rope=ris.rope_cfg(3, 1e6, 256),
@@ -451,6 +452,24 @@ def test_groups_wider_than_eight_on_tiles(Hq, Hkv, d, S):
     np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
     with pytest.raises(ris.RisError):
         ris.ris_sparse_attention_fwd(q.float(), k.float(), v.float(), 0, d, seeds, out_dtype=torch.float32)
-    (q6, k6, v6), _ = make_inputs(N, Hq, Hkv, 64, seed=44)
-    with pytest.raises(ris.RisError):
-        ris.ris_sparse_attention_fwd(q6, k6, v6, 0, d, seeds, out_dtype=torch.float32)
+
+
+@pytest.mark.parametrize("N,mode,d,S,W,Hq,Hkv,design", [
+    (1100, 0, 0.3, 2, 1, 32, 4, 2), (900, 2, 1.0, 1, 1, 8, 1, 2), (3000, 1, 0.1, 1, 1, 32, 4, 4),
+    (2000, 0, 0.01, 1, 400, 16, 2, 4)], ids=["tiles", "dense", "suffix_split_blocks", "suffix_split_window"])
+def test_head_dim_64_on_tiles(N, mode, d, S, W, Hq, Hkv, design):
+    """head_dim 64 (TinyLlama-shaped heads) on the tile design and the dense-suffix split,
+    every row against the oracle, with the log-sum-exp."""
+    D = 64
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=N + 1, outliers=True)
+    seeds = list(range(S))
+    m = ris.ris_mask_generate(N, Hkv, mode, d, seeds, opts=ris.mask_opts(local_window=W))
+    assert ris.ris_attention_design(m, torch.bfloat16, D) == design
+    out, lse = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e4, 256), out_dtype=torch.float32,
+                                        return_lse=True)
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    m.free()
+    ref, ref_lse = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e4, 256, W=W)
+    check_bf16_path(to_np(out), ref)
+    np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
