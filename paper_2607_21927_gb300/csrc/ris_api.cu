@@ -168,8 +168,11 @@ const char *forced_design()
 // Union density at and above which masked dense tiles beat gathering pair by pair (bf16,
 // head dim 128): a tile costs the dense causal products (x2.5 for the precision splits)
 // whatever the mask, a gathered pair 1.5 KB of K/V rows. Measured crossover on Qwen2-shaped
-// layers: 8.6% of the causal pairs at N = 32768 and 8.4% at N = 65536.
+// layers (head dim 128): 8.6% of the causal pairs at N = 32768 and 8.4% at N = 65536; on
+// TinyLlama-shaped layers (head dim 64, 32 query and 4 KV heads, N = 16384) 16.8%, where the
+// tiles are half the products but the same softmax work.
 constexpr double kTileDensity = 0.085;
+constexpr double kTileDensity64 = 0.168;
 
 // Shortest dense span (Structural block or local window) for which the split pays: two
 // 128-key tiles.
@@ -227,7 +230,7 @@ int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim, int32_t grou
     if (tiles) {
         const double causal = (double)m->n_masks * ((double)m->N * (double)(m->N + 1) / 2.0);
         const double gathered = (double)m->n_pairs - (split ? (double)m->n_masks * (double)m->suffix_pairs : 0.0);
-        if (gathered >= kTileDensity * causal) return 2;
+        if (gathered >= (head_dim == 64 ? kTileDensity64 : kTileDensity) * causal) return 2;
     }
     return split ? 4 : 0;
 }
