@@ -1,4 +1,4 @@
-// Measurement support: the hardware ceilings the attention kernels are judged against that
+// Measurement support: the hardware ceilings the attention kernels are measured against that
 // a plain copy or a library GEMM does not give, each measured by a small kernel of its own.
 //
 //  - L2 read bandwidth for streaming 16-byte loads over a working set that stays resident in
