@@ -15,17 +15,15 @@
 //   k_decode_partial : one CTA per (chunk of 32 keys, KV head): issues all of the chunk's
 //                      16-byte K~ (high + low parts) and V row loads at once, rotates the G
 //                      query heads of the KV head at position t (fp64 angle, as the prefill
-//                      RoPE) while they are in flight, and computes each head's partial
-//                      (max, sum, unnormalised output) in shared memory; clusters of 8 CTAs
-//                      merge their partials through distributed shared memory, and the first
-//                      CTA of each cluster writes one partial.
-//   k_decode_combine : one CTA per query head: rescales the cluster partials to the global
-//                      maximum, sums and normalises; optional natural-log LSE.
+//                      RoPE) while they are in flight, takes the scores of all heads straight
+//                      from the key pieces in registers, and writes each head's partial
+//                      (max, sum, unnormalised output) to global memory.
+//   k_decode_combine : one CTA per (query head, 32 channels): rescales the chunk partials to
+//                      the global maximum, sums and normalises; optional natural-log LSE.
 //
 // A decode step is one query row: a GEMV-shaped product that reads each selected K/V row once,
 // so it runs on the FP32 pipes (no tensor-core tile to fill) and is bound by the K/V row
 // reads; fp32 scores and probabilities keep it well inside the bf16 tolerance.
-#include <cooperative_groups.h>
 #include <utility>
 #include <cuda_bf16.h>
 
@@ -34,7 +32,6 @@
 
 #include "ris_internal.h"
 
-namespace cg = cooperative_groups;
 
 namespace ris {
 namespace {
@@ -58,6 +55,14 @@ __device__ __forceinline__ void sincos_reduced(double a, float *sn, float *cs)
     double red = fma(-n, 6.28318530717958623200, a);
     red = fma(-n, 2.4492935982947064e-16, red);
     sincosf((float)red, sn, cs);
+}
+
+// Asynchronous prefetch of `bytes` (a multiple of 16, 16-byte aligned address) into L2; no
+// result comes back to the thread.
+__device__ __forceinline__ void prefetch_l2(const void *p, int bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(__cvta_generic_to_global(p)), "r"(bytes)
+                 : "memory");
 }
 
 // 16-byte row pieces of the staged K/V rows: bf16 holds 8 values per piece, fp32 holds 4.
@@ -84,51 +89,71 @@ __device__ __forceinline__ void unpack(const uint4 &u, float *o, const float *)
     o[3] = __uint_as_float(u.w);
 }
 
-// One CTA per (chunk of kDecodeChunk keys, KV head); kDecodeCluster consecutive chunks form a
-// thread-block cluster whose first CTA merges the cluster's partials through distributed
-// shared memory, so only one partial per cluster goes to global memory. Chunks below
+// One CTA per (chunk of kDecodeChunk keys, KV head), each writing its own partial. Chunks below
 // n_anchor_chunks take anchor entries, the others window positions. On the way to the K/V
 // rows there is one round of dependent global loads: the position and this chunk's slice of
-// the anchor list, side by side.
+// the anchor list, side by side. (Merging the partials of 2, 4 or 8 CTAs on chip through
+// thread-block clusters and distributed shared memory measured slower: the cluster barriers
+// and the remote reads cost more than the combine kernel's extra partials.)
 template <typename T, bool LO, int D>
-__global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecodeThreads)
-    k_decode_partial(const DecodeArgs a)
+__global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeArgs a)
 {
     constexpr int kPiecesRow = D * (int)sizeof(T) / 16;                   // 16-byte pieces per row
     constexpr int kPieces = kDecodeChunk * kPiecesRow / kDecodeThreads;  // per thread and plane
     constexpr int kHalf = D / 2;
-    constexpr int kQuarter = D / 4;
+    constexpr int kVals = Piece<T>::kVals;                               // values per piece
+    constexpr int kRowStep = kDecodeThreads / kPiecesRow;                // rows between a thread's pieces
+    constexpr int kLog = kPiecesRow == 8 ? 3 : kPiecesRow == 16 ? 4 : 5;  // log2(kPiecesRow)
     static_assert(kDecodeChunk * kPiecesRow % kDecodeThreads == 0, "pieces per thread");
+    static_assert(kDecodeThreads % kPiecesRow == 0 && (1 << kLog) == kPiecesRow, "a row's pieces in one warp");
+    static_assert(kMaxG == 8, "the score butterfly splits 8 heads");
     static_assert(D <= kDecodeThreads, "one thread per channel in the value product");
-    __shared__ __align__(16) float qs[kMaxG][D];
-    __shared__ __align__(16) float ks[kDecodeChunk][D + 4];  // +4: 16-byte rows in distinct bank groups
-    __shared__ float vs[kDecodeChunk][D];
+    __shared__ __align__(16) float qs[kMaxG][D];  // rotated query heads (rows G .. kMaxG-1 zero)
+    __shared__ __align__(16) float vs[kDecodeChunk][D];
+    __shared__ float sc[kMaxG][kDecodeChunk];     // scores
     __shared__ __align__(16) float ps[kMaxG][kDecodeChunk];
-    __shared__ __align__(16) float os[kMaxG][D];  // this CTA's unnormalised outputs
-    __shared__ float2 ml[kMaxG];                  // this CTA's (max, sum), log2 domain
-    __shared__ float wt[kMaxG][kDecodeCluster];   // merge weights (first CTA of the cluster)
     __shared__ float2 rot[kHalf];                 // (cos, sin) of t * f_c
     __shared__ int32_t keys[kDecodeChunk];
 
     __shared__ uint32_t kept;  // bit r: key r of the chunk is in the merged set
 
-    cg::cluster_group cluster = cg::this_cluster();
     const int g = blockIdx.y, chunk = blockIdx.x, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
+    const int pc = tid % kPiecesRow, r0 = tid / kPiecesRow;  // this thread's 16-byte column piece and first row
     const int G = a.G;
     const int m = a.heads_keyed > 1 ? g : 0;
     const bool from_anchor = chunk < a.n_anchor_chunks;
     const int64_t k0 = (int64_t)(from_anchor ? chunk : chunk - a.n_anchor_chunks) * kDecodeChunk;
+    // Launched as a programmatic dependent of the kernel before it (in a token chain, the
+    // previous layer step's combine), this CTA may start while that kernel still runs. Until
+    // the wait below it only warms L2: warp 0 reads the position and the chunk's anchor slice
+    // through L2 (no L1 copy) and prefetches the K/V rows they name, so that the row loads
+    // after the wait hit L2 instead of HBM. What is read here may be stale; it only steers
+    // prefetches of rows inside the cache, and everything is read again after the wait.
+    if (warp == 0) {
+        const int64_t tg = a.t_dev != nullptr ? (int64_t)__ldcg(reinterpret_cast<const long long *>(a.t_dev)) : a.t;
+        int64_t key = -1;
+        if (from_anchor) {
+            if (k0 + lane < a.anchor_len[m]) key = __ldcg(a.anchor + a.anchor_base[m] + k0 + lane);
+        } else if (tg >= 0 && tg < a.cache_len) {
+            key = (tg - a.window + 1 > 0 ? tg - a.window + 1 : 0) + k0 + lane;
+            if (key > tg) key = -1;
+        }
+        if (key >= 0 && key < a.cache_len) {
+            const int64_t row = (key * a.Hkv + g) * D;
+            prefetch_l2(reinterpret_cast<const T *>(a.k) + row, D * (int)sizeof(T));
+            if (LO) prefetch_l2(reinterpret_cast<const __nv_bfloat16 *>(a.k_lo) + row, D * 2);
+            prefetch_l2(reinterpret_cast<const T *>(a.v) + row, D * (int)sizeof(T));
+        }
+    }
+    // Wait for the kernel before (the position, q, the anchor list of a fresh build and the
+    // partials' buffer come after it), then let the next kernel be scheduled while this one runs.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     // this lane's anchor entry, loaded alongside the position
     int32_t spec = -1;
     if (from_anchor && tid < kDecodeChunk && k0 + tid < a.anchor_len[m])
-        spec = __ldg(a.anchor + a.anchor_base[m] + k0 + tid);
-    // Launched as a programmatic dependent of the kernel before it (the previous step's
-    // combine): everything above only reads the anchor list, built before the first step.
-    // Wait for that kernel (the position, q and the partials' buffer come after it), then let
-    // the next kernel be scheduled while this one runs.
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+        spec = __ldcg(a.anchor + a.anchor_base[m] + k0 + tid);
     const int64_t t = a.t_dev != nullptr ? *a.t_dev : a.t;
     const bool valid = t >= a.t0 && t < a.cache_len;  // only a device-side t can be outside
     if (!valid && tid == 0 && chunk == 0 && g == 0) atomicOr(&g_ris_decode_error, 2u);
@@ -143,68 +168,110 @@ __global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecode
     }
     __syncthreads();
     const uint32_t kbits = kept;
-    const bool active = kbits != 0u;  // block-uniform; inactive CTAs still take part in the cluster syncs
+    const bool active = kbits != 0u;  // block-uniform
+    const int64_t slot = (int64_t)g * a.n_chunks + chunk;  // this CTA's partial
 
     if (active) {
-        // every row load of the chunk is issued before any is used
+        // every row load of the chunk is issued before any is used; a thread's pieces are all
+        // at the same column offset (pc), in rows r0, r0 + kRowStep, ...
         uint4 kh[kPieces], kl[kPieces], vv[kPieces];
 #pragma unroll
         for (int j = 0; j < kPieces; ++j) {
-            const int u = tid + j * kDecodeThreads, r = u / kPiecesRow, pc = u - r * kPiecesRow;
-            const int64_t row = ((int64_t)keys[r] * a.Hkv + g) * D;
+            const int64_t row = ((int64_t)keys[r0 + j * kRowStep] * a.Hkv + g) * D;
             kh[j] = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const T *>(a.k) + row) + pc);
             if (LO) kl[j] = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(a.k_lo) + row) + pc);
             vv[j] = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const T *>(a.v) + row) + pc);
         }
-        // rotate the G query heads at position t while the rows are in flight
+        // rotate the G query heads at position t while the rows are in flight (heads G .. kMaxG-1
+        // are zero, so that the score loop below runs over kMaxG heads without guards)
         if (tid < kHalf) {
             float sn, cs;
             sincos_reduced((double)t * a.f[tid], &sn, &cs);
             rot[tid] = make_float2(cs, sn);
         }
         __syncthreads();
-        for (int idx = tid; idx < G * kHalf; idx += kDecodeThreads) {
+        for (int idx = tid; idx < kMaxG * kHalf; idx += kDecodeThreads) {
             const int h = idx / kHalf, c = idx - h * kHalf;
-            const float2 cs = rot[c];
-            const T *qp = reinterpret_cast<const T *>(a.q) + (int64_t)(g * G + h) * D;
-            const float x0 = ldf(qp + c), x1 = ldf(qp + c + kHalf);
-            qs[h][c] = fmaf(x0, cs.x, -x1 * cs.y) * a.mscale;
-            qs[h][c + kHalf] = fmaf(x1, cs.x, x0 * cs.y) * a.mscale;
+            float y0 = 0.f, y1 = 0.f;
+            if (h < G) {
+                const float2 cs = rot[c];
+                const T *qp = reinterpret_cast<const T *>(a.q) + (int64_t)(g * G + h) * D;
+                const float x0 = ldf(qp + c), x1 = ldf(qp + c + kHalf);
+                y0 = fmaf(x0, cs.x, -x1 * cs.y) * a.mscale;
+                y1 = fmaf(x1, cs.x, x0 * cs.y) * a.mscale;
+            }
+            qs[h][c] = y0;
+            qs[h][c + kHalf] = y1;
         }
+        // the value rows go to shared memory for the value product
 #pragma unroll
         for (int j = 0; j < kPieces; ++j) {
-            const int u = tid + j * kDecodeThreads, r = u / kPiecesRow, pc = u - r * kPiecesRow;
-            constexpr int nv = Piece<T>::kVals;
-            float x[nv], y[nv];
+            float y[kVals];
+            unpack(vv[j], y, (const T *)nullptr);
+#pragma unroll
+            for (int e = 0; e < kVals; e += 4)
+                *reinterpret_cast<float4 *>(&vs[r0 + j * kRowStep][pc * kVals + e]) =
+                    make_float4(y[e], y[e + 1], y[e + 2], y[e + 3]);
+        }
+        __syncthreads();
+        // scores straight from the key pieces in registers: each thread forms the partial dot
+        // products of its kVals channels with all kMaxG heads, and the kPiecesRow lanes of a row
+        // add them up with a splitting butterfly (each exchange halves the heads a lane keeps:
+        // 4 + 2 + 1 shuffles, then plain sums over the remaining lane bits), after which lane
+        // pair ((lane >> (kLog - 3)) & 7) holds the full score of that head
+#pragma unroll
+        for (int j = 0; j < kPieces; ++j) {
+            float x[kVals];
             unpack(kh[j], x, (const T *)nullptr);
             if (LO) {
                 float lo8[8];
                 unpack(kl[j], lo8, (const __nv_bfloat16 *)nullptr);
 #pragma unroll
-                for (int e = 0; e < nv; ++e) x[e] += lo8[e];
+                for (int e = 0; e < kVals; ++e) x[e] += lo8[e];
             }
-            unpack(vv[j], y, (const T *)nullptr);
+            float sh[kMaxG];
 #pragma unroll
-            for (int e = 0; e < nv; e += 4) {
-                *reinterpret_cast<float4 *>(&ks[r][pc * nv + e]) = make_float4(x[e], x[e + 1], x[e + 2], x[e + 3]);
-                *reinterpret_cast<float4 *>(&vs[r][pc * nv + e]) = make_float4(y[e], y[e + 1], y[e + 2], y[e + 3]);
+            for (int h = 0; h < kMaxG; ++h) {
+                float acc = 0.f;
+#pragma unroll
+                for (int e = 0; e < kVals; e += 4) {
+                    const float4 q4 = *reinterpret_cast<const float4 *>(&qs[h][pc * kVals + e]);
+                    acc = fmaf(q4.x, x[e], fmaf(q4.y, x[e + 1], fmaf(q4.z, x[e + 2], fmaf(q4.w, x[e + 3], acc))));
+                }
+                sh[h] = acc;
             }
+            {
+                const bool b = (lane >> (kLog - 1)) & 1;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float send = b ? sh[i] : sh[i + 4], keep = b ? sh[i + 4] : sh[i];
+                    sh[i] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, 1 << (kLog - 1));
+                }
+            }
+            {
+                const bool b = (lane >> (kLog - 2)) & 1;
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    const float send = b ? sh[i] : sh[i + 2], keep = b ? sh[i + 2] : sh[i];
+                    sh[i] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, 1 << (kLog - 2));
+                }
+            }
+            {
+                const bool b = (lane >> (kLog - 3)) & 1;
+                const float send = b ? sh[0] : sh[1], keep = b ? sh[1] : sh[0];
+                sh[0] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, 1 << (kLog - 3));
+            }
+#pragma unroll
+            for (int o = 0; o < kLog - 3; ++o) sh[0] += __shfl_xor_sync(0xFFFFFFFFu, sh[0], 1 << o);
+            const int lr = lane & (kPiecesRow - 1);
+            const int h = ((lr >> (kLog - 1)) & 1) * 4 + ((lr >> (kLog - 2)) & 1) * 2 + ((lr >> (kLog - 3)) & 1);
+            if ((lr & ((1 << (kLog - 3)) - 1)) == 0 && h < G) sc[h][r0 + j * kRowStep] = sh[0];
         }
         __syncthreads();
-        // scores and the chunk's softmax: warp h takes query head h, lane r takes key r
+        // the chunk's softmax: warp h takes query head h, lane r takes key r
         if (warp < G) {
             const int h = warp, r = lane;
-            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll 8
-            for (int c = 0; c < D; c += 4) {
-                const float4 q4 = *reinterpret_cast<const float4 *>(&qs[h][c]);
-                const float4 k4 = *reinterpret_cast<const float4 *>(&ks[r][c]);
-                s0 = fmaf(q4.x, k4.x, s0);
-                s1 = fmaf(q4.y, k4.y, s1);
-                s2 = fmaf(q4.z, k4.z, s2);
-                s3 = fmaf(q4.w, k4.w, s3);
-            }
-            const float x = ((kbits >> r) & 1u) ? ((s0 + s1) + (s2 + s3)) * a.scale_log2 : -INFINITY;
+            const float x = ((kbits >> r) & 1u) ? sc[h][r] * a.scale_log2 : -INFINITY;
             float mx = x;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
@@ -213,7 +280,7 @@ __global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecode
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, o);
             ps[h][r] = p;
-            if (lane == 0) ml[h] = make_float2(mx, l);
+            if (lane == 0) a.part_ml[slot * G + h] = make_float2(mx, l);
         }
         __syncthreads();
         // value product: thread (channel c, head set hs) over heads hs, hs + step, ...
@@ -238,57 +305,20 @@ __global__ void __cluster_dims__(kDecodeCluster, 1, 1) __launch_bounds__(kDecode
 #pragma unroll
             for (int e = 0; e < kPer; ++e) {
                 const int h = hs + e * kStep;
-                if (h < G) os[h][c] = acc[e];
+                if (h < G) a.part_o[(slot * G + h) * D + c] = acc[e];
             }
         }
-    } else if (tid < kMaxG) {
-        ml[tid] = make_float2(-INFINITY, 0.f);
+    } else {
+        // a chunk with no key: an empty partial (weight 0 in the combine, finite outputs)
+        for (int idx = tid; idx < G * D; idx += kDecodeThreads) a.part_o[slot * G * D + idx] = 0.f;
+        if (tid < G) a.part_ml[slot * G + tid] = make_float2(-INFINITY, 0.f);
     }
-    cluster.sync();
-    if (cluster.block_rank() == 0) {
-        // merge the cluster's partials (distributed shared memory) into one
-        const int grp = chunk / kDecodeCluster;
-        const int64_t slot = (int64_t)g * a.n_groups + grp;
-        if (tid < G) {
-            float2 mr[kDecodeCluster];
-            float M = -INFINITY;
-#pragma unroll
-            for (int r = 0; r < kDecodeCluster; ++r) {
-                mr[r] = cluster.map_shared_rank(&ml[0], r)[tid];
-                M = fmaxf(M, mr[r].x);
-            }
-            float L = 0.f;
-#pragma unroll
-            for (int r = 0; r < kDecodeCluster; ++r) {
-                const float w = mr[r].x == -INFINITY ? 0.f : exp2f(mr[r].x - M);
-                wt[tid][r] = w;
-                L = fmaf(mr[r].y, w, L);
-            }
-            a.part_ml[slot * G + tid] = make_float2(M, L);
-        }
-        __syncthreads();
-        for (int idx = tid; idx < G * kQuarter; idx += kDecodeThreads) {
-            const int h = idx / kQuarter, c4 = (idx - h * kQuarter) * 4;
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-            for (int r = 0; r < kDecodeCluster; ++r) {
-                const float w = wt[h][r];
-                if (w == 0.f) continue;  // empty chunk: its outputs were never written
-                const float4 o = *reinterpret_cast<const float4 *>(cluster.map_shared_rank(&os[0][0], r) + h * D + c4);
-                acc.x = fmaf(o.x, w, acc.x);
-                acc.y = fmaf(o.y, w, acc.y);
-                acc.z = fmaf(o.z, w, acc.z);
-                acc.w = fmaf(o.w, w, acc.w);
-            }
-            *reinterpret_cast<float4 *>(a.part_o + (slot * G + h) * D + c4) = acc;
-        }
-    }
-    cluster.sync();  // the other CTAs' shared memory stays alive until the merge has read it
 }
 
 // One CTA per (query head, 32-channel slice); each of its 8 warps folds a strided subset of
-// the cluster partials with an online maximum, then the warps are merged in shared memory.
+// the chunk partials with an online maximum, then the warps are merged in shared memory.
 constexpr int kCombineWarps = 8;
+constexpr int kCombineBatch = 8;
 
 template <typename TO>
 __global__ void __launch_bounds__(kCombineWarps * 32) k_decode_combine(const DecodeArgs a)
@@ -300,19 +330,38 @@ __global__ void __launch_bounds__(kCombineWarps * 32) k_decode_combine(const Dec
     const int h = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int c = blockIdx.y * 32 + lane;
     const int g = h / a.G, hl = h - g * a.G;
-    const float2 *ml = a.part_ml + (int64_t)g * a.n_groups * a.G + hl;
-    const float *po = a.part_o + ((int64_t)g * a.n_groups * a.G + hl) * a.D + c;
+    const float2 *ml = a.part_ml + (int64_t)g * a.n_chunks * a.G + hl;
+    const float *po = a.part_o + ((int64_t)g * a.n_chunks * a.G + hl) * a.D + c;
+    // batches of kCombineBatch partials per warp: all loads of a batch are in flight before
+    // any is folded (one rescale per batch)
     float M = -INFINITY, L = 0.f, acc = 0.f;
-#pragma unroll 4
-    for (int i = warp; i < a.n_groups; i += kCombineWarps) {
-        const float2 mi = ml[(int64_t)i * a.G];
-        const float oi = po[(int64_t)i * a.G * a.D];
-        if (mi.x == -INFINITY) continue;
-        const float nm = fmaxf(M, mi.x);
-        const float so = exp2f(M - nm), si = exp2f(mi.x - nm);  // M = -inf gives so = 0
-        L = fmaf(L, so, mi.y * si);
-        acc = fmaf(acc, so, oi * si);
-        M = nm;
+    for (int i0 = warp; i0 < a.n_chunks; i0 += kCombineBatch * kCombineWarps) {
+        float2 mi[kCombineBatch];
+        float oi[kCombineBatch];
+#pragma unroll
+        for (int u = 0; u < kCombineBatch; ++u) {
+            const int i = i0 + u * kCombineWarps;
+            mi[u] = make_float2(-INFINITY, 0.f);
+            oi[u] = 0.f;
+            if (i < a.n_chunks) {
+                mi[u] = ml[(int64_t)i * a.G];
+                oi[u] = po[(int64_t)i * a.G * a.D];
+            }
+        }
+        float bm = M;
+#pragma unroll
+        for (int u = 0; u < kCombineBatch; ++u) bm = fmaxf(bm, mi[u].x);
+        if (bm == -INFINITY) continue;  // nothing kept so far
+        const float so = exp2f(M - bm);  // M = -inf gives 0
+        L *= so;
+        acc *= so;
+#pragma unroll
+        for (int u = 0; u < kCombineBatch; ++u) {
+            const float w = exp2f(mi[u].x - bm);  // an empty partial (-inf) weighs 0
+            L = fmaf(mi[u].y, w, L);
+            acc = fmaf(oi[u], w, acc);
+        }
+        M = bm;
     }
     if (lane == 0) {
         wm[warp] = M;
@@ -382,7 +431,6 @@ cudaError_t launch_partial(const DecodeArgs &a, int dtype, dim3 grid, cudaStream
 
 cudaError_t launch_decode(const DecodeArgs &a, int dtype, int out_dtype, cudaStream_t s)
 {
-    // n_chunks is a multiple of the cluster size (the host rounds it up)
     const dim3 grid_p((unsigned)a.n_chunks, (unsigned)a.Hkv);
     cudaError_t e = a.D == 128 ? launch_partial<128>(a, dtype, grid_p, s) : launch_partial<64>(a, dtype, grid_p, s);
     if (e != cudaSuccess) return e;

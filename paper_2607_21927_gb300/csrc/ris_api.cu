@@ -1069,8 +1069,7 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     // anchor chunks cover the longest list, window chunks a full window, whatever t is
     a.n_anchor_chunks = (int32_t)((anchor->max_keys + kDecodeChunk - 1) / kDecodeChunk);
     const int64_t chunks = a.n_anchor_chunks + ((int64_t)window + kDecodeChunk - 1) / kDecodeChunk;
-    a.n_groups = (int32_t)((chunks + kDecodeCluster - 1) / kDecodeCluster);
-    a.n_chunks = a.n_groups * kDecodeCluster;
+    a.n_chunks = (int32_t)chunks;
     double ms = 1.0;
     if (rope != nullptr && rope->kind != RIS_ROPE_NONE) RIS_TRY(ris_rope_freqs(rope, n_ctx, head_dim, a.f, &ms));
     a.mscale = (float)ms;
@@ -1079,7 +1078,7 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
     a.out = out;
     a.lse = lse;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    const size_t slots = (size_t)kv_heads * a.n_groups * a.G;
+    const size_t slots = (size_t)kv_heads * a.n_chunks * a.G;
     const size_t o_bytes = (sizeof(float) * slots * head_dim + 255) & ~size_t(255);
     const size_t need = o_bytes + sizeof(float2) * slots;
     if (need > anchor->scratch_bytes) {

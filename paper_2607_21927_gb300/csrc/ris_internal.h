@@ -108,7 +108,6 @@ struct AttnArgs {
 // positions, one CTA per (chunk, g). The grid does not depend on t, so t may be read from
 // device memory.
 constexpr int kDecodeChunk = 32;
-constexpr int kDecodeCluster = 8;  // chunks merged on chip per partial written
 constexpr int kMaxDecodeKvHeads = 64;
 
 struct DecodeArgs {
@@ -126,9 +125,8 @@ struct DecodeArgs {
     int32_t Hkv;
     int32_t G;
     int32_t D;
-    int32_t n_chunks;          // chunks per KV head (grid.x), a multiple of kDecodeCluster
+    int32_t n_chunks;          // chunks per KV head (grid.x): partials per KV head
     int32_t n_anchor_chunks;   // the first n_anchor_chunks chunks take anchor entries
-    int32_t n_groups;          // n_chunks / kDecodeCluster: partials per KV head
     int32_t window;            // W >= 1
     int32_t advance;           // with t_dev: the combine kernel adds 1 to *t_dev when done
     int64_t t;                 // position of the token (when t_dev is null)
@@ -137,8 +135,8 @@ struct DecodeArgs {
     double f[kMaxHeadDimHalf]; // rotation frequencies of q (fp64)
     float mscale;
     float scale_log2;          // log2(e) / sqrt(D)
-    float *part_o;             // [Hkv * n_groups][G][D] partial outputs
-    float2 *part_ml;           // [Hkv * n_groups][G] partial (max, sum) in the log2 domain
+    float *part_o;             // [Hkv * n_chunks][G][D] partial outputs
+    float2 *part_ml;           // [Hkv * n_chunks][G] partial (max, sum) in the log2 domain
     void *out;                 // [Hq][D]
     float *lse;                // [Hq] or null
 };
