@@ -15,15 +15,17 @@
 //   k_decode_partial : one CTA per (chunk of 32 keys, KV head): issues all of the chunk's
 //                      16-byte K~ (high + low parts) and V row loads at once, rotates the G
 //                      query heads of the KV head at position t (fp64 angle, as the prefill
-//                      RoPE) while they are in flight, takes the scores of all heads straight
-//                      from the key pieces in registers, and writes each head's partial
-//                      (max, sum, unnormalised output) to global memory.
+//                      RoPE) while they are in flight, takes the scores of all heads from the
+//                      key pieces in registers (bf16 caches: mma.sync with the pieces as B
+//                      fragments), and writes each head's partial (max, sum, unnormalised
+//                      output) to global memory, head-major.
 //   k_decode_combine : one CTA per (query head, 32 channels): rescales the chunk partials to
 //                      the global maximum, sums and normalises; optional natural-log LSE.
 //
-// A decode step is one query row: a GEMV-shaped product that reads each selected K/V row once,
-// so it runs on the FP32 pipes (no tensor-core tile to fill) and is bound by the K/V row
-// reads; fp32 scores and probabilities keep it well inside the bf16 tolerance.
+// A decode step is one query row: a GEMV-shaped step that reads each selected K/V row once and
+// is bound by the latency of the loads that find and fetch them. The scores of a chunk's 8 x 32
+// (head, key) pairs fit one small tensor-core product per key warp; probabilities and the value
+// product stay in fp32.
 #include <utility>
 #include <cuda_bf16.h>
 
@@ -38,7 +40,7 @@ namespace {
 
 __device__ unsigned int g_ris_decode_error;
 
-constexpr int kDecodeThreads = 256;  // eight warps: one per query head of the KV head
+constexpr int kDecodeThreads = 256;  // eight warps (the softmax: one per query head of the KV head)
 constexpr int kMaxG = 8;
 
 template <typename T>
@@ -63,6 +65,19 @@ __device__ __forceinline__ void prefetch_l2(const void *p, int bytes)
 {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(__cvta_generic_to_global(p)), "r"(bytes)
                  : "memory");
+}
+
+// d += A B on the tensor cores (m16n8k16, bf16 in, fp32 accumulate) with rows 8..15 of A zero:
+// a0 / a2 hold row lane/4 of A at columns 2(lane%4) + {0, 1} / + {8, 9}, b0 / b1 rows
+// 2(lane%4) + {0, 1} / + {8, 9} of B at column lane/4; d0 / d1 are row lane/4 of the product at
+// columns 2(lane%4) + {0, 1}.
+__device__ __forceinline__ void mma_bf16(float &d0, float &d1, float &d2, float &d3, uint32_t a0, uint32_t a2,
+                                         uint32_t b0, uint32_t b1)
+{
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+                 "{%0, %1, %2, %3};"
+                 : "+f"(d0), "+f"(d1), "+f"(d2), "+f"(d3)
+                 : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
 }
 
 // 16-byte row pieces of the staged K/V rows: bf16 holds 8 values per piece, fp32 holds 4.
@@ -96,7 +111,7 @@ __device__ __forceinline__ void unpack(const uint4 &u, float *o, const float *)
 // thread-block clusters and distributed shared memory measured slower: the cluster barriers
 // and the remote reads cost more than the combine kernel's extra partials.)
 template <typename T, bool LO, int D>
-__global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeArgs a)
+__global__ void __launch_bounds__(kDecodeThreads, 4) k_decode_partial(const DecodeArgs a)
 {
     constexpr int kPiecesRow = D * (int)sizeof(T) / 16;                   // 16-byte pieces per row
     constexpr int kPieces = kDecodeChunk * kPiecesRow / kDecodeThreads;  // per thread and plane
@@ -104,11 +119,21 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
     constexpr int kVals = Piece<T>::kVals;                               // values per piece
     constexpr int kRowStep = kDecodeThreads / kPiecesRow;                // rows between a thread's pieces
     constexpr int kLog = kPiecesRow == 8 ? 3 : kPiecesRow == 16 ? 4 : 5;  // log2(kPiecesRow)
+    // bf16 caches: scores on the tensor cores (mma m16n8k16), 4 key warps and 4 value warps
+    constexpr bool kTc = sizeof(T) == 2;
+    constexpr int kKSteps = D / 16;                 // k-steps of 16 head-dim columns
+    constexpr int kKQ = kKSteps / 2;                // key pieces per lane and plane
+    constexpr int kVRowStep = 128 / kPiecesRow;     // value rows between a value thread's pieces
+    constexpr int kVPieces = kDecodeChunk / kVRowStep;
+    static_assert(!kTc || (kDecodeChunk == 32 && kDecodeThreads == 256), "4 key warps of 8 keys, 4 value warps");
+    constexpr int kQItems = kMaxG * kHalf / kDecodeThreads;  // query rotation items per thread
+    static_assert(kMaxG * kHalf % kDecodeThreads == 0, "rotation items per thread");
     static_assert(kDecodeChunk * kPiecesRow % kDecodeThreads == 0, "pieces per thread");
     static_assert(kDecodeThreads % kPiecesRow == 0 && (1 << kLog) == kPiecesRow, "a row's pieces in one warp");
     static_assert(kMaxG == 8, "the score butterfly splits 8 heads");
     static_assert(D <= kDecodeThreads, "one thread per channel in the value product");
     __shared__ __align__(16) float qs[kMaxG][D];  // rotated query heads (rows G .. kMaxG-1 zero)
+    __shared__ __align__(16) __nv_bfloat16 qb[2][kMaxG][D + 8];  // the same as a bf16 high / low pair
     __shared__ __align__(16) float vs[kDecodeChunk][D];
     __shared__ float sc[kMaxG][kDecodeChunk];     // scores
     __shared__ __align__(16) float ps[kMaxG][kDecodeChunk];
@@ -120,6 +145,7 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
     const int g = blockIdx.y, chunk = blockIdx.x, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int pc = tid % kPiecesRow, r0 = tid / kPiecesRow;  // this thread's 16-byte column piece and first row
+    const int pcv = (tid & 127) % kPiecesRow, rv0 = (tid & 127) / kPiecesRow;  // the same for a value warp
     const int G = a.G;
     const int m = a.heads_keyed > 1 ? g : 0;
     const bool from_anchor = chunk < a.n_anchor_chunks;
@@ -146,6 +172,16 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
             prefetch_l2(reinterpret_cast<const T *>(a.v) + row, D * (int)sizeof(T));
         }
     }
+    // The rotation table of the query at the position as read now (each thread its own entry
+    // and its own read of the position; an entry is computed again after the wait if the
+    // position turns out to differ), so that its fp64 angles stay off the path after the wait.
+    int64_t t_rot = 0;
+    if (tid < kHalf) {
+        t_rot = a.t_dev != nullptr ? (int64_t)__ldcg(reinterpret_cast<const long long *>(a.t_dev)) : a.t;
+        float sn, cs;
+        sincos_reduced((double)t_rot * a.f[tid], &sn, &cs);
+        rot[tid] = make_float2(cs, sn);
+    }
     // Wait for the kernel before (the position, q, the anchor list of a fresh build and the
     // partials' buffer come after it), then let the next kernel be scheduled while this one runs.
     asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -155,6 +191,19 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
     if (from_anchor && tid < kDecodeChunk && k0 + tid < a.anchor_len[m])
         spec = __ldcg(a.anchor + a.anchor_base[m] + k0 + tid);
     const int64_t t = a.t_dev != nullptr ? *a.t_dev : a.t;
+    // this thread's query values (rotation items tid + i * kDecodeThreads), in the same round
+    float qx0[kQItems], qx1[kQItems];
+#pragma unroll
+    for (int i = 0; i < kQItems; ++i) {
+        const int idx = tid + i * kDecodeThreads, h = idx / kHalf, c = idx - h * kHalf;
+        qx0[i] = 0.f;
+        qx1[i] = 0.f;
+        if (h < G) {
+            const T *qp = reinterpret_cast<const T *>(a.q) + (int64_t)(g * G + h) * D;
+            qx0[i] = ldf(qp + c);
+            qx1[i] = ldf(qp + c + kHalf);
+        }
+    }
     const bool valid = t >= a.t0 && t < a.cache_len;  // only a device-side t can be outside
     if (!valid && tid == 0 && chunk == 0 && g == 0) atomicOr(&g_ris_decode_error, 2u);
     const int64_t win_lo = t - a.window + 1 > 0 ? t - a.window + 1 : 0;
@@ -169,9 +218,91 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
     __syncthreads();
     const uint32_t kbits = kept;
     const bool active = kbits != 0u;  // block-uniform
-    const int64_t slot = (int64_t)g * a.n_chunks + chunk;  // this CTA's partial
+    // partials are head-major: those of query head (g, h) are slots (g * G + h) * n_chunks + i
+    const int64_t slot0 = (int64_t)g * G * a.n_chunks + chunk;  // this CTA's slot for h = 0
+    const int64_t hstride = a.n_chunks;
 
     if (active) {
+      if constexpr (kTc) {
+        // bf16 cache: warps 0..3 load the chunk's key pieces in the mma B-fragment layout (warp
+        // w takes keys 8w .. 8w+7; lane l the key 8w + l/4 and its pieces 4q + l%4, which hold
+        // the stored head-dim columns of k-steps 2q and 2q+1 as the fragment wants them), warps
+        // 4..7 load the value rows; every load is issued before any is used
+        uint4 kb[kKQ], kbl[kKQ], vv[kVPieces];
+        if (warp < 4) {
+            const int64_t row = ((int64_t)keys[warp * 8 + (lane >> 2)] * a.Hkv + g) * D;
+            const uint4 *kp = reinterpret_cast<const uint4 *>(reinterpret_cast<const T *>(a.k) + row);
+            const uint4 *klp = reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(a.k_lo) + row);
+#pragma unroll
+            for (int q = 0; q < kKQ; ++q) {
+                kb[q] = __ldg(kp + 4 * q + (lane & 3));
+                if (LO) kbl[q] = __ldg(klp + 4 * q + (lane & 3));
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < kVPieces; ++j) {
+                const int64_t row = ((int64_t)keys[rv0 + j * kVRowStep] * a.Hkv + g) * D;
+                vv[j] = __ldg(reinterpret_cast<const uint4 *>(reinterpret_cast<const T *>(a.v) + row) + pcv);
+            }
+        }
+        // rotate the G query heads at position t while the rows are in flight, as a bf16 high
+        // + low pair (heads G .. kMaxG-1 zero)
+        if (tid < kHalf && t_rot != t) {
+            float sn, cs;
+            sincos_reduced((double)t * a.f[tid], &sn, &cs);
+            rot[tid] = make_float2(cs, sn);
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < kQItems; ++i) {
+            const int idx = tid + i * kDecodeThreads, h = idx / kHalf, c = idx - h * kHalf;
+            const float2 cs = rot[c];
+            const float y0 = fmaf(qx0[i], cs.x, -qx1[i] * cs.y) * a.mscale;  // heads >= G: zero
+            const float y1 = fmaf(qx1[i], cs.x, qx0[i] * cs.y) * a.mscale;
+            const __nv_bfloat16 h0 = __float2bfloat16_rn(y0), h1 = __float2bfloat16_rn(y1);
+            qb[0][h][c] = h0;
+            qb[1][h][c] = __float2bfloat16_rn(y0 - __bfloat162float(h0));
+            qb[0][h][c + kHalf] = h1;
+            qb[1][h][c + kHalf] = __float2bfloat16_rn(y1 - __bfloat162float(h1));
+        }
+        if (warp >= 4) {  // the value rows go to shared memory for the value product
+#pragma unroll
+            for (int j = 0; j < kVPieces; ++j) {
+                float y[8];
+                unpack(vv[j], y, (const __nv_bfloat16 *)nullptr);
+#pragma unroll
+                for (int e = 0; e < 8; e += 4)
+                    *reinterpret_cast<float4 *>(&vs[rv0 + j * kVRowStep][pcv * 8 + e]) =
+                        make_float4(y[e], y[e + 1], y[e + 2], y[e + 3]);
+            }
+        }
+        __syncthreads();
+        if (warp < 4) {
+            // scores of the 8 heads x 8 keys of this warp on the tensor cores: A = query (rows =
+            // heads, rows 8..15 zero), B = keys; q hi.k hi + q lo.k hi + q hi.k lo in fp32
+            const int hq = lane >> 2, c = lane & 3;
+            float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+#pragma unroll
+            for (int s = 0; s < kKSteps; ++s) {
+                const int off = 8 * (4 * (s >> 1) + c) + 4 * (s & 1);
+                const uint2 ah = *reinterpret_cast<const uint2 *>(&qb[0][hq][off]);
+                const uint2 al = *reinterpret_cast<const uint2 *>(&qb[1][hq][off]);
+                const uint32_t b0 = (s & 1) ? kb[s >> 1].z : kb[s >> 1].x;
+                const uint32_t b1 = (s & 1) ? kb[s >> 1].w : kb[s >> 1].y;
+                mma_bf16(d0, d1, d2, d3, ah.x, ah.y, b0, b1);
+                mma_bf16(d0, d1, d2, d3, al.x, al.y, b0, b1);
+                if (LO) {
+                    const uint32_t l0 = (s & 1) ? kbl[s >> 1].z : kbl[s >> 1].x;
+                    const uint32_t l1 = (s & 1) ? kbl[s >> 1].w : kbl[s >> 1].y;
+                    mma_bf16(d0, d1, d2, d3, ah.x, ah.y, l0, l1);
+                }
+            }
+            if (hq < G) {  // d0, d1: head hq, keys 8w + 2c and 8w + 2c + 1
+                sc[hq][warp * 8 + 2 * c] = d0;
+                sc[hq][warp * 8 + 2 * c + 1] = d1;
+            }
+        }
+      } else {
         // every row load of the chunk is issued before any is used; a thread's pieces are all
         // at the same column offset (pc), in rows r0, r0 + kRowStep, ...
         uint4 kh[kPieces], kl[kPieces], vv[kPieces];
@@ -184,22 +315,18 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
         }
         // rotate the G query heads at position t while the rows are in flight (heads G .. kMaxG-1
         // are zero, so that the score loop below runs over kMaxG heads without guards)
-        if (tid < kHalf) {
+        if (tid < kHalf && t_rot != t) {
             float sn, cs;
             sincos_reduced((double)t * a.f[tid], &sn, &cs);
             rot[tid] = make_float2(cs, sn);
         }
         __syncthreads();
-        for (int idx = tid; idx < kMaxG * kHalf; idx += kDecodeThreads) {
-            const int h = idx / kHalf, c = idx - h * kHalf;
-            float y0 = 0.f, y1 = 0.f;
-            if (h < G) {
-                const float2 cs = rot[c];
-                const T *qp = reinterpret_cast<const T *>(a.q) + (int64_t)(g * G + h) * D;
-                const float x0 = ldf(qp + c), x1 = ldf(qp + c + kHalf);
-                y0 = fmaf(x0, cs.x, -x1 * cs.y) * a.mscale;
-                y1 = fmaf(x1, cs.x, x0 * cs.y) * a.mscale;
-            }
+#pragma unroll
+        for (int i = 0; i < kQItems; ++i) {
+            const int idx = tid + i * kDecodeThreads, h = idx / kHalf, c = idx - h * kHalf;
+            const float2 cs = rot[c];
+            const float y0 = fmaf(qx0[i], cs.x, -qx1[i] * cs.y) * a.mscale;  // heads >= G: zero
+            const float y1 = fmaf(qx1[i], cs.x, qx0[i] * cs.y) * a.mscale;
             qs[h][c] = y0;
             qs[h][c + kHalf] = y1;
         }
@@ -267,6 +394,7 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
             const int h = ((lr >> (kLog - 1)) & 1) * 4 + ((lr >> (kLog - 2)) & 1) * 2 + ((lr >> (kLog - 3)) & 1);
             if ((lr & ((1 << (kLog - 3)) - 1)) == 0 && h < G) sc[h][r0 + j * kRowStep] = sh[0];
         }
+      }
         __syncthreads();
         // the chunk's softmax: warp h takes query head h, lane r takes key r
         if (warp < G) {
@@ -280,7 +408,7 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, o);
             ps[h][r] = p;
-            if (lane == 0) a.part_ml[slot * G + h] = make_float2(mx, l);
+            if (lane == 0) a.part_ml[slot0 + h * hstride] = make_float2(mx, l);
         }
         __syncthreads();
         // value product: thread (channel c, head set hs) over heads hs, hs + step, ...
@@ -305,22 +433,26 @@ __global__ void __launch_bounds__(kDecodeThreads) k_decode_partial(const DecodeA
 #pragma unroll
             for (int e = 0; e < kPer; ++e) {
                 const int h = hs + e * kStep;
-                if (h < G) a.part_o[(slot * G + h) * D + c] = acc[e];
+                if (h < G) a.part_o[(slot0 + h * hstride) * D + c] = acc[e];
             }
         }
     } else {
         // a chunk with no key: an empty partial (weight 0 in the combine, finite outputs)
-        for (int idx = tid; idx < G * D; idx += kDecodeThreads) a.part_o[slot * G * D + idx] = 0.f;
-        if (tid < G) a.part_ml[slot * G + tid] = make_float2(-INFINITY, 0.f);
+        for (int idx = tid; idx < G * D; idx += kDecodeThreads)
+            a.part_o[(slot0 + (idx / D) * hstride) * D + idx % D] = 0.f;
+        if (tid < G) a.part_ml[slot0 + tid * hstride] = make_float2(-INFINITY, 0.f);
     }
 }
 
-// One CTA per (query head, 32-channel slice); each of its 8 warps folds a strided subset of
-// the chunk partials with an online maximum, then the warps are merged in shared memory.
+// One CTA per (query head, 32-channel slice). Warp w takes the ranges of 32 consecutive
+// partials w, w + kCombineWarps, ...: lane j loads the (max, sum) of partial j of the range
+// while every lane loads the outputs of all 32 partials at its channel (head-major partials
+// are D floats apart, so the 32 loads are immediate offsets from one address), all in one
+// round; then the range's maximum, the lane's weight (broadcast by shuffle) and the fold.
+// The warps are merged in shared memory.
 constexpr int kCombineWarps = 8;
-constexpr int kCombineBatch = 8;
 
-template <typename TO>
+template <typename TO, int D>
 __global__ void __launch_bounds__(kCombineWarps * 32) k_decode_combine(const DecodeArgs a)
 {
     // a programmatic dependent of the partial kernel: wait for its partials
@@ -329,39 +461,35 @@ __global__ void __launch_bounds__(kCombineWarps * 32) k_decode_combine(const Dec
     __shared__ float wm[kCombineWarps], wl[kCombineWarps], wacc[kCombineWarps][32];
     const int h = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int c = blockIdx.y * 32 + lane;
-    const int g = h / a.G, hl = h - g * a.G;
-    const float2 *ml = a.part_ml + (int64_t)g * a.n_chunks * a.G + hl;
-    const float *po = a.part_o + ((int64_t)g * a.n_chunks * a.G + hl) * a.D + c;
-    // batches of kCombineBatch partials per warp: all loads of a batch are in flight before
-    // any is folded (one rescale per batch)
-    float M = -INFINITY, L = 0.f, acc = 0.f;
-    for (int i0 = warp; i0 < a.n_chunks; i0 += kCombineBatch * kCombineWarps) {
-        float2 mi[kCombineBatch];
-        float oi[kCombineBatch];
+    const int n = a.n_chunks;
+    const float2 *ml = a.part_ml + (int64_t)h * n;  // query head h = g * G + hl: slots h * n + i
+    const float *po = a.part_o + (int64_t)h * n * D + c;
+    float M = -INFINITY, L = 0.f, acc = 0.f;  // the same M and L in every lane of the warp
+    for (int r0 = warp * 32; r0 < n; r0 += kCombineWarps * 32) {
+        const int cnt = n - r0 < 32 ? n - r0 : 32;
+        const float2 mv = lane < cnt ? ml[r0 + lane] : make_float2(-INFINITY, 0.f);
+        const float *pb = po + (int64_t)r0 * D;
+        float oi[32];
 #pragma unroll
-        for (int u = 0; u < kCombineBatch; ++u) {
-            const int i = i0 + u * kCombineWarps;
-            mi[u] = make_float2(-INFINITY, 0.f);
+        for (int u = 0; u < 32; ++u) {
             oi[u] = 0.f;
-            if (i < a.n_chunks) {
-                mi[u] = ml[(int64_t)i * a.G];
-                oi[u] = po[(int64_t)i * a.G * a.D];
-            }
+            if (u < cnt) oi[u] = pb[u * D];
         }
-        float bm = M;
+        float bm = mv.x;
 #pragma unroll
-        for (int u = 0; u < kCombineBatch; ++u) bm = fmaxf(bm, mi[u].x);
-        if (bm == -INFINITY) continue;  // nothing kept so far
-        const float so = exp2f(M - bm);  // M = -inf gives 0
-        L *= so;
+        for (int o = 16; o > 0; o >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xFFFFFFFFu, bm, o));
+        const float nm = fmaxf(M, bm);
+        if (nm == -INFINITY) continue;  // warp-uniform: nothing kept so far
+        const float so = exp2f(M - nm);  // M = -inf gives 0
+        M = nm;
+        const float w = exp2f(mv.x - M);  // this lane's partial; an empty one (-inf) weighs 0
+        float lw = w * mv.y;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) lw += __shfl_xor_sync(0xFFFFFFFFu, lw, o);
+        L = fmaf(L, so, lw);
         acc *= so;
 #pragma unroll
-        for (int u = 0; u < kCombineBatch; ++u) {
-            const float w = exp2f(mi[u].x - bm);  // an empty partial (-inf) weighs 0
-            L = fmaf(mi[u].y, w, L);
-            acc = fmaf(oi[u], w, acc);
-        }
-        M = bm;
+        for (int u = 0; u < 32; ++u) acc = fmaf(oi[u], __shfl_sync(0xFFFFFFFFu, w, u), acc);
     }
     if (lane == 0) {
         wm[warp] = M;
@@ -377,15 +505,15 @@ __global__ void __launch_bounds__(kCombineWarps * 32) k_decode_combine(const Dec
 #pragma unroll
         for (int w = 0; w < kCombineWarps; ++w) {
             if (wm[w] == -INFINITY) continue;
-            const float s = exp2f(wm[w] - Mt);
-            Lt = fmaf(wl[w], s, Lt);
-            o = fmaf(wacc[w][lane], s, o);
+            const float sw = exp2f(wm[w] - Mt);
+            Lt = fmaf(wl[w], sw, Lt);
+            o = fmaf(wacc[w][lane], sw, o);
         }
         o /= Lt;
         if constexpr (sizeof(TO) == 4)
-            reinterpret_cast<float *>(a.out)[(int64_t)h * a.D + c] = o;
+            reinterpret_cast<float *>(a.out)[(int64_t)h * D + c] = o;
         else
-            reinterpret_cast<__nv_bfloat16 *>(a.out)[(int64_t)h * a.D + c] = __float2bfloat16_rn(o);
+            reinterpret_cast<__nv_bfloat16 *>(a.out)[(int64_t)h * D + c] = __float2bfloat16_rn(o);
         if (lane == 0 && blockIdx.y == 0 && a.lse != nullptr) a.lse[h] = (Mt + log2f(Lt)) * 0.69314718055994530942f;
         // the partial kernel, the only reader of t, has finished: move to the next position
         if (a.advance && a.t_dev != nullptr && h == 0 && blockIdx.y == 0 && lane == 0) *a.t_dev += 1;
@@ -435,8 +563,12 @@ cudaError_t launch_decode(const DecodeArgs &a, int dtype, int out_dtype, cudaStr
     cudaError_t e = a.D == 128 ? launch_partial<128>(a, dtype, grid_p, s) : launch_partial<64>(a, dtype, grid_p, s);
     if (e != cudaSuccess) return e;
     const dim3 grid_c((unsigned)a.Hq, (unsigned)(a.D / 32));
-    e = out_dtype == RIS_F32 ? launch_pdl(k_decode_combine<float>, grid_c, dim3(kCombineWarps * 32), s, a)
-                             : launch_pdl(k_decode_combine<__nv_bfloat16>, grid_c, dim3(kCombineWarps * 32), s, a);
+    if (a.D == 128)
+        e = out_dtype == RIS_F32 ? launch_pdl(k_decode_combine<float, 128>, grid_c, dim3(kCombineWarps * 32), s, a)
+                                 : launch_pdl(k_decode_combine<__nv_bfloat16, 128>, grid_c, dim3(kCombineWarps * 32), s, a);
+    else
+        e = out_dtype == RIS_F32 ? launch_pdl(k_decode_combine<float, 64>, grid_c, dim3(kCombineWarps * 32), s, a)
+                                 : launch_pdl(k_decode_combine<__nv_bfloat16, 64>, grid_c, dim3(kCombineWarps * 32), s, a);
     note_launch(2);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();

@@ -135,8 +135,8 @@ struct DecodeArgs {
     double f[kMaxHeadDimHalf]; // rotation frequencies of q (fp64)
     float mscale;
     float scale_log2;          // log2(e) / sqrt(D)
-    float *part_o;             // [Hkv * n_chunks][G][D] partial outputs
-    float2 *part_ml;           // [Hkv * n_chunks][G] partial (max, sum) in the log2 domain
+    float *part_o;             // [Hq][n_chunks][D] partial outputs (query head g * G + h)
+    float2 *part_ml;           // [Hq][n_chunks] partial (max, sum) in the log2 domain
     void *out;                 // [Hq][D]
     float *lse;                // [Hq] or null
 };
