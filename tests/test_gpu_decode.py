@@ -109,6 +109,13 @@ def test_decode_small_bf16_out_and_tinyllama_shape():
     _decode_case(500, 620, 32, 4, 64, torch.bfloat16, 1, 0.02, [7, 8], [500, 555, 619], 32, theta=1e4, native=64)
 
 
+@pytest.mark.parametrize("Hq,Hkv,D", [(4, 4, 128), (6, 2, 64), (15, 3, 128)], ids=["mha_G1", "G3_d64", "G5"])
+def test_decode_bf16_query_groups(Hq, Hkv, D):
+    """Groups smaller than the 8 rows the score product carries (the other rows are zero)."""
+    _decode_case(350, 420, Hq, Hkv, D, torch.bfloat16, 0, 0.05, [3, 4], [350, 377, 419], 24,
+                 out_dtype=torch.float32)
+
+
 def test_decode_fp32_path():
     _decode_case(257, 400, 4, 4, 64, torch.float32, 0, 0.1, [1], [257, 300, 399], 20, rope_kind=1, outliers=False)
 
