@@ -23,9 +23,9 @@
 //                      the global maximum, sums and normalises; optional natural-log LSE.
 //
 // A decode step is one query row: a GEMV-shaped step that reads each selected K/V row once and
-// is bound by the latency of the loads that find and fetch them. The scores of a chunk's 8 x 32
-// (head, key) pairs fit one small tensor-core product per key warp; probabilities and the value
-// product stay in fp32.
+// is bound by the latency of the loads that find and fetch them. For bf16 caches the scores
+// (8 heads x 32 keys) and the value product (8 heads x D channels over 32 keys) are small
+// tensor-core products with fp32 accumulation; the softmax is fp32.
 #include <utility>
 #include <cuda_bf16.h>
 
@@ -78,6 +78,16 @@ __device__ __forceinline__ void mma_bf16(float &d0, float &d1, float &d2, float 
                  "{%0, %1, %2, %3};"
                  : "+f"(d0), "+f"(d1), "+f"(d2), "+f"(d3)
                  : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+}
+
+// B operand of mma m16n8k16 from a row-major [k][n] bf16 tile in shared memory: lanes 0..7
+// give the addresses of rows k = 0..7, lanes 8..15 of rows 8..15 (8 columns from n0 each).
+__device__ __forceinline__ void ldmatrix_x2_trans(uint32_t &b0, uint32_t &b1, const void *row)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];"
+                 : "=r"(b0), "=r"(b1)
+                 : "r"((uint32_t)__cvta_generic_to_shared(row))
+                 : "memory");
 }
 
 // 16-byte row pieces of the staged K/V rows: bf16 holds 8 values per piece, fp32 holds 4.
@@ -134,7 +144,9 @@ __global__ void __launch_bounds__(kDecodeThreads, 4) k_decode_partial(const Deco
     static_assert(D <= kDecodeThreads, "one thread per channel in the value product");
     __shared__ __align__(16) float qs[kMaxG][D];  // rotated query heads (rows G .. kMaxG-1 zero)
     __shared__ __align__(16) __nv_bfloat16 qb[2][kMaxG][D + 8];  // the same as a bf16 high / low pair
-    __shared__ __align__(16) float vs[kDecodeChunk][D];
+    __shared__ __align__(16) float vs[kDecodeChunk][D];               // fp32 caches: value rows
+    __shared__ __align__(16) __nv_bfloat16 vb[kDecodeChunk][D + 8];   // bf16 caches: value rows
+    __shared__ __align__(16) __nv_bfloat16 pb[2][kMaxG][kDecodeChunk + 8];  // bf16 caches: P high / low
     __shared__ float sc[kMaxG][kDecodeChunk];     // scores
     __shared__ __align__(16) float ps[kMaxG][kDecodeChunk];
     __shared__ float2 rot[kHalf];                 // (cos, sin) of t * f_c
@@ -265,16 +277,10 @@ __global__ void __launch_bounds__(kDecodeThreads, 4) k_decode_partial(const Deco
             qb[0][h][c + kHalf] = h1;
             qb[1][h][c + kHalf] = __float2bfloat16_rn(y1 - __bfloat162float(h1));
         }
-        if (warp >= 4) {  // the value rows go to shared memory for the value product
+        if (warp >= 4) {  // the value rows go to shared memory as they are (bf16)
 #pragma unroll
-            for (int j = 0; j < kVPieces; ++j) {
-                float y[8];
-                unpack(vv[j], y, (const __nv_bfloat16 *)nullptr);
-#pragma unroll
-                for (int e = 0; e < 8; e += 4)
-                    *reinterpret_cast<float4 *>(&vs[rv0 + j * kVRowStep][pcv * 8 + e]) =
-                        make_float4(y[e], y[e + 1], y[e + 2], y[e + 3]);
-            }
+            for (int j = 0; j < kVPieces; ++j)
+                *reinterpret_cast<uint4 *>(&vb[rv0 + j * kVRowStep][pcv * 8]) = vv[j];
         }
         __syncthreads();
         if (warp < 4) {
@@ -407,12 +413,41 @@ __global__ void __launch_bounds__(kDecodeThreads, 4) k_decode_partial(const Deco
             float l = p;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, o);
-            ps[h][r] = p;
+            if constexpr (kTc) {  // P as a bf16 high + low pair, the A operand of the value product
+                const __nv_bfloat16 ph = __float2bfloat16_rn(p);
+                pb[0][h][r] = ph;
+                pb[1][h][r] = __float2bfloat16_rn(p - __bfloat162float(ph));
+            } else {
+                ps[h][r] = p;
+            }
             if (lane == 0) a.part_ml[slot0 + h * hstride] = make_float2(mx, l);
         }
         __syncthreads();
+        if constexpr (kTc) {
+            // value product on the tensor cores: A = P (heads x keys, hi + lo), B = V (keys x
+            // channels, read transposed by ldmatrix); warp w takes the channel tiles of 8
+            // columns w * kNT .. w * kNT + kNT - 1 and stores its rows of the partial
+            constexpr int kNT = D / 64;
+            const int hq = lane >> 2, c = lane & 3;
+#pragma unroll
+            for (int nt = 0; nt < kNT; ++nt) {
+                const int n0 = (warp * kNT + nt) * 8;
+                float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+#pragma unroll
+                for (int ks = 0; ks < kDecodeChunk / 16; ++ks) {
+                    uint32_t b0, b1;
+                    ldmatrix_x2_trans(b0, b1, &vb[ks * 16 + (lane & 15)][n0]);
+                    const int k = ks * 16 + 2 * c;
+                    mma_bf16(d0, d1, d2, d3, *reinterpret_cast<const uint32_t *>(&pb[0][hq][k]),
+                             *reinterpret_cast<const uint32_t *>(&pb[0][hq][k + 8]), b0, b1);
+                    mma_bf16(d0, d1, d2, d3, *reinterpret_cast<const uint32_t *>(&pb[1][hq][k]),
+                             *reinterpret_cast<const uint32_t *>(&pb[1][hq][k + 8]), b0, b1);
+                }
+                if (hq < G)
+                    *reinterpret_cast<float2 *>(&a.part_o[(slot0 + hq * hstride) * D + n0 + 2 * c]) = make_float2(d0, d1);
+            }
+        } else {
         // value product: thread (channel c, head set hs) over heads hs, hs + step, ...
-        {
             constexpr int kStep = kDecodeThreads / D;
             constexpr int kPer = (kMaxG + kStep - 1) / kStep;
             const int c = tid % D, hs = tid / D;
