@@ -129,7 +129,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 4) k_decode_partial(const Deco
     constexpr int kVals = Piece<T>::kVals;                               // values per piece
     constexpr int kRowStep = kDecodeThreads / kPiecesRow;                // rows between a thread's pieces
     constexpr int kLog = kPiecesRow == 8 ? 3 : kPiecesRow == 16 ? 4 : 5;  // log2(kPiecesRow)
-    // bf16 caches: scores on the tensor cores (mma m16n8k16), 4 key warps and 4 value warps
+    // bf16 caches: score and value products on the tensor cores (mma m16n8k16); 4 warps load
+    // the keys, 4 the value rows
     constexpr bool kTc = sizeof(T) == 2;
     constexpr int kKSteps = D / 16;                 // k-steps of 16 head-dim columns
     constexpr int kKQ = kKSteps / 2;                // key pieces per lane and plane
@@ -309,8 +310,8 @@ __global__ void __launch_bounds__(kDecodeThreads, 4) k_decode_partial(const Deco
             }
         }
       } else {
-        // every row load of the chunk is issued before any is used; a thread's pieces are all
-        // at the same column offset (pc), in rows r0, r0 + kRowStep, ...
+        // fp32 caches: every row load of the chunk is issued before any is used; a thread's
+        // pieces are all at the same column offset (pc), in rows r0, r0 + kRowStep, ...
         uint4 kh[kPieces], kl[kPieces], vv[kPieces];
 #pragma unroll
         for (int j = 0; j < kPieces; ++j) {
