@@ -324,6 +324,29 @@ def test_yarn_frequency_bands_and_mscale(oracle):
     assert ms == pytest.approx(1.0 + 0.1 * math.log(2.0), rel=1e-15)
 
 
+def test_yarn_mid_band_hand_worked(oracle):
+    """A frequency inside YaRN's ramp, worked by hand from Peng et al. 2023 (NTK-by-parts,
+    alpha = 1, beta = 32): head dim 8, base 1e4, native window L = 64, N = 256 (s = 4).
+    Pair 0 has base frequency 1, wavelength 2 pi, so r = 64 / (2 pi) = 10.18591636 rotations per
+    window; the ramp gives gamma = (r - 1) / 31 = 0.29631988 and the frequency
+    (1 - gamma) * 1/4 + gamma * 1 = 0.47223991. Pair 1 (base 0.1, r = 1.01859164) sits just
+    inside the ramp: gamma = 0.00059973, frequency 0.02504498. The temperature is
+    0.1 ln 4 + 1 = 1.13862944. A unit vector rotated at position p turns by p times the
+    frequency and is scaled by the temperature."""
+    D, N = 8, 256
+    cfg = oracle.RopeCfg(kind=3, theta=1e4, native_len=64)
+    hand_f = {0: 0.47223991188, 1: 0.02504497976}
+    hand_ms = 1.13862943611
+    for c, f in hand_f.items():
+        x = np.zeros((2, 1, D))
+        x[:, 0, c] = 1.0
+        y = oracle.rope(x, [1.0, 3.0], cfg, N)
+        for row, p in enumerate((1.0, 3.0)):
+            a, b = y[row, 0, c], y[row, 0, c + D // 2]
+            assert math.hypot(a, b) == pytest.approx(hand_ms, abs=1e-10)
+            assert math.atan2(b, a) == pytest.approx(p * f, abs=1e-10)
+
+
 @pytest.mark.parametrize("kind", [1, 2, 3])
 def test_rope_norm_and_relative_position(oracle, kind):
     """Each rotated pair keeps its norm (times mscale), and <R(p)q, R(p')k> depends on p - p' only."""
