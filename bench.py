@@ -794,12 +794,13 @@ def main():
                         "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
                         "design_frac": (dense / (tc * 1e12)) / (mean_ms / 1e3),
                         "design_note": "dense-causal tile FLOPs / sustained bf16 peak over the launch time (the "
-                                       "kernel issues 2.5x that in hi/lo split products)"})
+                                       "kernel issues 2x that: three score products for the hi/lo splits of "
+                                       "q and k, one value product)"})
             if rope is not None and w["dtype"] == "bf16":
-                # rotated bf16 inputs: three score products (q hi/lo x k hi/lo) and two value
-                # products (P hi/lo) per tile, all of them tensor-core work the kernel issues
-                ent["issued_frac"] = 2.5 * ent["design_frac"]
-                ent["issued_note"] = ("issued bf16 tensor-core FLOPs (5 products of 128x128x128 per causal tile "
+                # rotated bf16 inputs: three score products (q hi/lo x k hi/lo) and one value
+                # product (fp16 P against fp16 values) per tile, all of them tensor-core work
+                ent["issued_frac"] = 2.0 * ent["design_frac"]
+                ent["issued_note"] = ("issued 16-bit tensor-core FLOPs (4 products of 128x128x128 per causal tile "
                                       "pair) / sustained bf16 peak over the launch time")
         else:
             # gathered pairs: all of them, or with the dense-suffix split all but the suffixes

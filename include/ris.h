@@ -234,19 +234,26 @@ ris_status ris_attention_masked_rows(ris_mask_t mask, int64_t row_begin, int64_t
 ris_status ris_row_split(const int64_t *row_ptr, int64_t N, int32_t parts, int64_t *bounds);
 ris_status ris_mask_row_split(ris_mask_t mask, int32_t parts, int64_t *bounds);
 
-/* Allocation-free variant of ris_attention_masked (same arguments, results and errors).
+/* Allocation-free variant of ris_attention_masked: same arguments and the same results
+ * within the parity tolerance (not bit for bit), with these differences.
  * The paper has no counterpart: this entry point exists for callers that may not allocate
  * device memory while a layer runs, such as an inference engine's enqueue callback that may
  * only launch work, or a server that plans all device memory at load time. They build the
  * mask once beforehand (ris_mask_generate allocates) and call this per layer.
- * Instead of the stream-ordered pool, the rotated q (fp32) and k (bf16 hi + lo, or fp32)
- * live in one library-owned device array of 64 MiB per device, which every GPU that uses
- * this entry point holds until the process exits. The call needs
- *   align256(N*heads*head_dim*4) + (bf16 ? 2 : 1) * align256(N*kv_heads*head_dim*(bf16 ? 2 : 4))
- * bytes when rope is set (none without rope) and returns RIS_ERR_INVALID, launching nothing,
- * when that exceeds 64 MiB (about N = 9300 tokens at 12 / 2 heads of 128). It calls no
- * allocation routine. The first call on a device looks up the array's device address (and
- * may load the library's device code): make that first call before any stream capture.
+ *   - Every mask runs on the register gather (fp32: the fp32 gather), whatever design
+ *     ris_attention_masked would pick: dense and high-density masks run at gather speed, not
+ *     on the tiles, and heads / kv_heads above 8 are refused (RIS_ERR_UNSUPPORTED).
+ *   - Instead of the stream-ordered pool, the rotated q (fp32) and k (bf16 hi + lo, or fp32)
+ *     live in one library-owned device array of 64 MiB per device. Every GPU on which the
+ *     library's device code is loaded holds it until the process exits: with lazy module
+ *     loading (the CUDA default) the GPUs on which a kernel of this library ran, with
+ *     CUDA_MODULE_LOADING=EAGER every context that loads the library. The call needs
+ *       align256(N*heads*head_dim*4) + (bf16 ? 2 : 1) * align256(N*kv_heads*head_dim*(bf16 ? 2 : 4))
+ *     bytes when rope is set (none without rope) and returns RIS_ERR_INVALID, launching
+ *     nothing, when that exceeds 64 MiB (about N = 9300 tokens at 12 / 2 heads of 128).
+ * It calls no allocation routine. The first call in a device's context looks up the array's
+ * device address (and may load the library's device code): make that first call before any
+ * stream capture; a context created anew (after cudaDeviceReset) is looked up again.
  * Every call on a device shares the array and leaves its contents behind; each call writes
  * all scratch it reads, so nothing needs clearing, but calls whose GPU work overlaps (e.g.
  * on two streams) race on it and must be ordered by the caller. */
@@ -254,6 +261,11 @@ ris_status ris_attention_masked_noalloc(ris_mask_t mask, const void *q, const vo
                                         void *out, int32_t heads, int32_t kv_heads, int32_t head_dim,
                                         int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
                                         float *lse, void *stream);
+
+/* The allocation-free entry point's scratch array in the current device's context: its
+ * device address and size in bytes (the paper has no counterpart). Looks the address up like
+ * the entry point's first call does. Errors: RIS_ERR_INVALID (NULL outputs), RIS_ERR_CUDA. */
+ris_status ris_noalloc_scratch_info(void **device_address, int64_t *bytes);
 
 /* Kernel timer for measurement (off by default). While enabled, every attention kernel launch
  * (the fused QK^T -> softmax -> PV kernel of a layer, or a decode step's two kernels; not
@@ -288,6 +300,30 @@ int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim);
  * a word skips the rest of its work, so outputs of that launch are undefined. Blocks.
  * Errors: RIS_ERR_CUDA. */
 ris_status ris_device_status(void *stream);
+
+/* Release the library's cached per-device state (the paper has no counterpart): the kernel
+ * timer's events, and the device memory that the stream-ordered pools of the devices this
+ * library used keep cached (each pool is trimmed and its release threshold set back to the
+ * CUDA default, 0). The allocation-free entry point's scratch array is a static device
+ * array: it stays mapped until the process exits, and its address is looked up again on the
+ * next call. Live masks and anchors stay valid and are still released by ris_mask_free /
+ * ris_anchor_free. Testing switches (ris_debug_*) are reset. The library may be used again
+ * afterwards. Call it with no library work in flight on any stream. Errors: RIS_ERR_CUDA. */
+ris_status ris_shutdown(void);
+
+/* ---- Failure injection for tests (the paper has no counterpart) ---------------------------
+ * ris_debug_fail_allocation: the n-th stream-ordered device allocation the library makes from
+ * now on (0 = the next one) fails as if the pool were exhausted; later ones succeed again.
+ * n < 0 disarms. Every entry point must then return RIS_ERR_OOM, leave its output handle NULL
+ * and release, on its stream, whatever it had allocated.
+ * ris_debug_tile_stall: with no_loads = 1 the tile kernel's loader issues no copies, so its
+ * first wait on them gives up after wait_limit_cycles (0 = the default, about 2^31 cycles):
+ * the kernel sets its device error word, releases its tensor memory and returns, and
+ * ris_device_status reports RIS_ERR_DEVICE_TIMEOUT (outputs of that launch are undefined).
+ * no_loads = 0 with a nonzero limit only shortens the waits. (0, 0) restores the defaults.
+ * Both switches are process-wide. Errors: RIS_ERR_INVALID. */
+ris_status ris_debug_fail_allocation(int64_t n);
+ris_status ris_debug_tile_stall(int32_t no_loads, int64_t wait_limit_cycles);
 
 /* ---- Hybrid Anchor decode (Methods, "Hybrid Anchor and Pre-Fusion Unified Softmax (PFUS)") ----
  * After a prefill of n_prefill tokens, the token generated at position t >= t0 = n_prefill

@@ -63,6 +63,15 @@ __device__ __forceinline__ int key_at(const TIdx *cols, int64_t pos)
     return (int)cols[pos];
 }
 
+// Power-of-two exponent E that brings the values into fp16's range for the value product
+// (v / 2^E with |v| / 2^E < 2^14): 0 unless the largest |v| is 2^14 or more. The conversion
+// kernel and the tile kernel's epilogue take E from the same max, so they agree exactly.
+__device__ __forceinline__ int v_scale_exp(float vmax)
+{
+    const int e = (int)((__float_as_uint(vmax) >> 23) & 0xFF) - 127;  // floor(log2 vmax) for normal vmax
+    return e >= 14 ? e - 13 : 0;
+}
+
 __device__ __forceinline__ float warp_max(float x)
 {
 #pragma unroll

@@ -9,11 +9,19 @@
 //
 // The rotated queries (fp32) and keys (bf16 hi + lo, or fp32) that ris_attention_masked
 // takes from the stream-ordered pool live here in one file-scope device array of
-// kNoAllocScratchBytes. Every GPU on which this library's copy of the array is used holds
-// it until the process exits. The array is shared by every call on a device and keeps the
+// kNoAllocScratchBytes. Every GPU on which this library's device code is loaded holds it
+// until the process exits: with the default lazy module loading only GPUs on which this
+// entry point (or another kernel of the library) ran, with CUDA_MODULE_LOADING=EAGER every
+// context that loads the library. The array is shared by every call on a device and keeps the
 // last call's contents; this entry point writes every byte it later reads within the same
 // call, so nothing has to be cleared, but calls whose work overlaps on the GPU (for
 // example on two streams) race on it and must be ordered by the caller.
+//
+// Every layer runs on the register gather (or the fp32 gather), whatever design
+// ris_attention_masked would pick: the tile and dense-suffix designs need more scratch
+// (the suffix pass's partial outputs) than the array holds at useful sizes. The results
+// agree with ris_attention_masked within the parity tolerance, not bit for bit.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -51,29 +59,79 @@ ris_status na_fail(ris_status st, const char *fmt, ...)
     return st;
 }
 
-// Device address of the scratch array for the current device, looked up once per device
-// (host code must not use the array's name as an address).
+// Unique ID of the calling thread's current CUDA context (0 if none or unknown). Context
+// IDs are never reused within a process, unlike context handles.
+unsigned long long current_context_id()
+{
+    using GetCurrent = CUresult (*)(CUcontext *);
+    using GetId = CUresult (*)(CUcontext, unsigned long long *);
+    static std::once_flag once;
+    static GetCurrent get_current = nullptr;
+    static GetId get_id = nullptr;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<GetCurrent>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<GetId>(p);
+    });
+    CUcontext c = nullptr;
+    unsigned long long id = 0;
+    if (get_current == nullptr || get_id == nullptr || get_current(&c) != CUDA_SUCCESS || c == nullptr) return 0;
+    if (get_id(c, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
+
+// Device address of the scratch array in the current device's context (host code must not
+// use the array's name as an address). The lookup is made once per (device, context): a
+// context torn down and created again (cudaDeviceReset, then later use) maps the array at a
+// new address, so a cached address is reused only while the same context is current.
+std::mutex g_addr_mu;
+void *g_addr[64] = {nullptr};
+unsigned long long g_ctx_of[64] = {0};
+
 ris_status scratch_address(void **out)
 {
-    static std::mutex mu;
-    static void *addr[64] = {nullptr};
+    std::mutex &mu = g_addr_mu;
+    void **addr = g_addr;
+    unsigned long long *ctx_of = g_ctx_of;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return na_fail(RIS_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
     if (dev < 0 || dev >= 64) return na_fail(RIS_ERR_UNSUPPORTED, "device ordinal %d >= 64", dev);
     std::lock_guard<std::mutex> lk(mu);
-    if (addr[dev] == nullptr) {
+    const unsigned long long ctx = current_context_id();
+    if (addr[dev] == nullptr || ctx == 0 || ctx != ctx_of[dev]) {
         void *p = nullptr;
         e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
         if (e != cudaSuccess || p == nullptr) {
             cudaGetLastError();
+            addr[dev] = nullptr;
             return na_fail(RIS_ERR_CUDA, "cudaGetSymbolAddress(scratch): %s", cudaGetErrorString(e));
         }
         addr[dev] = p;
+        ctx_of[dev] = current_context_id();  // the lookup has made the runtime's context current
     }
     *out = addr[dev];
     return RIS_OK;
 }
+
+}  // namespace
+
+void noalloc_forget_addresses()
+{
+    std::lock_guard<std::mutex> lk(g_addr_mu);
+    for (int d = 0; d < 64; ++d) {
+        g_addr[d] = nullptr;
+        g_ctx_of[d] = 0;
+    }
+}
+
+namespace {
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
@@ -179,4 +237,12 @@ extern "C" ris_status ris_attention_masked_noalloc(ris_mask_t mask, const void *
                         : launch_attention_f32(a, head_dim, out_dtype, md.col_bytes, md.dense != 0, s);
     if (e != cudaSuccess) return na_fail(RIS_ERR_CUDA, "attention: %s", cudaGetErrorString(e));
     return RIS_OK;
+}
+
+extern "C" ris_status ris_noalloc_scratch_info(void **device_address, int64_t *bytes)
+{
+    if (device_address == nullptr || bytes == nullptr) return na_fail(RIS_ERR_INVALID, "output pointer is NULL");
+    *device_address = nullptr;
+    *bytes = (int64_t)kNoAllocScratchBytes;
+    return scratch_address(device_address);
 }

@@ -44,6 +44,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include <cstdint>
 #include <mutex>
@@ -59,8 +60,18 @@ namespace {
 
 constexpr int BM = 128;          // query rows per tile (TMEM lanes)
 constexpr int BN = 128;          // keys per stage
-constexpr int kThreads = 320;    // warps 0-7 softmax (two column halves), 8 TMA, 9 MMA
-constexpr int kTmaWarp = 8, kMmaWarp = 9;
+// Softmax: kRowThreads threads per query row, each owning BN / kRowThreads score columns of
+// every tile and DT / kRowThreads output columns; 4 warps cover the 128 TMEM lanes, so there
+// are 4 * kRowThreads softmax warps (four per SM sub-partition, to hide the latency of each
+// warp's dependent TMEM load -> max exchange -> exp -> TMEM store chain), then the TMA and MMA warps.
+constexpr int kRowThreads = 2;
+// P as one fp16 (11 significant bits, one value product against fp16 values) instead of a
+// bf16 hi + lo pair (two value products against bf16 values)
+constexpr bool kP16 = true;
+constexpr int kSoftmaxWarps = 4 * kRowThreads;
+constexpr int kSoftmaxThreads = 32 * kSoftmaxWarps;
+constexpr int kTmaWarp = kSoftmaxWarps, kMmaWarp = kSoftmaxWarps + 1;
+constexpr int kThreads = 32 * (kSoftmaxWarps + 2);
 constexpr uint32_t kTmemCols = 512;  // S/P[2] (2 x 128) + O (128) + Q hi / lo (2 x 64)
 
 // shared-memory map (bytes, from a 1024-aligned base) for head dim DT (128 or 64)
@@ -79,8 +90,8 @@ constexpr int SMEM_BYTES = OFF_K + kStages * (Smem<128>::K_STAGE + Smem<128>::V_
 
 // P_FULL and PV_DONE have one barrier per P buffer (tile parity), so that no waiter can fall
 // two phases behind a barrier it polls by parity.
-// B_X: per pair of softmax warps sharing rows (columns 0-31 / 32-63) and tile parity, the
-// exchange of their partial row maxima (and at the end their partial sums).
+// B_X: per group of kRowThreads softmax warps sharing rows (one per column quarter) and tile
+// parity, the exchange of their partial row maxima (and at the end their partial sums).
 enum Bar {
     B_Q = 0, B_K_FULL = 1, B_K_EMPTY = 3, B_V_FULL = 5, B_V_EMPTY = 7, B_S_FULL = 9, B_S_EMPTY = 11, B_P_FULL = 13,
     B_PV_DONE = 15, B_X = 17, B_END = 25, NBAR = 26
@@ -122,13 +133,14 @@ __device__ __forceinline__ bool mbar_wait_own(uint32_t bar, uint32_t parity)
     return true;
 }
 
-// Bounded wait (about 2^31 cycles); false if the phase did not complete in time.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
+// Bounded wait (`limit` cycles, about 2^31 unless a test lowers it); false if the phase did
+// not complete in time or another CTA already gave up.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long long limit)
 {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (!mbar_try_wait(bar, parity)) {
-        if (clock64() - t0 > (1LL << 31)) return false;
+        if (clock64() - t0 > limit) return false;
         if (*reinterpret_cast<volatile unsigned int *>(&g_ris_tile_error) != 0u) return false;
     }
     return true;
@@ -157,6 +169,15 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t addr, uint32_t lbo, uint32_t 
     d |= (uint64_t)1 << 46;  // descriptor version
     d |= (uint64_t)2 << 61;  // 128-byte swizzle
     return d;
+}
+
+// Instruction descriptor, kind::f16: fp16 x fp16 -> f32, dense.
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool b_mn_major)
+{
+    return (1u << 4)                      // D format f32 (A and B format 0: fp16)
+           | ((b_mn_major ? 1u : 0u) << 16)
+           | ((uint32_t)(N >> 3) << 17)
+           | ((uint32_t)(M >> 4) << 24);
 }
 
 // Instruction descriptor, kind::f16: bf16 x bf16 -> f32, dense.
@@ -250,6 +271,45 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float *v)
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
+// 32 lanes x 16 consecutive 32-bit columns, loaded and waited for in one statement.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float *v)
+{
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Two 16-column stores (32 lanes each) and one wait for both.
+__device__ __forceinline__ void tmem_st16x2(uint32_t ta, const uint32_t *a, uint32_t tb, const uint32_t *b)
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17};\n\t"
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%1], {%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33};\n\t"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(ta), "r"(tb),
+        "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(a[4]), "r"(a[5]), "r"(a[6]), "r"(a[7]), "r"(a[8]), "r"(a[9]),
+        "r"(a[10]), "r"(a[11]), "r"(a[12]), "r"(a[13]), "r"(a[14]), "r"(a[15]),
+        "r"(b[0]), "r"(b[1]), "r"(b[2]), "r"(b[3]), "r"(b[4]), "r"(b[5]), "r"(b[6]), "r"(b[7]), "r"(b[8]), "r"(b[9]),
+        "r"(b[10]), "r"(b[11]), "r"(b[12]), "r"(b[13]), "r"(b[14]), "r"(b[15])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t *v)
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(v[0]), "r"(v[1]),
+        "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *v)
 {
     asm volatile(
@@ -259,6 +319,48 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *v)
         "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
         : "memory");
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_st32u(uint32_t taddr, const uint32_t *v)
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+        "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]), "r"(v[17]), "r"(v[18]),
+        "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]),
+        "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// NC consecutive 32-bit columns (64, 32 or 16) of 32 lanes, loaded and waited for.
+template <int NC>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float *v)
+{
+    if constexpr (NC == 64)
+        tmem_ld64(taddr, v);
+    else if constexpr (NC == 32)
+        tmem_ld32(taddr, v);
+    else {
+        static_assert(NC == 16, "64, 32 or 16 columns");
+        tmem_ld16(taddr, v);
+    }
+}
+
+// NC consecutive 32-bit columns (32, 16 or 8) of 32 lanes, stored and waited for.
+template <int NC>
+__device__ __forceinline__ void tmem_st_words(uint32_t taddr, const uint32_t *w)
+{
+    if constexpr (NC == 32)
+        tmem_st32u(taddr, w);
+    else if constexpr (NC == 16)
+        tmem_st16(taddr, w);
+    else {
+        static_assert(NC == 8, "32, 16 or 8 columns");
+        tmem_st8(taddr, w);
+    }
 }
 
 // 2^x by the SFU (ex2.approx, relative error about 2^-22, subnormal results flushed to 0);
@@ -313,11 +415,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr int KV_ARR = Smem<DT>::KV_ARR, K_STAGE = Smem<DT>::K_STAGE, V_STAGE = Smem<DT>::V_STAGE;
     constexpr int OFF_V = OFF_K + kStages * K_STAGE;
     constexpr int NB = DT / 64;  // 64-column blocks of a row
-    constexpr int HALF = DT / 2; // head-dim columns of one softmax thread (one of two per row)
     extern __shared__ unsigned char smem_raw[];
     __shared__ __align__(8) uint64_t bars[NBAR];
     __shared__ uint32_t tmem_base_sh;
-    __shared__ float xch[2][2][BM];  // [tile parity][column half][row]
+    __shared__ float xch[2][kRowThreads][BM];  // [tile parity][column quarter][row]
     unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                             ~uintptr_t(1023));
     const uint32_t sbase = smem_u32(smem);
@@ -342,8 +443,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < NBAR; ++i) {
             uint32_t cnt = 1;
-            if (i == B_Q || i == B_S_EMPTY || i == B_S_EMPTY + 1 || i == B_P_FULL || i == B_P_FULL + 1) cnt = 256;
-            if (i >= B_X && i < B_END) cnt = 64;
+            if (i == B_Q || i == B_S_EMPTY || i == B_S_EMPTY + 1 || i == B_P_FULL || i == B_P_FULL + 1)
+                cnt = kSoftmaxThreads;
+            if (i >= B_X && i < B_END) cnt = 32 * kRowThreads;
             mbar_init(smem_u32(&bars[i]), cnt);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -360,11 +462,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
     const uint32_t t_s0 = tmem, t_s1 = tmem + BN, t_o = tmem + 2 * BN, t_q = tmem + 2 * BN + DT;
+    const long long wl = a.wait_limit > 0 ? (long long)a.wait_limit : (1LL << 31);
     bool ok = true;
 
     if (warp == kTmaWarp) {
         // =============================== TMA producer
-        if (lane == 0) {
+        if (lane == 0 && a.debug_no_loads == 0) {
             // tile j: keys once the score products of tile j - 2 are done, then values once the
             // value product of tile j - 2 is (it was issued after the score products of tile
             // j - 1, whose keys are already in flight: no wait here depends on a later load)
@@ -372,7 +475,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int j = 0; j < n_kt && ok; ++j) {
                 const int st = j % kStages;
                 const uint32_t par = ((j / kStages) - 1) & 1;
-                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_K_EMPTY + st]), par);
+                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_K_EMPTY + st]), par, wl);
                 if (!ok) break;
                 const uint32_t bk = smem_u32(&bars[B_K_FULL + st]);
                 const uint32_t dk = sbase + OFF_K + st * K_STAGE;
@@ -382,7 +485,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (SPLIT) tma_load_3d(dk + KV_ARR + blk * KV_BLK, &maps.kl, 64 * blk, g, (kt0 + j) * BN, bk);
                 }
                 nk = j + 1;
-                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_V_EMPTY + st]), par);
+                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_V_EMPTY + st]), par, wl);
                 if (!ok) break;
                 const uint32_t bv = smem_u32(&bars[B_V_FULL + st]);
                 const uint32_t dv = sbase + OFF_V + st * V_STAGE;
@@ -401,8 +504,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // =============================== MMA issuer
         if (lane == 0) {
             constexpr uint32_t ID_S = idesc_bf16(BM, BN, false);  // S[128 x 128] = Q K^T, both K-major
-            constexpr uint32_t ID_O = idesc_bf16(BM, DT, true);   // O[128 x 128] += P V, V MN-major
-            ok = mbar_wait(smem_u32(&bars[B_Q]), 0);
+            // O[128 x DT] += P V, V MN-major (fp16 P against fp16 values, or bf16 P hi / lo
+            // against bf16 values)
+            constexpr uint32_t ID_O = kP16 ? idesc_f16(BM, DT, true) : idesc_bf16(BM, DT, true);
+            ok = mbar_wait(smem_u32(&bars[B_Q]), 0, wl);
             tc_fence_after();
             auto issue_s = [&](int j) {
                 const int st = j & 1;
@@ -427,10 +532,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             auto issue_o = [&](int j) {
                 const int st = j % kStages;
                 const uint32_t vb = sbase + OFF_V + st * V_STAGE;
-                // P hi / lo of this tile sit in TMEM over its score columns: 128 keys of 16-bit
-                // values packed two per column, hi in columns 0-63, lo in 64-127
+                // P of this tile sits in TMEM over its score columns: 128 keys of 16-bit values
+                // packed two per column, in columns 0-63 (fp16 P, or the bf16 hi part) and 64-127
+                // (the bf16 lo part)
                 const uint32_t pt = (j & 1) ? t_s1 : t_s0;
-                for (int prod = 0; prod < 2; ++prod) {
+                for (int prod = 0; prod < (kP16 ? 1 : 2); ++prod) {
                     for (int ks = 0; ks < BN / 16; ++ks) {
                         // V block: 64 keys x 128 B rows; 16 keys = two 8-row atoms (SBO 1024);
                         // the second 64-column block of head dim is LBO = 8 KB away
@@ -443,22 +549,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             };
             for (int j = 0; j < n_kt && ok; ++j) {
                 const int st = j & 1;
-                ok = mbar_wait(smem_u32(&bars[B_K_FULL + j % kStages]), (j / kStages) & 1);
-                if (ok && j >= 2) ok = mbar_wait(smem_u32(&bars[B_S_EMPTY + st]), ((j >> 1) - 1) & 1);
+                ok = mbar_wait(smem_u32(&bars[B_K_FULL + j % kStages]), (j / kStages) & 1, wl);
+                if (ok && j >= 2) ok = mbar_wait(smem_u32(&bars[B_S_EMPTY + st]), ((j >> 1) - 1) & 1, wl);
                 if (!ok) break;
                 tc_fence_after();
                 issue_s(j);
                 if (j >= 1) {
-                    ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((j - 1) & 1)]), ((j - 1) >> 1) & 1);
-                    if (ok) ok = mbar_wait(smem_u32(&bars[B_V_FULL + (j - 1) % kStages]), ((j - 1) / kStages) & 1);
+                    ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((j - 1) & 1)]), ((j - 1) >> 1) & 1, wl);
+                    if (ok) ok = mbar_wait(smem_u32(&bars[B_V_FULL + (j - 1) % kStages]), ((j - 1) / kStages) & 1, wl);
                     if (!ok) break;
                     tc_fence_after();
                     issue_o(j - 1);
                 }
             }
             if (ok) {
-                ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1);
-                if (ok) ok = mbar_wait(smem_u32(&bars[B_V_FULL + (n_kt - 1) % kStages]), ((n_kt - 1) / kStages) & 1);
+                ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1, wl);
+                if (ok) ok = mbar_wait(smem_u32(&bars[B_V_FULL + (n_kt - 1) % kStages]), ((n_kt - 1) / kStages) & 1, wl);
                 if (ok) {
                     tc_fence_after();
                     issue_o(n_kt - 1);
@@ -469,9 +575,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait_own(smem_u32(&bars[B_END]), 0);
         }
     } else {
-        // =============================== softmax: two threads per query row q0 + r, one per
-        // column half hf (scores 64 hf .. 64 hf + 63 of each tile, O columns 64 hf .. 64 hf + 63)
-        const int wq = warp & 3, hf = warp >> 2;
+        // =============================== softmax: kRowThreads threads per query row q0 + r,
+        // thread cq owning score columns SC cq .. SC cq + SC - 1 of every tile and output
+        // columns OC cq .. OC cq + OC - 1
+        constexpr int SC = BN / kRowThreads;   // scores of a tile per thread (64 or 32)
+        constexpr int OC = DT / kRowThreads;   // output columns per thread (64, 32 or 16)
+        constexpr int OCH = OC < 32 ? OC : 32; // output columns per TMEM access
+        const int wq = warp & 3, cq = warp >> 2;
         const int r = wq * 32 + lane;  // TMEM lane
         const int64_t i = q0 + r;
         const bool row_ok = i >= a.row0 && i < a.row1;
@@ -481,11 +591,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int64_t last_word = i >> 5;
         const float sc = a.scale_log2;
         float m_used = -INFINITY, l = 0.f;
-        // bitmap word e (0, 1) of keys 128 (kt0 + j) + 64hf + 32e .. +31 of this row, fetched
-        // one tile ahead
+        // bitmap word e of keys 128 (kt0 + j) + SC cq + 32 e .. +31 of this row, fetched one
+        // tile ahead
         auto mask_word = [&](int j, int e) -> uint32_t {
             if (!row_ok) return 0u;
-            const int64_t k0 = (int64_t)(kt0 + j) * BN + 64 * hf + 32 * e;
+            const int64_t k0 = (int64_t)(kt0 + j) * BN + SC * cq + 32 * e;
             if (SUFFIX) {  // the row's dense suffix: offsets lo .. hi of the word
                 const int64_t lo = dense_suffix_start(a, i) - k0, hi = i - k0;
                 if (hi < 0 || lo > 31) return 0u;
@@ -500,77 +610,86 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int64_t wd = k0 >> 5;
             return wd <= last_word ? bm[wd] : 0u;
         };
-        // exchange a value with the partner thread of the other column half (bounded wait)
-        auto exchange = [&](int tag, float v, float &other) -> bool {
+        // exchange a value with the other threads of the row (bounded wait); v[q] = the value of
+        // column part q, in the same order for every thread of the row
+        auto exchange = [&](int tag, float mine, float *v) -> bool {
             const int pb = tag & 1;
-            xch[pb][hf][r] = v;
+            xch[pb][cq][r] = mine;
             const uint32_t bar = smem_u32(&bars[B_X + 2 * wq + pb]);
             mbar_arrive(bar);
-            const bool got = __all_sync(0xFFFFFFFFu, mbar_wait(bar, (tag >> 1) & 1));
-            other = xch[pb][hf ^ 1][r];
+            const bool got = __all_sync(0xFFFFFFFFu, mbar_wait(bar, (tag >> 1) & 1, wl));
+#pragma unroll
+            for (int qq = 0; qq < kRowThreads; ++qq) v[qq] = xch[pb][qq][r];
             return got;
         };
-        // this thread's half row of the query tile (head-dim HALF hf .. HALF hf + HALF - 1,
-        // DT / 4 packed columns) into TMEM
+        // this thread's part of the query row (head-dim OC cq .. OC cq + OC - 1, OC / 2 packed
+        // columns of each of hi and lo) into TMEM
         {
-            uint32_t qw[DT / 4];
-            const int64_t qrow = ((row_ok ? i : 0) * a.Hq + h) * DT + HALF * hf;
+            uint32_t qw[OC / 2];
+            const int64_t qrow = ((row_ok ? i : 0) * a.Hq + h) * DT + OC * cq;
             for (int part = 0; part < (SPLIT ? 2 : 1); ++part) {
                 const uint4 *src = reinterpret_cast<const uint4 *>(
                     reinterpret_cast<const __nv_bfloat16 *>(part == 0 ? q_hi : q_lo) + qrow);
 #pragma unroll
-                for (int u = 0; u < DT / 16; ++u) {
+                for (int u = 0; u < OC / 8; ++u) {
                     const uint4 x = row_ok ? src[u] : make_uint4(0u, 0u, 0u, 0u);
                     qw[4 * u] = x.x;
                     qw[4 * u + 1] = x.y;
                     qw[4 * u + 2] = x.z;
                     qw[4 * u + 3] = x.w;
                 }
+                const uint32_t tq = t_q + lane_off + (DT / 2) * part + (OC / 2) * cq;
 #pragma unroll
-                for (int w16 = 0; w16 < DT / 64; ++w16)
-                    tmem_st16(t_q + lane_off + (DT / 2) * part + (DT / 4) * hf + 16 * w16, qw + 16 * w16);
+                for (int c = 0; c < OC / 2; c += (OC / 2 < 16 ? OC / 2 : 16))
+                    tmem_st_words<(OC / 2 < 16 ? OC / 2 : 16)>(tq + c, qw + c);
             }
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_Q]));
         }
-        uint32_t cw0 = mask_word(0, 0), cw1 = mask_word(0, 1);
+        uint32_t cw[SC / 32];
+#pragma unroll
+        for (int e = 0; e < SC / 32; ++e) cw[e] = mask_word(0, e);
         for (int j = 0; j < n_kt; ++j) {
             const int st = j & 1;
-            const uint32_t nw0 = (j + 1 < n_kt) ? mask_word(j + 1, 0) : 0u;
-            const uint32_t nw1 = (j + 1 < n_kt) ? mask_word(j + 1, 1) : 0u;
-            ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&bars[B_S_FULL + st]), (j >> 1) & 1));
+            uint32_t nw[SC / 32];
+#pragma unroll
+            for (int e = 0; e < SC / 32; ++e) nw[e] = (j + 1 < n_kt) ? mask_word(j + 1, e) : 0u;
+            ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&bars[B_S_FULL + st]), (j >> 1) & 1, wl));
             if (!ok) break;
             tc_fence_after();
-            float sv[64];
-            const uint32_t sb = ((j & 1) ? t_s1 : t_s0) + lane_off + 64 * hf;
-            tmem_ld64(sb, sv);
+            float sv[SC];
+            const uint32_t sb = ((j & 1) ? t_s1 : t_s0) + lane_off + SC * cq;
+            tmem_ld_cols<SC>(sb, sv);
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_S_EMPTY + st]));
 
             // mask, partial row max as a tree (the scale is positive: it is applied to the max
-            // and folded into the exponent of P), then the full row max with the partner
+            // and folded into the exponent of P), then the full row max from the other threads
 #pragma unroll
-            for (int c = 0; c < 32; ++c) {
-                sv[c] = ((cw0 >> c) & 1u) ? sv[c] : -INFINITY;
-                sv[32 + c] = ((cw1 >> c) & 1u) ? sv[32 + c] : -INFINITY;
+            for (int e = 0; e < SC / 32; ++e) {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) sv[32 * e + c] = ((cw[e] >> c) & 1u) ? sv[32 * e + c] : -INFINITY;
+                cw[e] = nw[e];
             }
-            cw0 = nw0;
-            cw1 = nw1;
             float mx8[8];
 #pragma unroll
-            for (int e = 0; e < 8; ++e)
-                mx8[e] = fmaxf(fmaxf(fmaxf(sv[e], sv[e + 8]), fmaxf(sv[e + 16], sv[e + 24])),
-                               fmaxf(fmaxf(sv[e + 32], sv[e + 40]), fmaxf(sv[e + 48], sv[e + 56])));
+            for (int e = 0; e < 8; ++e) {
+                mx8[e] = sv[e];
+#pragma unroll
+                for (int c = e + 8; c < SC; c += 8) mx8[e] = fmaxf(mx8[e], sv[c]);
+            }
             const float pm = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                                    fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * sc;
-            float om;
-            ok = exchange(j, pm, om);
+            float pms[kRowThreads];
+            ok = exchange(j, pm, pms);
             if (!ok) break;
-            const float mx = fmaxf(pm, om);
-            // Lazy rescale: a row rescales O only when its max grows by more than 2^8 (both
-            // halves see the same max and decide alike). The TMEM loads / stores are
-            // warp-collective (.sync.aligned), so the whole warp runs them when any of its rows
-            // needs it; the other rows multiply by 1.
+            float mx = pms[0];
+#pragma unroll
+            for (int qq = 1; qq < kRowThreads; ++qq) mx = fmaxf(mx, pms[qq]);
+            // Lazy rescale: a row rescales O only when its max grows by more than 2^8 (all
+            // threads of the row see the same max and decide alike). The TMEM loads / stores
+            // are warp-collective (.sync.aligned), so the whole warp runs them when any of its
+            // rows needs it; the other rows multiply by 1.
             const bool upd = mx > m_used + 8.f;
             const float al = upd ? (m_used == -INFINITY ? 0.f : exp2f(m_used - mx)) : 1.f;
             if (upd) {
@@ -581,67 +700,91 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // O must have settled: the value product of tile j - 1 has to be done
                 if (j >= 1) {
                     ok = __all_sync(0xFFFFFFFFu,
-                                    mbar_wait(smem_u32(&bars[B_PV_DONE + ((j - 1) & 1)]), ((j - 1) >> 1) & 1));
+                                    mbar_wait(smem_u32(&bars[B_PV_DONE + ((j - 1) & 1)]), ((j - 1) >> 1) & 1, wl));
                     if (!ok) break;
                 }
                 tc_fence_after();
-                float ov[32];
 #pragma unroll
-                for (int c4 = 0; c4 < HALF / 32; ++c4) {
-                    tmem_ld32(t_o + lane_off + HALF * hf + 32 * c4, ov);
+                for (int c0 = 0; c0 < OC; c0 += OCH) {
+                    float ov[OCH];
+                    uint32_t ow[OCH];
+                    tmem_ld_cols<OCH>(t_o + lane_off + OC * cq + c0, ov);
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) ov[c] *= al;
-                    tmem_st32(t_o + lane_off + HALF * hf + 32 * c4, ov);
+                    for (int c = 0; c < OCH; ++c) ow[c] = __float_as_uint(ov[c] * al);
+                    tmem_st_words<OCH>(t_o + lane_off + OC * cq + c0, ow);
                 }
             }
             const float mu = (m_used == -INFINITY) ? 0.f : m_used;
-            // P = exp2(s - m_used) split as hi = p with its low 16 bits cleared (exactly a bf16)
-            // and lo = p - hi rounded to bf16 (p to ~16 significant bits with one conversion per
-            // pair), written into TMEM over this tile's score columns (both halves have read
-            // their scores: the max exchange came first) as the A operand of the value product:
-            // keys 64 hf .. 64 hf + 63 as hi in columns 32 hf .. +31 and lo in 64 + 32 hf .. +31
+            // P = exp2(s - m_used), written into TMEM over this tile's score columns (every
+            // thread of the row has read its scores: the max exchange came first) as the A
+            // operand of the value product, keys SC cq .. SC cq + SC - 1 in packed columns
+            // (SC / 2) cq .. (SC / 2) cq + SC / 2 - 1 (and the bf16 lo part 64 columns on).
+            // fp16 P: the row sum adds P as rounded, so that the rounding of each weight moves
+            // the output by at most 2^-11 of the weight times |v_j - o| (a normalised average
+            // of the values with slightly perturbed weights). bf16 pair: hi = p with its low 16
+            // bits cleared (exactly a bf16), lo = p - hi rounded to bf16 (~16 significant bits).
             float lsum[4] = {0.f, 0.f, 0.f, 0.f};
-            uint32_t hw[32], lw[32];
+            uint32_t hw[SC / 2];
+            const uint32_t pt = ((j & 1) ? t_s1 : t_s0) + lane_off;
+            if constexpr (kP16) {
 #pragma unroll
-            for (int w = 0; w < 32; ++w) {
-                const float p0 = ex2(fmaf(sv[2 * w], sc, -mu)), p1 = ex2(fmaf(sv[2 * w + 1], sc, -mu));
-                lsum[w & 3] += p0 + p1;
-                const uint32_t b0 = __float_as_uint(p0), b1 = __float_as_uint(p1);
-                hw[w] = __byte_perm(b0, b1, 0x7632);
-                lw[w] = pack_bf16(p0 - __uint_as_float(b0 & 0xFFFF0000u), p1 - __uint_as_float(b1 & 0xFFFF0000u));
+                for (int w = 0; w < SC / 2; ++w) {
+                    const float p0 = ex2(fmaf(sv[2 * w], sc, -mu)), p1 = ex2(fmaf(sv[2 * w + 1], sc, -mu));
+                    const __half2 hp = __floats2half2_rn(p0, p1);
+                    const float2 pr = __half22float2(hp);
+                    lsum[w & 3] += pr.x + pr.y;
+                    hw[w] = *reinterpret_cast<const uint32_t *>(&hp);
+                }
+#pragma unroll
+                for (int c = 0; c < SC / 2; c += 16) tmem_st16(pt + (SC / 2) * cq + c, hw + c);
+            } else {
+                uint32_t lw[SC / 2];
+#pragma unroll
+                for (int w = 0; w < SC / 2; ++w) {
+                    const float p0 = ex2(fmaf(sv[2 * w], sc, -mu)), p1 = ex2(fmaf(sv[2 * w + 1], sc, -mu));
+                    lsum[w & 3] += p0 + p1;
+                    const uint32_t b0 = __float_as_uint(p0), b1 = __float_as_uint(p1);
+                    hw[w] = __byte_perm(b0, b1, 0x7632);
+                    lw[w] = pack_bf16(p0 - __uint_as_float(b0 & 0xFFFF0000u), p1 - __uint_as_float(b1 & 0xFFFF0000u));
+                }
+#pragma unroll
+                for (int c = 0; c < SC / 2; c += 16)
+                    tmem_st16x2(pt + (SC / 2) * cq + c, hw + c, pt + BN / 2 + (SC / 2) * cq + c, lw + c);
             }
             l += (lsum[0] + lsum[1]) + (lsum[2] + lsum[3]);
-            const uint32_t pt = ((j & 1) ? t_s1 : t_s0) + lane_off;
-            tmem_st32x2(pt + 32 * hf, hw, pt + 64 + 32 * hf, lw);
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_P_FULL + st]));
         }
-        float ol = 0.f;
-        if (ok) ok = exchange(n_kt, l, ol);
+        float ls[kRowThreads];
+        if (ok) ok = exchange(n_kt, l, ls);
         if (ok)
             ok = __all_sync(0xFFFFFFFFu,
-                            mbar_wait(smem_u32(&bars[B_PV_DONE + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1));
+                            mbar_wait(smem_u32(&bars[B_PV_DONE + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1, wl));
         if (ok) {
             tc_fence_after();
-            const float lt = l + ol;
-            const float inv = lt > 0.f ? 1.f / lt : 0.f;
-            TOut *out = SUFFIX ? reinterpret_cast<TOut *>(a.part_o + ((row_ok ? i : 0) * a.Hq + h) * DT + HALF * hf)
-                               : reinterpret_cast<TOut *>(a.out) + (((int64_t)s * a.N + (row_ok ? i : 0)) * a.Hq + h) * DT +
-                                     HALF * hf;
-            float ov[32];
+            float lt = 0.f;
 #pragma unroll
-            for (int c4 = 0; c4 < HALF / 32; ++c4) {
-                tmem_ld32(t_o + lane_off + HALF * hf + 32 * c4, ov);
+            for (int qq = 0; qq < kRowThreads; ++qq) lt += ls[qq];
+            // fp16 values were scaled by 2^-E for the value product
+            const float vs = kP16 ? __uint_as_float((uint32_t)(127 + v_scale_exp(*a.v_absmax)) << 23) : 1.f;
+            const float inv = lt > 0.f ? vs / lt : 0.f;
+            TOut *out = SUFFIX ? reinterpret_cast<TOut *>(a.part_o + ((row_ok ? i : 0) * a.Hq + h) * DT + OC * cq)
+                               : reinterpret_cast<TOut *>(a.out) + (((int64_t)s * a.N + (row_ok ? i : 0)) * a.Hq + h) * DT +
+                                     OC * cq;
+#pragma unroll
+            for (int c0 = 0; c0 < OC; c0 += OCH) {
+                float ov[OCH];
+                tmem_ld_cols<OCH>(t_o + lane_off + OC * cq + c0, ov);
                 if (row_ok) {
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) ov[c] *= inv;
+                    for (int c = 0; c < OCH; ++c) ov[c] *= inv;
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) store8<TOut>(out + 32 * c4 + 8 * e, ov + 8 * e);
+                    for (int e = 0; e < OCH / 8; ++e) store8<TOut>(out + c0 + 8 * e, ov + 8 * e);
                 }
             }
             if (SUFFIX) {
-                if (row_ok && hf == 0) a.part_lse[i * a.Hq + h] = m_used + __log2f(lt);
-            } else if (row_ok && hf == 0 && a.lse != nullptr) {
+                if (row_ok && cq == 0) a.part_lse[i * a.Hq + h] = m_used + __log2f(lt);
+            } else if (row_ok && cq == 0 && a.lse != nullptr) {
                 a.lse[((int64_t)s * a.Hq + h) * a.N + i] = (m_used + __log2f(lt)) * kLn2;
             }
         }
@@ -670,8 +813,9 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-// [N][H][DT] bf16 viewed as 3D (d, head, token); box = 64 d x 1 head x `rows` tokens.
-bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows, int DT)
+// [N][H][DT] 16-bit values (bf16, or fp16 with f16 set) viewed as 3D (d, head, token); box =
+// 64 d x 1 head x `rows` tokens.
+bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows, int DT, bool f16 = false)
 {
     auto fn = encode_fn();
     if (fn == nullptr) return false;
@@ -679,7 +823,8 @@ bool make_map3(CUtensorMap *m, const void *base, int64_t N, int H, int rows, int
     cuuint64_t strides[2] = {(cuuint64_t)DT * 2, (cuuint64_t)H * DT * 2};
     cuuint32_t box[3] = {64, 1, (cuuint32_t)rows};
     cuuint32_t estr[3] = {1, 1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
+    return fn(m, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base),
+              dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -715,10 +860,14 @@ cudaError_t read_tile_error(unsigned int *out)
     return cudaMemcpyToSymbol(g_ris_tile_error, &zero, sizeof(unsigned int));
 }
 
-// K / V tensor maps of a call (the key low part only with split queries and keys).
+// K / V tensor maps of a call (the key low part only with split queries and keys; the values
+// as fp16 when P is fp16).
 bool make_maps(TileMaps &maps, const AttnArgs &a, bool split, int D)
 {
-    if (!make_map3(&maps.kh, a.k, a.N, a.Hkv, BN, D) || !make_map3(&maps.v, a.v, a.N, a.Hkv, BN, D)) return false;
+    if (kP16 && (a.v16 == nullptr || a.v_absmax == nullptr)) return false;
+    if (!make_map3(&maps.kh, a.k, a.N, a.Hkv, BN, D) ||
+        !make_map3(&maps.v, kP16 ? a.v16 : a.v, a.N, a.Hkv, BN, D, kP16))
+        return false;
     if (split) return make_map3(&maps.kl, a.k_lo, a.N, a.Hkv, BN, D);
     maps.kl = maps.kh;
     return true;

@@ -91,13 +91,15 @@ ris_status cuda_fail(cudaError_t e, const char *what)
 
 // Keep freed pool memory cached in the process (the default pool would hand it back to the
 // driver at every synchronisation, and re-mapping gigabytes costs milliseconds).
+std::mutex g_pool_mu;
+bool g_pool_done[64] = {false};
+
 void prepare_pool_once()
 {
-    static std::mutex mu;
-    static bool done[64] = {false};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return;
-    std::lock_guard<std::mutex> lk(mu);
+    std::lock_guard<std::mutex> lk(g_pool_mu);
+    bool *done = g_pool_done;
     if (done[dev]) return;
     cudaMemPool_t pool;
     if (cudaDeviceGetDefaultMemPool(&pool, dev) == cudaSuccess) {
@@ -107,6 +109,26 @@ void prepare_pool_once()
     done[dev] = true;
 }
 
+// Allocation-failure injection for tests (ris_debug_fail_allocation): the number of
+// stream-ordered allocations still to succeed before one fails, or -1 (off).
+std::atomic<int64_t> g_fail_alloc_after{-1};
+
+// Every stream-ordered allocation of the library goes through here.
+cudaError_t pool_alloc(void **p, size_t bytes, cudaStream_t st)
+{
+    int64_t n = g_fail_alloc_after.load(std::memory_order_relaxed);
+    while (n >= 0) {
+        if (g_fail_alloc_after.compare_exchange_weak(n, n - 1, std::memory_order_relaxed)) {
+            if (n == 0) {  // this is the allocation chosen to fail (once)
+                *p = nullptr;
+                return cudaErrorMemoryAllocation;
+            }
+            break;
+        }
+    }
+    return cudaMallocAsync(p, bytes, st);
+}
+
 // Stream-ordered temporary buffer, released on its stream when it leaves scope.
 struct Scratch {
     void *p = nullptr;
@@ -114,7 +136,7 @@ struct Scratch {
     cudaError_t alloc(size_t bytes, cudaStream_t st)
     {
         s = st;
-        return cudaMallocAsync(&p, bytes < 16 ? 16 : bytes, st);
+        return pool_alloc(&p, bytes < 16 ? 16 : bytes, st);
     }
     ~Scratch()
     {
@@ -151,6 +173,11 @@ std::pair<cudaEvent_t, cudaEvent_t> timer_pair()
     g_timer.used.push_back(e);
     return e;
 }
+
+// Device-side wait limit of the tile kernel in cycles (0: the default, about 2^31) and the
+// test switch that makes its loader issue no copies (ris_debug_tile_stall).
+std::atomic<int64_t> g_wait_limit{0};
+std::atomic<int32_t> g_tile_no_loads{0};
 
 // Kernel design override for benchmarking the designs against each other:
 // RIS_FORCE_DESIGN = gather (register gather), tma (TMA gather), tile (masked dense tiles) or
@@ -480,8 +507,8 @@ ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double d
 
     mk->words_per_mask = row_word_offset(N);
     const int64_t n_rows = n_masks * N;
-    RIS_CUDA(cudaMallocAsync((void **)&mk->bitmap, sizeof(uint32_t) * (size_t)(n_masks * mk->words_per_mask), s));
-    RIS_CUDA(cudaMallocAsync((void **)&mk->row_ptr, sizeof(int64_t) * (size_t)(n_rows + 1), s));
+    RIS_CUDA(pool_alloc((void **)&mk->bitmap, sizeof(uint32_t) * (size_t)(n_masks * mk->words_per_mask), s));
+    RIS_CUDA(pool_alloc((void **)&mk->row_ptr, sizeof(int64_t) * (size_t)(n_rows + 1), s));
     RIS_CUDA(cudaMemsetAsync(mk->row_ptr, 0, sizeof(int64_t), s));
 
     MaskBitsArgs a{};
@@ -520,7 +547,7 @@ ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double d
     RIS_CUDA(cudaMemcpyAsync(&total, mk->row_ptr + n_rows, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
     RIS_CUDA(cudaStreamSynchronize(s));
     mk->n_pairs = total;
-    RIS_CUDA(cudaMallocAsync(&mk->col, (size_t)(total > 0 ? total : 1) * mk->col_bytes, s));
+    RIS_CUDA(pool_alloc(&mk->col, (size_t)(total > 0 ? total : 1) * mk->col_bytes, s));
 
     MaskFillArgs f{};
     f.single_row = -1;
@@ -615,7 +642,7 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     const int design = design_of(m, dtype, head_dim, heads / kv_heads);
     const bool tile = design == 2, suffix = design == 4;
     const bool q_pair = tile || suffix;  // queries as a bf16 hi + lo pair
-    Scratch qt, qtl, kt, ktl, po, pl;
+    Scratch qt, qtl, kt, ktl, po, pl, v16, vmax;
     const void *qu = q, *ku = k, *kl = nullptr, *q_lo = nullptr;
     bool q_split = false;
     if (rope != nullptr && rope->kind != RIS_ROPE_NONE) {
@@ -672,9 +699,20 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.heads_keyed = m->heads_keyed;
     a.n_sets = m->per_seed ? m->n_seeds : 1;
     a.scale_log2 = (float)(1.4426950408889634074 / std::sqrt((double)head_dim));
+    a.wait_limit = g_wait_limit.load(std::memory_order_relaxed);
+    a.debug_no_loads = g_tile_no_loads.load(std::memory_order_relaxed);
     a.row0 = row0;
     a.row1 = row1;
     a.n_tasks = (int64_t)a.n_sets * (row1 - row0) * kv_heads;
+    if (q_pair) {
+        // the tile kernel's value product takes the values as fp16 (scaled into range)
+        const size_t nv = (size_t)N * kv_heads * head_dim;
+        RIS_CUDA(v16.alloc(nv * 2, s));
+        RIS_CUDA(vmax.alloc(sizeof(float), s));
+        RIS_CUDA(launch_values_f16(v, (int64_t)nv, v16.p, (float *)vmax.p, s));
+        a.v16 = v16.p;
+        a.v_absmax = (const float *)vmax.p;
+    }
     if (suffix) {
         RIS_CUDA(po.alloc((size_t)N * heads * head_dim * sizeof(float), s));
         RIS_CUDA(pl.alloc((size_t)N * heads * sizeof(float), s));
@@ -775,6 +813,57 @@ ris_status ris_device_status(void *stream)
     if (word != 0u) return fail(RIS_ERR_DEVICE_TIMEOUT, "a device-side wait gave up (error word 0x%x)", word);
     if (decode_word != 0u)
         return fail(RIS_ERR_INVALID, "a decode step read a position outside [t0, cache_len) from t_dev");
+    return RIS_OK;
+}
+
+ris_status ris_shutdown(void)
+{
+    {
+        std::lock_guard<std::mutex> lk(g_timer.mu);
+        timer_clear_locked();
+        for (auto &e : g_timer.spare) {
+            cudaEventDestroy(e.first);
+            cudaEventDestroy(e.second);
+        }
+        g_timer.spare.clear();
+        g_timer.on = false;
+    }
+    cudaError_t first = cudaSuccess;
+    {
+        std::lock_guard<std::mutex> lk(g_pool_mu);
+        for (int dev = 0; dev < 64; ++dev) {
+            if (!g_pool_done[dev]) continue;
+            cudaMemPool_t pool;
+            cudaError_t e = cudaDeviceGetDefaultMemPool(&pool, dev);
+            if (e == cudaSuccess) {
+                uint64_t thr = 0;  // the CUDA default: cached memory goes back at each synchronisation
+                e = cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &thr);
+                if (e == cudaSuccess) e = cudaMemPoolTrimTo(pool, 0);
+            }
+            if (e != cudaSuccess && first == cudaSuccess) first = e;
+            g_pool_done[dev] = false;
+        }
+    }
+    noalloc_forget_addresses();
+    g_fail_alloc_after.store(-1);
+    g_wait_limit.store(0);
+    g_tile_no_loads.store(0);
+    if (first != cudaSuccess) return cuda_fail(first, "releasing the memory pool cache");
+    return RIS_OK;
+}
+
+ris_status ris_debug_fail_allocation(int64_t n)
+{
+    g_fail_alloc_after.store(n < 0 ? -1 : n);
+    return RIS_OK;
+}
+
+ris_status ris_debug_tile_stall(int32_t no_loads, int64_t wait_limit_cycles)
+{
+    if (no_loads != 0 && no_loads != 1) return fail(RIS_ERR_INVALID, "no_loads must be 0 or 1");
+    if (wait_limit_cycles < 0) return fail(RIS_ERR_INVALID, "wait_limit_cycles must be >= 0");
+    g_wait_limit.store(wait_limit_cycles);
+    g_tile_no_loads.store(no_loads);
     return RIS_OK;
 }
 
@@ -907,7 +996,7 @@ ris_status ris_decode_anchor(int64_t n_prefill, int32_t kv_heads, int32_t mode, 
     an->params = p;
     an->stream = s;
     prepare_pool_once();
-    RIS_CUDA(cudaMallocAsync((void **)&an->off, sizeof(int64_t) * (size_t)(hk + 1), s));
+    RIS_CUDA(pool_alloc((void **)&an->off, sizeof(int64_t) * (size_t)(hk + 1), s));
     // row t0 of the prefill's mask, without its local window (the decode window replaces it);
     // the dense mode keeps every earlier key
     const int64_t words = (t0 >> 5) + 1;
@@ -947,7 +1036,7 @@ ris_status ris_decode_anchor(int64_t n_prefill, int32_t kv_heads, int32_t mode, 
     RIS_CUDA(cudaMemcpyAsync(an->h_off.data(), an->off, sizeof(int64_t) * (size_t)(hk + 1), cudaMemcpyDeviceToHost, s));
     RIS_CUDA(cudaStreamSynchronize(s));
     const int64_t total = an->h_off[hk];
-    RIS_CUDA(cudaMallocAsync((void **)&an->keys, sizeof(int32_t) * (size_t)(total > 0 ? total : 1), s));
+    RIS_CUDA(pool_alloc((void **)&an->keys, sizeof(int32_t) * (size_t)(total > 0 ? total : 1), s));
     MaskFillArgs f{};
     f.single_row = t0;
     f.N = n_prefill;
@@ -1087,7 +1176,7 @@ ris_status ris_decode_step(ris_anchor_t anchor, const void *q, const void *k, co
         if (anchor->scratch) RIS_CUDA(cudaFreeAsync(anchor->scratch, s));
         anchor->scratch = nullptr;
         anchor->scratch_bytes = 0;
-        RIS_CUDA(cudaMallocAsync(&anchor->scratch, need, s));
+        RIS_CUDA(pool_alloc(&anchor->scratch, need, s));
         anchor->scratch_bytes = need;
         anchor->stream = s;
     }

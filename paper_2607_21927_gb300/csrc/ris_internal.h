@@ -100,6 +100,11 @@ struct AttnArgs {
     int32_t window;
     float scale_log2;      // log2(e) / sqrt(D)
     int64_t n_tasks;       // n_sets * (row1 - row0) * Hkv
+    const void *v16;       // tile kernel: the values as fp16, scaled by 2^-E (launch_values_f16)
+    const float *v_absmax; // tile kernel: max |v| over the values (device), from which E follows
+    int64_t wait_limit;    // tile kernel: cycles a device-side wait may take (0: about 2^31)
+    int32_t debug_no_loads;  // tile kernel, tests only: the loader issues no copies, so the
+                             // first wait on them gives up (ris_debug_tile_stall)
 };
 
 // Arguments of the Hybrid Anchor decode kernels (one generated token at position t). The
@@ -141,6 +146,9 @@ struct DecodeArgs {
     float *lse;                // [Hq] or null
 };
 
+// Forget the allocation-free entry point's cached scratch addresses (ris_shutdown).
+void noalloc_forget_addresses();
+
 // Library-wide kernel launch counter (ris_launch_count).
 void note_launch(int n = 1);
 
@@ -161,6 +169,11 @@ unsigned int read_decode_error();
 
 // dtype_in / dtype_out are ris_dtype values.
 cudaError_t launch_rope(const RopeArgs &a, int dtype_in, int dtype_out, cudaStream_t s);
+
+// bf16 values v[n] (n a multiple of 8, 16-byte aligned) -> *vmax = max |v| (vmax zeroed by
+// this call) and v16[i] = fp16(v[i] / 2^E), E = v_scale_exp(max |v|): the fp16 operand of the
+// tile kernel's value product, exact for every bf16 value in fp16's normal range.
+cudaError_t launch_values_f16(const void *v, int64_t n, void *v16, float *vmax, cudaStream_t s);
 
 // q_split: q is fp32 and is split into bf16 hi + lo on the tensor-core path; a.k_lo set:
 // the keys arrive as a bf16 hi + lo pair.

@@ -7,9 +7,11 @@
 // CUDA math library in fp32 and the rotation runs in fp32. The work is HBM-bound: one read
 // and one write of the tensor.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include <cstdint>
 
+#include "attn_common.cuh"
 #include "ris_internal.h"
 
 namespace ris {
@@ -63,7 +65,57 @@ __global__ void k_rope(const RopeArgs a)
     }
 }
 
+// max |v| over 8 bf16 values per thread and step (grid-stride), one atomic per warp; |v| >= 0,
+// so the order of the float bit patterns is the order of the values
+__global__ void k_absmax_bf16(const uint4 *v, int64_t n8, unsigned int *vmax)
+{
+    float m = 0.f;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n8; t += (int64_t)gridDim.x * blockDim.x) {
+        const uint4 x = v[t];
+        const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            m = fmaxf(m, fabsf(__uint_as_float(w[k] << 16)));
+            m = fmaxf(m, fabsf(__uint_as_float(w[k] & 0xFFFF0000u)));
+        }
+    }
+    m = warp_max(m);
+    if ((threadIdx.x & 31) == 0) atomicMax(vmax, __float_as_uint(m));
+}
+
+__global__ void k_values_f16(const uint4 *v, int64_t n8, const float *vmax, uint4 *v16)
+{
+    const float scale = __uint_as_float((uint32_t)(127 - v_scale_exp(*vmax)) << 23);  // 2^-E
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n8; t += (int64_t)gridDim.x * blockDim.x) {
+        const uint4 x = v[t];
+        const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const __half2 h = __floats2half2_rn(__uint_as_float(w[k] << 16) * scale,
+                                                __uint_as_float(w[k] & 0xFFFF0000u) * scale);
+            o[k] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        v16[t] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_values_f16(const void *v, int64_t n, void *v16, float *vmax, cudaStream_t s)
+{
+    if ((n & 7) != 0) return cudaErrorInvalidValue;
+    const int64_t n8 = n / 8;
+    cudaError_t e = cudaMemsetAsync(vmax, 0, sizeof(float), s);
+    if (e != cudaSuccess) return e;
+    const int threads = 256;
+    const int64_t need = (n8 + threads - 1) / threads;
+    const unsigned grid = (unsigned)(need < 152 * 8 ? (need > 0 ? need : 1) : 152 * 8);
+    k_absmax_bf16<<<grid, threads, 0, s>>>(reinterpret_cast<const uint4 *>(v), n8, reinterpret_cast<unsigned int *>(vmax));
+    k_values_f16<<<grid, threads, 0, s>>>(reinterpret_cast<const uint4 *>(v), n8, vmax, reinterpret_cast<uint4 *>(v16));
+    note_launch(2);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_rope(const RopeArgs &a, int dtype_in, int dtype_out, cudaStream_t s)
 {

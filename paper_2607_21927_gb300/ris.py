@@ -95,6 +95,10 @@ _SIGS = {
     "ris_attention_masked_noalloc": [ctypes.c_void_p] * 5 + [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                      ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p,
                                      ctypes.c_void_p],
+    "ris_noalloc_scratch_info": [ctypes.c_void_p, ctypes.c_void_p],
+    "ris_shutdown": [],
+    "ris_debug_fail_allocation": [ctypes.c_int64],
+    "ris_debug_tile_stall": [ctypes.c_int32, ctypes.c_int64],
     "ris_kernel_timer_enable": [ctypes.c_int32],
     "ris_device_status": [ctypes.c_void_p],
     "ris_attention_design": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32],
@@ -415,7 +419,7 @@ def ris_attention_masked(mask: Mask, q, k, v, rope: Optional[RopeCfg] = None,
 def ris_attention_masked_noalloc(mask: Mask, q, k, v, out: torch.Tensor, rope: Optional[RopeCfg] = None,
                                  lse: Optional[torch.Tensor] = None, stream=None):
     """Allocation-free layer call: the caller passes every output buffer; the library's
-    scratch is a fixed 64 MiB device array (see include/ris.h)."""
+    scratch is a fixed 64 MiB device array, and every mask runs on the gather design."""
     N, Hq, Hkv, D = _shapes(q, k, v)
     d = mask.info()
     if d.N != N:
@@ -425,6 +429,28 @@ def ris_attention_masked_noalloc(mask: Mask, q, k, v, out: torch.Tensor, rope: O
         mask.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(out), Hq, Hkv, D, _dtype(q), _dtype(out), _ref(rope),
         _ptr(lse), _stream(stream)))
     return out
+
+
+def ris_noalloc_scratch_info():
+    """(device address, bytes) of the allocation-free entry point's scratch array."""
+    addr, n = ctypes.c_void_p(), ctypes.c_int64()
+    _check("ris_noalloc_scratch_info", lib().ris_noalloc_scratch_info(ctypes.byref(addr), ctypes.byref(n)))
+    return int(addr.value or 0), int(n.value)
+
+
+def ris_shutdown() -> None:
+    """Release the library's cached per-device state (timer events, pool caches)."""
+    _check("ris_shutdown", lib().ris_shutdown())
+
+
+def ris_debug_fail_allocation(n: int) -> None:
+    """Tests: the n-th stream-ordered allocation from now on fails (n < 0 disarms)."""
+    _check("ris_debug_fail_allocation", lib().ris_debug_fail_allocation(int(n)))
+
+
+def ris_debug_tile_stall(no_loads: bool, wait_limit_cycles: int = 0) -> None:
+    """Tests: the tile kernel's loader issues no copies and its waits give up after the limit."""
+    _check("ris_debug_tile_stall", lib().ris_debug_tile_stall(int(bool(no_loads)), int(wait_limit_cycles)))
 
 
 # ----------------------------------------------------------------------------- Hybrid Anchor decode

@@ -473,3 +473,29 @@ def test_head_dim_64_on_tiles(N, mode, d, S, W, Hq, Hkv, design):
     ref, ref_lse = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e4, 256, W=W)
     check_bf16_path(to_np(out), ref)
     np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
+
+
+@pytest.mark.parametrize("N,mode,d,S,layer", [
+    (32768, 0, 0.01, 70, 0), (65536, 0, 0.01, 10, 7), (65536, 1, 0.01, 10, 7), (65536, 0, 0.01, 70, 27),
+    (65536, 1, 0.01, 70, 27)],
+    ids=["c4a_32k_1pct_x70", "c5_64k_stochastic_x10", "c5_64k_structural_x10", "c5_64k_stochastic_x70",
+         "c5_64k_structural_x70"])
+def test_benchmarked_layers_bf16_output(N, mode, d, S, layer):
+    """The layers the benchmark times, in its own configuration: a mask built once and
+    ris_attention_masked with bf16 outputs (the bench's output dtype), YaRN with native window
+    32768, inputs of the layer's seed; about 1024 sampled rows (all heads) against the oracle.
+    Covers the 65,536-token 70-seed run in both modes (Results, "Ensemble Coverage Analysis")."""
+    (q, k, v), (qn, kn, vn) = make_inputs(N, QWEN["Hq"], QWEN["Hkv"], QWEN["D"], seed=layer, outliers=True)
+    seeds = list(range(S))
+    m = ris.ris_mask_generate(N, QWEN["Hkv"], mode, d, seeds)
+    design = ris.ris_attention_design(m, torch.bfloat16, QWEN["D"])
+    out = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e6, 32768))
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    m.free()
+    assert out.dtype == torch.bfloat16
+    rows = sample_rows(N, 1024, seed=N + S + mode)
+    assert rows.shape[0] >= 1000
+    ref, _ = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e6, 32768, rows=rows)
+    err, rel = check_bf16_path(to_np(out[rows]), ref, out_bf16=True)
+    print(f"design {design}: max-abs {err:.2e}, rel-L2 {rel:.2e}")
