@@ -6,33 +6,44 @@
 // percent, and the dense mode) a dense 128 x 128 score tile with the mask applied as -inf
 // beats gathering rows pair by pair. One CTA owns one (128-query tile, query head, set):
 //
-//   warp 8 (TMA)   streams 128-key tiles of K~ hi + K~ lo (64 KB) and of V (32 KB) in
-//                  128-byte swizzled boxes into two two-stage shared-memory rings: a key stage
-//                  is refilled as soon as its score products are done, a value stage once its
-//                  value product is, so the next keys load while P and the value product of
-//                  the current tile are still pending;
+//   warp 8 (TMA)   streams 128-key tiles of K~ hi + K~ lo (64 KB) and of the values (fp16,
+//                  32 KB) in 128-byte swizzled boxes into two two-stage shared-memory rings:
+//                  a key stage is refilled as soon as its score products are done, a value
+//                  stage once its value product is, so the next keys load while P and the
+//                  value product of the current tile are still pending;
 //   warp 9 (MMA)   one elected lane issues tcgen05.mma: S = Q_hi K_hi^T + Q_lo K_hi^T +
 //                  Q_hi K_lo^T (A = the query tile, kept in TMEM) into a double-buffered TMEM
-//                  score tile, and O += P_hi V + P_lo V (A = P, written into TMEM over the
-//                  consumed scores) into the TMEM output tile, committing each step to an
-//                  mbarrier; TMEM holds S/P twice (2 x 128 columns), O (128) and Q hi / lo
-//                  (2 x 64), all 512 columns;
+//                  score tile, and O += P V (A = P as fp16, written into TMEM over the consumed
+//                  scores) into the TMEM output tile, committing each step to an mbarrier;
+//                  TMEM holds S/P twice (2 x 128 columns), O (128) and Q hi / lo (2 x 64), all
+//                  512 columns;
 //   warps 0-7      two threads per query row (score and output columns 0-63 / 64-127): write
 //                  the row's query half into TMEM, then per tile tcgen05.ld the scores, apply
 //                  the bitmap (or the causal cut), exchange the partial row max with the
 //                  partner thread, fp32 online softmax with lazy rescaling of O in TMEM (only
-//                  when the row max grows by more than 2^8), write P hi / lo into TMEM, and at
-//                  the end normalise O and store the row.
+//                  when the row max grows by more than 2^8), write P into TMEM, and at the end
+//                  normalise O (and undo the values' power-of-two scale) and store the row.
 //
-// Precision: the five products keep about 16 significant bits of every operand. Single
-// fp16 keys move outputs by up to 0.1 on inputs with outlier channels, and P rounded to fp16
-// (one value product instead of two: 13% faster) by up to 1.1e-2 at 2k tokens, above the
-// 1e-2 bar, so neither is taken.
+// Precision. With activation outlier channels the scores reach tens of units while the
+// output moves by p (v_j - o) per unit of score error, so the scores need about 17
+// significant bits: the three products keep q and k to about 16 bits each (bf16 hi + lo).
+// One product of fp16 keys moves outputs by up to 0.1; fp16 main products with fp8 (e4m3 /
+// e5m2) correction products by up to 4e-3 to 7e-3 (CPU emulation on inputs with outlier
+// channels), so neither is taken. P enters the value product as one fp16 (11 significant
+// bits; max-abs 6.5e-3 in the same emulation against 1.7e-3 for a bf16 hi + lo pair), and the
+// row sum adds P as rounded, so that each weight's rounding moves the output by at most 2^-11
+// of that weight times |v_j - o|. The values are exact in fp16 after a power-of-two scale
+// (none unless some |v| reaches 2^14), undone in the epilogue.
 //
-// Measured on a 32k-token layer: 5.7 ms. With one ring of combined K/V stages, released only
-// after the value product, the next tile's keys started loading only then and the tensor
-// pipe waited for them: 7.2 ms (the products alone 6.0 ms). 128-key tiles with the query in
-// TMEM beat 64-key tiles with the query in shared memory and three stages (7.8 ms).
+// Measured: the kernel issues its products at the measured sustained bf16 rate (about 95
+// cycles per 128 x 128 x 16 product at the power-capped clock): 32 products per tile pair
+// take ~3,090 cycles (C5's Stochastic layer at 64k: 16.4 ms per launch; with a bf16 P pair
+// and 40 products, 19.6 ms). Dropping score products (timing experiments, wrong results)
+// runs into the softmax's own per-tile latency (~3,000 cycles), so fewer products would need
+// a shorter softmax chain as well. Four threads per row (16 softmax warps) measured the same
+// as two. With one ring of combined K/V stages, released only after the value product, the
+// next tile's keys started loading only then and the tensor pipe waited for them; 128-key
+// tiles with the query in TMEM beat 64-key tiles with the query in shared memory.
 //
 // The suffix pass of the dense-suffix split (SUFFIX) runs the same pipeline over the key
 // tiles of each row's dense suffix only (its Structural block and / or local window: every key
@@ -241,36 +252,6 @@ __device__ __forceinline__ void tmem_ld64(uint32_t taddr, float *v)
     for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Two 32-column stores (32 lanes each) and one wait for both.
-__device__ __forceinline__ void tmem_st32x2(uint32_t ta, const uint32_t *a, uint32_t tb, const uint32_t *b)
-{
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33};\n\t"
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%1], {%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63,%64,%65};\n\t"
-        "tcgen05.wait::st.sync.aligned;" ::"r"(ta), "r"(tb),
-        "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(a[4]), "r"(a[5]), "r"(a[6]), "r"(a[7]), "r"(a[8]), "r"(a[9]), "r"(a[10]), "r"(a[11]), "r"(a[12]), "r"(a[13]), "r"(a[14]), "r"(a[15]), "r"(a[16]), "r"(a[17]), "r"(a[18]), "r"(a[19]), "r"(a[20]), "r"(a[21]), "r"(a[22]), "r"(a[23]), "r"(a[24]), "r"(a[25]), "r"(a[26]), "r"(a[27]), "r"(a[28]), "r"(a[29]), "r"(a[30]), "r"(a[31]),
-        "r"(b[0]), "r"(b[1]), "r"(b[2]), "r"(b[3]), "r"(b[4]), "r"(b[5]), "r"(b[6]), "r"(b[7]), "r"(b[8]), "r"(b[9]), "r"(b[10]), "r"(b[11]), "r"(b[12]), "r"(b[13]), "r"(b[14]), "r"(b[15]), "r"(b[16]), "r"(b[17]), "r"(b[18]), "r"(b[19]), "r"(b[20]), "r"(b[21]), "r"(b[22]), "r"(b[23]), "r"(b[24]), "r"(b[25]), "r"(b[26]), "r"(b[27]), "r"(b[28]), "r"(b[29]), "r"(b[30]), "r"(b[31])
-        : "memory");
-}
-
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float *v)
-{
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
-        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
-        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
-        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
-        "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
-        "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
-        "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15])),
-        "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])), "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])),
-        "r"(__float_as_uint(v[20])), "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
-        "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])), "r"(__float_as_uint(v[27])),
-        "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])), "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
-        : "memory");
-    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-
 // 32 lanes x 16 consecutive 32-bit columns, loaded and waited for in one statement.
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float *v)
 {
@@ -361,6 +342,14 @@ __device__ __forceinline__ void tmem_st_words(uint32_t taddr, const uint32_t *w)
         static_assert(NC == 8, "32, 16 or 8 columns");
         tmem_st8(taddr, w);
     }
+}
+
+// max of three floats in one instruction
+__device__ __forceinline__ float fmax3(float x, float y, float z)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(x), "f"(y), "f"(z));
+    return d;
 }
 
 // 2^x by the SFU (ex2.approx, relative error about 2^-22, subnormal results flushed to 0);
@@ -671,15 +660,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int c = 0; c < 32; ++c) sv[32 * e + c] = ((cw[e] >> c) & 1u) ? sv[32 * e + c] : -INFINITY;
                 cw[e] = nw[e];
             }
-            float mx8[8];
+            float mx9[9];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                mx8[e] = sv[e];
+            for (int e = 0; e < 9; ++e) {
+                mx9[e] = sv[e];
 #pragma unroll
-                for (int c = e + 8; c < SC; c += 8) mx8[e] = fmaxf(mx8[e], sv[c]);
+                for (int c = e + 9; c < SC; c += 18)
+                    mx9[e] = c + 9 < SC ? fmax3(mx9[e], sv[c], sv[c + 9]) : fmaxf(mx9[e], sv[c]);
             }
-            const float pm = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * sc;
+            const float pm = fmax3(fmax3(mx9[0], mx9[1], mx9[2]), fmax3(mx9[3], mx9[4], mx9[5]),
+                                   fmax3(mx9[6], mx9[7], mx9[8])) * sc;
             float pms[kRowThreads];
             ok = exchange(j, pm, pms);
             if (!ok) break;
