@@ -768,7 +768,7 @@ def main():
     hbm, tc = ceil["hbm_gbs"], ceil["tc_tflops"]
     kv_row_bytes = Hkv * 2 * D * e  # K and V rows of one key, all KV heads
     kv_set = N * Hkv * D * e * (3 if e == 2 else 2)  # rotated K (hi + lo for bf16) and V of a layer
-    gather_names = {0: "k_attn_bf16 (register gather)", 1: "k_attn_tma (TMA gather4)", 2: "k_attn_tile (tcgen05 masked tiles)",
+    gather_names = {0: "k_attn_bf16 (register gather)", 2: "k_attn_tile (tcgen05 masked tiles)",
                     3: "k_attn_f32 (fp32 gather)",
                     4: "k_attn_tile suffix pass + k_attn_bf16 (dense-suffix split: Structural blocks / local window "
                        "on the tiles, the rest gathered)"}

@@ -280,7 +280,7 @@ ris_status ris_kernel_timer_read(double *total_ms, int64_t *launches);
 ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double *ms_each, int64_t capacity);
 
 /* Attention kernel design a layer call on `mask` uses for this input dtype and head_dim
- * (host-only, no device work): 0 register gather, 1 TMA gather, 2 tcgen05 masked dense tiles,
+ * (host-only, no device work): 0 register gather, 2 tcgen05 masked dense tiles,
  * 3 fp32 gather, 4 dense-suffix split; -1 for invalid arguments. bf16 calls use tiles when
  * the mask is dense or keeps at least 6.9% (head_dim 128) or 13.6% (head_dim 64) of the
  * causal pairs in what a gather would fetch (and always when heads/kv_heads > 8, which this
@@ -290,7 +290,7 @@ ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double 
  * "Sampling Modes": in-block pairs are cliques; the window is forced), so a first launch
  * attends every row to that suffix on the tiles and the register gather continues that
  * softmax over the row's other keys; the result is the same single softmax over the row's
- * whole key set. RIS_FORCE_DESIGN = gather | tma | tile | suffix in the environment
+ * whole key set. RIS_FORCE_DESIGN = gather | tile | suffix in the environment
  * overrides (benchmarking). */
 int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim);
 

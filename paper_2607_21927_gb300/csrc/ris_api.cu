@@ -180,7 +180,7 @@ std::atomic<int64_t> g_wait_limit{0};
 std::atomic<int32_t> g_tile_no_loads{0};
 
 // Kernel design override for benchmarking the designs against each other:
-// RIS_FORCE_DESIGN = gather (register gather), tma (TMA gather), tile (masked dense tiles) or
+// RIS_FORCE_DESIGN = gather (register gather), tile (masked dense tiles) or
 // suffix (the dense-suffix split, where the mask allows it).
 const char *forced_design()
 {
@@ -240,7 +240,7 @@ int64_t suffix_pairs_of(int64_t N, int64_t block, int64_t W)
     return total;
 }
 
-// Design of a layer call: 0 register gather, 1 TMA gather, 2 masked dense tiles, 3 fp32
+// Design of a layer call: 0 register gather, 2 masked dense tiles, 3 fp32
 // gather, 4 dense-suffix split (each row's dense suffix on the tile kernel, its other keys on
 // the register gather, one softmax). The gather's cost grows with the pairs it gathers (with
 // the split: all but the suffixes), a tile's does not, hence the density threshold.
@@ -249,7 +249,6 @@ int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim, int32_t grou
     if (dtype == RIS_F32) return 3;
     if (group > 8) return 2;  // only the tiles take more than 8 query heads per KV head
     const std::string f = forced_design();
-    if (f == "tma" && tma_gather_available()) return 1;
     if (f == "gather") return 0;
     const bool tiles = (head_dim == 128 || head_dim == 64) && tile_design_available();
     if (tiles && (f == "tile" || m->dense)) return 2;
@@ -729,9 +728,7 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     } else if (suffix) {  // the dense suffixes on the tiles, then the gather continues their softmax
         RIS_CUDA(launch_attention_tile_suffix(a, head_dim, qu, a.q_lo, s));
         RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, false, s));
-    } else if (design == 1)
-        RIS_CUDA(launch_attention_tma(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
-    else if (dtype == RIS_BF16)
+    } else if (dtype == RIS_BF16)
         RIS_CUDA(launch_attention_bf16(a, head_dim, out_dtype, q_split, m->col_bytes, m->dense != 0, s));
     else
         RIS_CUDA(launch_attention_f32(a, head_dim, out_dtype, m->col_bytes, m->dense != 0, s));
@@ -807,7 +804,7 @@ int32_t ris_attention_design(ris_mask_t mask, int32_t dtype, int32_t head_dim)
 ris_status ris_device_status(void *stream)
 {
     unsigned int word = 0, tile_word = 0;
-    RIS_CUDA(read_device_error(&word, reinterpret_cast<cudaStream_t>(stream)));
+    RIS_CUDA(cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)));
     RIS_CUDA(read_tile_error(&tile_word));
     const unsigned int decode_word = read_decode_error();
     word |= tile_word;

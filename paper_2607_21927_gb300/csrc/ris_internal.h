@@ -182,11 +182,6 @@ cudaError_t launch_attention_bf16(const AttnArgs &a, int D, int out_dtype, bool 
 cudaError_t launch_attention_f32(const AttnArgs &a, int D, int out_dtype, int col_bytes, bool dense,
                                  cudaStream_t s);
 
-// TMA-gather design of the bf16 kernel; split: fp32 queries and hi + lo keys.
-bool tma_gather_available();
-cudaError_t launch_attention_tma(const AttnArgs &a, int D, int out_dtype, bool split, int col_bytes, bool dense,
-                                 cudaStream_t s);
-cudaError_t read_device_error(unsigned int *out, cudaStream_t s);
 
 // Masked dense-tile design (tcgen05, head dim 128 or 64): q_hi / q_lo bf16 query pair (q_lo
 // null for exact bf16 inputs).

@@ -158,7 +158,7 @@ def ris_version() -> str:
     return lib().ris_version().decode()
 
 
-DESIGNS = {0: "register gather", 1: "TMA gather", 2: "tcgen05 masked tiles", 3: "fp32 gather",
+DESIGNS = {0: "register gather", 2: "tcgen05 masked tiles", 3: "fp32 gather",
            4: "dense suffix on tiles + register gather"}
 
 
