@@ -115,9 +115,11 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle CPU baseline")
     ap.add_argument("--no-probes", action="store_true", help="skip the L2 / FFMA ceiling probes")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle seconds per step")
-    ap.add_argument("--shard", choices=("replicas", "rows"), default="replicas",
+    ap.add_argument("--shard", choices=("replicas", "rows", "rows-kv"), default="replicas",
                     help="with several ranks: every rank runs the whole workload (weak scaling), or each "
-                         "rank takes a balanced range of query rows of the same workload (strong scaling)")
+                         "rank takes a balanced range of query rows of the same workload (strong scaling) "
+                         "with all of K and V (rows), or holding only its own rows of q, k and v and "
+                         "all-gathering each layer's K and V (rows-kv)")
     a = ap.parse_args()
     w = dict(WORKLOADS[a.workload])
     w["name"] = a.workload
@@ -157,8 +159,10 @@ def workload_config(a):
         "geometry": ("local window 1024 + 4 anchors" if w.get("geometry") == "paper" else "diagonal only"),
         "sampler": "index draws (K = round(dN) per row and seed)" if w.get("sampler") else "Bernoulli per pair",
         "seed_outputs": "one per seed (per-seed masks)" if w.get("per_seed") else "one (union of the seeds)",
-        "multi_gpu": ("balanced query-row ranges of one workload per rank" if a.shard == "rows"
-                      else "one whole workload per rank"),
+        "multi_gpu": {"rows": "balanced query-row ranges of one workload per rank",
+                      "rows-kv": "balanced query-row ranges of one workload per rank, each rank holding only "
+                                 "its rows of q, k and v and all-gathering each layer's K and V"}.get(
+                          a.shard, "one whole workload per rank"),
         "l2": (f"inputs larger than L2: each layer has its own q/k/v ({per_layer / 2**20:.0f} MiB), "
                f"{w['layers']} layers = {w['layers'] * per_layer / 2**20:.0f} MiB per run"),
     } | ({"decode": {"generated_tokens": w["gen"], "window": w["window"],
@@ -680,6 +684,21 @@ def main():
     oshape = lambda ns: (ns, N, Hq, D) if per_seed else (N, Hq, D)  # noqa: E731
     outs = [[torch.empty(oshape(ns), dtype=tdt, device=dev) for _ in range(L)] for (_, _, _, ns) in runs]
     stream = torch.cuda.current_stream()
+    # rows-kv: each rank keeps only its own rows of every layer's q, k and v (for each run's
+    # balanced partition, a pure function of the mask that every rank derives alike) and
+    # all-gathers K and V per layer inside the step
+    local = {}
+    if a.shard == "rows-kv":
+        from paper_2607_21927_gb300 import shard
+
+        for ri, (name, mode, dens, ns) in enumerate(runs):
+            m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom, per_seed=per_seed)
+            b = ris.ris_mask_row_split(m, world)
+            m.free()
+            r0, r1 = b[rank], b[rank + 1]
+            local[ri] = (b, [qs[l][r0:r1].clone() for l in range(L)], [ks[l][r0:r1].clone() for l in range(L)],
+                         [vs[l][r0:r1].clone() for l in range(L)],
+                         [torch.empty((r1 - r0, Hq, D), dtype=tdt, device=dev) for _ in range(L)])
     pairs, design, suffix = {}, {}, {}
     mask_events = []  # (run, start, mask built, layers done) events of each run while `timing` is set
     timing = [False]
@@ -698,7 +717,16 @@ def main():
             # the dense-suffix split attends the rows' dense suffixes (Structural blocks, local
             # window) on the tiles, not by gathering
             suffix[name] = mi.suffix_pairs * mi.n_masks if design[name] == 4 else 0
-            if a.shard == "rows" and world > 1:
+            if a.shard == "rows-kv":
+                b, ql, kl, vl, ol = local[ri]
+                for layer in range(L):
+                    if world > 1:
+                        kf, vf = shard.kv_allgather(kl[layer], vl[layer], b)
+                    else:
+                        kf, vf = kl[layer], vl[layer]
+                    ris.ris_attention_masked_local(m, b[rank], b[rank + 1], ql[layer], kf, vf, out_rows=ol[layer],
+                                                   rope=rope)
+            elif a.shard == "rows" and world > 1:
                 # every rank builds the same mask and attends its own balanced range of rows
                 b = ris.ris_mask_row_split(m, world)
                 for layer in range(L):
@@ -750,7 +778,7 @@ def main():
         layers_ms[name] = layers_ms.get(name, 0.0) + e1.elapsed_time(e2) / a.steps
     total_pairs = sum(pairs.values())
     pair_heads_step = total_pairs * L * Hq
-    strong = a.shard == "rows" and world > 1  # the ranks share one workload
+    strong = a.shard in ("rows", "rows-kv") and world > 1  # the ranks share one workload
     value = (1 if strong else world) * pair_heads_step * a.steps / (elapsed_ms / 1e3)
     ms_step = elapsed_ms / a.steps
 

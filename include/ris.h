@@ -225,6 +225,20 @@ ris_status ris_attention_masked_rows(ris_mask_t mask, int64_t row_begin, int64_t
                                      int32_t head_dim, int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
                                      float *lse, void *stream);
 
+/* Query rows row_begin .. row_end-1 of ris_attention_masked with only those rows in memory:
+ * q_rows [row_end - row_begin][heads][head_dim] holds query rows row_begin .., out_rows gets
+ * the same rows of the output, and lse_rows (optional) is [heads][row_end - row_begin]. K and V
+ * must hold every position 0 .. N-1: this is the per-device step of a prefill split by query
+ * rows in which each device holds only its own rows of q, k and v and all-gathers the layer's
+ * K and V first (the paper's row independence, Methods, "Memory-Bounded Geometry Generation":
+ * every device builds the same counter-based mask). Each row equals the same row of the
+ * whole-layer call bit for bit. Masks built per seed are refused (RIS_ERR_UNSUPPORTED).
+ * Errors: as ris_attention_masked_rows. */
+ris_status ris_attention_masked_local(ris_mask_t mask, int64_t row_begin, int64_t row_end, const void *q_rows,
+                                      const void *k, const void *v, void *out_rows, int32_t heads, int32_t kv_heads,
+                                      int32_t head_dim, int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
+                                      float *lse_rows, void *stream);
+
 /* Balanced contiguous row ranges for `parts` workers: bounds[0] = 0 < bounds[1] < ... <
  * bounds[parts] = N, cut where the running sampled-pair count reaches k/parts of the total
  * (every part gets at least one row). ris_row_split takes a HOST row_ptr of N + 1 offsets

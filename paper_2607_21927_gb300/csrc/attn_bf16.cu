@@ -451,9 +451,9 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         }
     }
     if (a.lse != nullptr && p == 0) {
-        float *lse = a.lse + ((int64_t)t.s * a.Hq + (int64_t)t.g * a.G) * a.N + t.i;
-        if (h0 < a.G) lse[(int64_t)h0 * a.N] = (m0 + __log2f(l0)) * kLn2;
-        if (h1 < a.G) lse[(int64_t)h1 * a.N] = (m1 + __log2f(l1)) * kLn2;
+        float *lse = a.lse + ((int64_t)t.s * a.Hq + (int64_t)t.g * a.G) * a.lse_ld + t.i;
+        if (h0 < a.G) lse[(int64_t)h0 * a.lse_ld] = (m0 + __log2f(l0)) * kLn2;
+        if (h1 < a.G) lse[(int64_t)h1 * a.lse_ld] = (m1 + __log2f(l1)) * kLn2;
     }
     if (SEEDS && set + 1 < n_sets) {
         // on to the next set: its first group's rows are in flight

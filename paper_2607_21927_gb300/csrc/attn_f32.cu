@@ -123,7 +123,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32) k_attn_f32(const AttnArgs a)
 #pragma unroll
         for (int e = 0; e < DL; ++e) st_out<TOut>(out + (int64_t)h * D + e, o[h][e] * inv);
         if (a.lse != nullptr && lane == 0)
-            a.lse[((int64_t)t.s * a.Hq + (int64_t)t.g * a.G + h) * a.N + t.i] = (m[h] + log2f(lt)) * kLn2;
+            a.lse[((int64_t)t.s * a.Hq + (int64_t)t.g * a.G + h) * a.lse_ld + t.i] = (m[h] + log2f(lt)) * kLn2;
     }
 }
 

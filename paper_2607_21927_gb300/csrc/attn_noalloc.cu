@@ -220,6 +220,7 @@ extern "C" ris_status ris_attention_masked_noalloc(ris_mask_t mask, const void *
     a.v = v;
     a.out = out;
     a.lse = lse;
+    a.lse_ld = N;
     a.row_ptr = md.row_ptr;
     a.col = md.col;
     a.N = N;

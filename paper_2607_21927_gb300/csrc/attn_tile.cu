@@ -775,7 +775,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (SUFFIX) {
                 if (row_ok && cq == 0) a.part_lse[i * a.Hq + h] = m_used + __log2f(lt);
             } else if (row_ok && cq == 0 && a.lse != nullptr) {
-                a.lse[((int64_t)s * a.Hq + h) * a.N + i] = (m_used + __log2f(lt)) * kLn2;
+                a.lse[((int64_t)s * a.Hq + h) * a.lse_ld + i] = (m_used + __log2f(lt)) * kLn2;
             }
         }
     }

@@ -632,12 +632,21 @@ ris_status ris_rope_apply(void *x, int32_t dtype, int64_t N, int32_t heads, int3
 namespace {
 
 // Attention of query rows row0 .. row1-1 over an existing mask; arguments already validated.
+// local: q, out and lse hold only those rows (q [rows][heads][D], out likewise, lse
+// [heads][rows]); otherwise they hold all N rows. K and V always hold all N positions.
 ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, const void *v, void *out,
                          int32_t heads, int32_t kv_heads, int32_t head_dim, int32_t dtype, int32_t out_dtype,
-                         const ris_rope_cfg *rope, float *lse, cudaStream_t s, int64_t row0 = 0, int64_t row1 = -1)
+                         const ris_rope_cfg *rope, float *lse, cudaStream_t s, int64_t row0 = 0, int64_t row1 = -1,
+                         bool local = false)
 {
     const int64_t N = m->N;
     if (row1 < 0) row1 = N;
+    // Local rows: the kernels index q, out and lse by absolute row, so they are handed base
+    // pointers moved back by row0 rows; only rows row0 .. row1-1 are ever addressed.
+    const int64_t q_rows = local ? row1 - row0 : N, q_first = local ? row0 : 0;
+    auto back = [&](const void *p, size_t row_bytes) -> const void * {
+        return p == nullptr ? nullptr : static_cast<const char *>(p) - (size_t)q_first * row_bytes;
+    };
     prepare_pool_once();
     const int design = design_of(m, dtype, head_dim, heads / kv_heads);
     const bool tile = design == 2, suffix = design == 4;
@@ -652,7 +661,7 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         ra.N = N;
         ra.D = head_dim;
         ra.mscale = (float)ms;
-        const size_t nq = (size_t)N * heads * head_dim, nk = (size_t)N * kv_heads * head_dim;
+        const size_t nq = (size_t)q_rows * heads * head_dim, nk = (size_t)N * kv_heads * head_dim;
         // rotated queries: fp32 (split into bf16 hi + lo by the gather kernels) or, when the
         // tile kernel runs, a bf16 hi + lo pair; rotated keys in fp32, or for bf16 inputs a
         // bf16 hi + lo pair
@@ -668,26 +677,32 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         ra.x_out = qt.p;
         ra.x_out_lo = q_pair ? qtl.p : nullptr;
         ra.H = heads;
+        ra.N = q_rows;
+        ra.pos0 = q_first;
         RIS_CUDA(launch_rope(ra, dtype, q_pair ? RIS_BF16 : RIS_F32, s));
+        ra.N = N;
+        ra.pos0 = 0;
         ra.x_in = k;
         ra.x_out = kt.p;
         ra.x_out_lo = ktl.p;
         ra.H = kv_heads;
         RIS_CUDA(launch_rope(ra, dtype, dtype, s));
-        qu = qt.p;
-        q_lo = qtl.p;
+        qu = back(qt.p, (size_t)heads * head_dim * (q_pair ? 2 : 4));
+        q_lo = back(qtl.p, (size_t)heads * head_dim * 2);
         ku = kt.p;
         kl = ktl.p;
         q_split = (dtype == RIS_BF16);
     }
+    if (qu == q) qu = back(q, (size_t)heads * head_dim * (dtype == RIS_BF16 ? 2 : 4));
     AttnArgs a{};
     a.q = qu;
     a.q_lo = q_pair ? q_lo : nullptr;
     a.k = ku;
     a.k_lo = kl;
     a.v = v;
-    a.out = out;
-    a.lse = lse;
+    a.out = const_cast<void *>(back(out, (size_t)heads * head_dim * (out_dtype == RIS_BF16 ? 2 : 4)));
+    a.lse = lse == nullptr ? nullptr : lse - q_first;
+    a.lse_ld = q_rows;
     a.row_ptr = m->row_ptr;
     a.col = m->col;
     a.bitmap = m->bitmap;
@@ -891,6 +906,23 @@ ris_status ris_attention_masked_rows(ris_mask_t mask, int64_t row_begin, int64_t
                     (long long)row_end, (long long)mask->N);
     return run_attention(mask, q, k, v, out, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse,
                          reinterpret_cast<cudaStream_t>(stream), row_begin, row_end);
+}
+
+ris_status ris_attention_masked_local(ris_mask_t mask, int64_t row_begin, int64_t row_end, const void *q_rows,
+                                      const void *k, const void *v, void *out_rows, int32_t heads, int32_t kv_heads,
+                                      int32_t head_dim, int32_t dtype, int32_t out_dtype, const ris_rope_cfg *rope,
+                                      float *lse_rows, void *stream)
+{
+    if (mask == nullptr) return fail(RIS_ERR_INVALID, "mask is NULL");
+    RIS_TRY(validate_attention(q_rows, k, v, out_rows, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse_rows));
+    if (mask->heads_keyed > 1 && mask->heads_keyed != kv_heads)
+        return fail(RIS_ERR_INVALID, "mask keyed for %d KV heads, call has %d", mask->heads_keyed, kv_heads);
+    if (row_begin < 0 || row_end > mask->N || row_begin >= row_end)
+        return fail(RIS_ERR_INVALID, "rows [%lld, %lld) not a non-empty range of [0, %lld)", (long long)row_begin,
+                    (long long)row_end, (long long)mask->N);
+    if (mask->per_seed) return fail(RIS_ERR_UNSUPPORTED, "local rows of a per-seed mask (use ris_attention_masked_rows)");
+    return run_attention(mask, q_rows, k, v, out_rows, heads, kv_heads, head_dim, dtype, out_dtype, rope, lse_rows,
+                         reinterpret_cast<cudaStream_t>(stream), row_begin, row_end, true);
 }
 
 ris_status ris_row_split(const int64_t *row_ptr, int64_t N, int32_t parts, int64_t *bounds)

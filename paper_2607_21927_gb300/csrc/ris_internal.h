@@ -75,7 +75,8 @@ struct AttnArgs {
     const void *k_lo;      // bf16 path: low part of the rotated keys (k~ = k + k_lo), or null
     const void *v;         // [N][Hkv][D]
     void *out;             // [n_sets][N][Hq][D]
-    float *lse;            // [n_sets][Hq][N] or null
+    float *lse;            // [n_sets][Hq][lse_ld]: row i at lse[(s Hq + h) lse_ld + i], or null
+    int64_t lse_ld;        // N, or the row count of a call on local rows (lse then offset by -row0)
     const int64_t *row_ptr;  // [n_masks * N + 1] (null when dense)
     const void *col;       // keys (null when dense)
     const uint32_t *bitmap;  // causal bitmap rows (null when dense)

@@ -104,6 +104,8 @@ _SIGS = {
     "ris_attention_design": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32],
     "ris_attention_masked_rows": [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64] + [ctypes.c_void_p] * 4 +
                                  [ctypes.c_int32] * 5 + [ctypes.c_void_p] * 3,
+    "ris_attention_masked_local": [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64] + [ctypes.c_void_p] * 4 +
+                                  [ctypes.c_int32] * 5 + [ctypes.c_void_p] * 3,
     "ris_row_split": [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p],
     "ris_mask_row_split": [ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p],
     "ris_kernel_timer_read": [ctypes.c_void_p, ctypes.c_void_p],
@@ -541,6 +543,23 @@ def ris_attention_masked_rows(mask: Mask, row_begin: int, row_end: int, q, k, v,
         mask.handle, int(row_begin), int(row_end), _ptr(q), _ptr(k), _ptr(v), _ptr(out), Hq, Hkv, D, _dtype(q),
         _dtype(out), _ref(rope), _ptr(lse), _stream(stream)))
     return out
+
+
+def ris_attention_masked_local(mask: Mask, row_begin: int, row_end: int, q_rows, k, v, out_rows=None,
+                               rope: Optional[RopeCfg] = None, out_dtype=None, return_lse: bool = False, stream=None):
+    """Rows row_begin .. row_end-1 with only those rows of q in memory (q_rows [rows, Hq, D]);
+    k and v hold every position. Returns out_rows [rows, Hq, D] (and lse [Hq, rows])."""
+    for t in (q_rows, k, v):
+        assert t.is_cuda and t.is_contiguous() and t.dim() == 3
+    rows, Hq, D = q_rows.shape
+    Hkv = k.shape[1]
+    assert rows == row_end - row_begin and k.shape == v.shape and k.shape[2] == D
+    out_rows = _alloc_out(out_rows, (rows, Hq, D), out_dtype or q_rows.dtype, q_rows.device)
+    lse = torch.empty((Hq, rows), dtype=torch.float32, device=q_rows.device) if return_lse else None
+    _check("ris_attention_masked_local", lib().ris_attention_masked_local(
+        mask.handle, int(row_begin), int(row_end), _ptr(q_rows), _ptr(k), _ptr(v), _ptr(out_rows), Hq, Hkv, D,
+        _dtype(q_rows), _dtype(out_rows), _ref(rope), _ptr(lse), _stream(stream)))
+    return (out_rows, lse) if return_lse else out_rows
 
 
 def ris_row_split(row_ptr, parts: int):

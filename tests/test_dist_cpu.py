@@ -129,3 +129,48 @@ def test_row_shards_partition_rows_gloo(monkeypatch):
     assert res[1][1] == parts
     assert parts[0][0] == 0 and parts[0][1] == parts[1][0] and parts[1][1] == 2000
     assert parts[0][2] + parts[1][2] == total and abs(parts[0][2] - parts[1][2]) <= 0.01 * total
+
+
+def _kv_gather_rank(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
+                      LOCAL_RANK=str(rank))
+    sys.path.insert(0, ROOT)
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_21927_gb300 import inputs, ris, shard
+
+    dist.init_process_group("gloo")
+    N, Hkv, D = 2000, 2, 128
+    # the same pure function on every rank: the mask's row counts and the balanced cuts
+    rp = _oracle_row_ptr(N, 0.03, 2)
+    b = ris.ris_row_split(rp, world)
+    _, k, v = inputs.make_qkv(N, 6, Hkv, D, dtype=torch.bfloat16, seed=9, outliers=True)
+    # this rank holds only its own rows of K and V
+    k_full, v_full = shard.kv_allgather(k[b[rank]:b[rank + 1]].clone(), v[b[rank]:b[rank + 1]].clone(), b)
+    q.put((rank, b, bool(torch.equal(k_full, k)), bool(torch.equal(v_full, v)), tuple(k_full.shape)))
+    dist.destroy_process_group()
+
+
+@pytest.mark.timeout(120)
+@pytest.mark.parametrize("world", [2, 3])
+def test_kv_allgather_of_row_shards_gloo(monkeypatch, world):
+    """Ranks that hold only their own balanced row range of K and V rebuild the layer's whole K
+    and V bit for bit with one all-gather each (ragged parts padded to the longest)."""
+    monkeypatch.setenv("CUDA_VISIBLE_DEVICES", "")
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_kv_gather_rank, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(90)
+        assert p.exitcode == 0
+    res = sorted(q.get(timeout=5) for _ in range(world))
+    bounds = res[0][1]
+    assert len(bounds) == world + 1 and len({tuple(r[1]) for r in res}) == 1
+    assert len({bounds[k + 1] - bounds[k] for k in range(world)}) > 1  # ragged parts
+    for rank, _, k_ok, v_ok, shape in res:
+        assert k_ok and v_ok and shape == (2000, 2, 128), rank

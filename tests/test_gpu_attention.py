@@ -499,3 +499,44 @@ def test_benchmarked_layers_bf16_output(N, mode, d, S, layer):
     ref, _ = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e6, 32768, rows=rows)
     err, rel = check_bf16_path(to_np(out[rows]), ref, out_bf16=True)
     print(f"design {design}: max-abs {err:.2e}, rel-L2 {rel:.2e}")
+
+
+@pytest.mark.parametrize("mode,d,S,W", [(0, 0.02, 3, 1), (0, 0.5, 2, 1), (2, 1.0, 1, 1), (1, 0.1, 1, 1), (0, 0.01, 1, 300)],
+                         ids=["gather", "tiles", "dense", "suffix_split_blocks", "suffix_split_window"])
+def test_local_row_shards_reassemble_the_layer(mode, d, S, W):
+    """The row-sharded prefill with K/V all-gather, its ranks run one after the other on one
+    GPU: every rank holds only its rows of q (and gets the whole K and V, as the all-gather
+    returns them), calls ris_attention_masked_local, and the parts reassemble the whole-layer
+    output and log-sum-exp bit for bit, in every design."""
+    N, Hq, Hkv, D = 1700, 6, 2, 128
+    (q, k, v), _ = make_inputs(N, Hq, Hkv, D, seed=53, outliers=True)
+    m = ris.ris_mask_generate(N, Hkv, mode, d, list(range(S)), opts=ris.mask_opts(local_window=W))
+    rope = ris.rope_cfg(3, 1e6, 256)
+    whole, lse = ris.ris_attention_masked(m, q, k, v, rope=rope, out_dtype=torch.float32, return_lse=True)
+    b = ris.ris_mask_row_split(m, 3)
+    parts, lparts = [], []
+    for r in range(3):
+        o, l = ris.ris_attention_masked_local(m, b[r], b[r + 1], q[b[r]:b[r + 1]].clone(), k, v, rope=rope,
+                                              out_dtype=torch.float32, return_lse=True)
+        parts.append(o)
+        lparts.append(l)
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    assert torch.equal(torch.cat(parts, 0), whole)
+    assert torch.equal(torch.cat(lparts, 1), lse)
+    # without RoPE (q and k used as given) and bf16 outputs
+    whole16 = ris.ris_attention_masked(m, q, k, v)
+    part = ris.ris_attention_masked_local(m, b[1], b[2], q[b[1]:b[2]].clone(), k, v)
+    torch.cuda.synchronize()
+    assert torch.equal(part, whole16[b[1]:b[2]])
+    m.free()
+
+
+def test_local_rows_refuse_per_seed_masks():
+    N, Hq, Hkv, D = 300, 6, 2, 128
+    (q, k, v), _ = make_inputs(N, Hq, Hkv, D, seed=5)
+    m = ris.ris_mask_generate(N, Hkv, 0, 0.05, [1, 2], per_seed=True)
+    with pytest.raises(ris.RisError) as e:
+        ris.ris_attention_masked_local(m, 0, 100, q[:100].clone(), k, v)
+    assert e.value.status == ris.RIS_ERR_UNSUPPORTED
+    m.free()
