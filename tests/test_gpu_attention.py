@@ -540,3 +540,30 @@ def test_local_rows_refuse_per_seed_masks():
         ris.ris_attention_masked_local(m, 0, 100, q[:100].clone(), k, v)
     assert e.value.status == ris.RIS_ERR_UNSUPPORTED
     m.free()
+
+
+@pytest.mark.parametrize("scale_exp", [14, 20])
+def test_tile_values_beyond_fp16_range(scale_exp):
+    """The tile kernel takes the values as fp16 scaled by a power of two chosen from their
+    largest magnitude (none below 2^14). Values scaled by 2^14 and 2^20 (beyond fp16's 65504)
+    must give exactly that multiple of the unscaled output (the scale is a power of two, so
+    every operand and the fp32 accumulation scale exactly), within the parity tolerance of the
+    oracle once divided back, for the tiles, the dense mode and the dense-suffix split."""
+    N, Hq, Hkv, D = 3000, 6, 2, 128  # Structural blocks of 300 tokens: the dense-suffix split
+    (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=61, outliers=True)
+    big = v * (2.0 ** scale_exp)
+    rope = ris.rope_cfg(3, 1e6, 256)
+    for mode, d, S, design in ((0, 0.5, 2, 2), (2, 1.0, 1, 2), (1, 0.1, 1, 4)):
+        m = ris.ris_mask_generate(N, Hkv, mode, d, list(range(S)))
+        assert ris.ris_attention_design(m, torch.bfloat16, D) == design
+        base = ris.ris_attention_masked(m, q, k, v, rope=rope, out_dtype=torch.float32)
+        out = ris.ris_attention_masked(m, q, k, big, rope=rope, out_dtype=torch.float32)
+        torch.cuda.synchronize()
+        ris.ris_device_status()
+        m.free()
+        assert torch.isfinite(out).all()
+        scaled_back = out / (2.0 ** scale_exp)
+        ref, _ = run_oracle(qn, kn, vn, mode, d, list(range(S)), 3, 1e6, 256)
+        check_bf16_path(to_np(scaled_back), ref)
+        # the same operands up to a power of two: within fp32 rounding of the unscaled output
+        assert torch.allclose(scaled_back, base, rtol=1e-5, atol=1e-5)
