@@ -822,14 +822,17 @@ def main():
                         "flops": "algorithmic: 4 * head_dim * query heads per sampled pair",
                         "design_frac": (dense / (tc * 1e12)) / (mean_ms / 1e3),
                         "design_note": "dense-causal tile FLOPs / sustained bf16 peak over the launch time (the "
-                                       "kernel issues 2x that: three score products for the hi/lo splits of "
-                                       "q and k, one value product)"})
+                                       "kernel issues 1.5x that at head dim 128: an fp16 score product, two "
+                                       "e4m3 score corrections at twice the rate, one fp16 value product)"})
             if rope is not None and w["dtype"] == "bf16":
-                # rotated bf16 inputs: three score products (q hi/lo x k hi/lo) and one value
-                # product (fp16 P against fp16 values) per tile, all of them tensor-core work
-                ent["issued_frac"] = 2.0 * ent["design_frac"]
-                ent["issued_note"] = ("issued 16-bit tensor-core FLOPs (4 products of 128x128x128 per causal tile "
-                                      "pair) / sustained bf16 peak over the launch time")
+                # rotated bf16 inputs at head dim 128 (bounds of |q~| |k~| well inside e4m3's range
+                # here): per tile pair one fp16 score product, two e4m3 correction products (each
+                # half the time of a 16-bit one) and one fp16 value product; at head dim 64, three
+                # bf16 score products and the value product
+                ent["issued_frac"] = (1.5 if D == 128 else 2.0) * ent["design_frac"]
+                ent["issued_note"] = ("issued tensor-core work in 16-bit-equivalent products of 128x128x128 per "
+                                      "causal tile pair (3 at head dim 128, 4 at 64) / sustained bf16 peak over the "
+                                      "launch time")
         else:
             # gathered pairs: all of them, or with the dense-suffix split all but the suffixes
             # (whose tile pass is inside the launch time: the split's two launches are timed as one)

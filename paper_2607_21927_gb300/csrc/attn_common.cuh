@@ -72,6 +72,32 @@ __device__ __forceinline__ int v_scale_exp(float vmax)
     return e >= 14 ? e - 13 : 0;
 }
 
+// 2^e as a float, for -126 <= e <= 127
+__device__ __forceinline__ float pow2i(int e) { return __uint_as_float((uint32_t)(127 + e) << 23); }
+
+// Scores of the tile kernel with fp8 corrections (rotated queries and keys, head dim 128):
+// q = q_h + q_l and k = k_h + k_l with fp16 q_h, k_h, and
+//   q.k ~ q_h.k_h + 2^-12 (e4m3(q_h 2^-ea) . e4m3(k_l 2^(12+ea)) + e4m3(q_l 2^(12+eb)) . e4m3(k_h 2^-eb)),
+// the dropped q_l.k_l being below 2^-22 of q.k. The exponents keep every e4m3 operand within
+// its range of 448 given bounds mq >= |q~| and mk >= |k~| (|k_l| <= 2^-11 |k|, so
+// |k_l 2^(12+ea)| <= 2^(1+ea) mk); false when no pair exists (very large q and k together), and
+// the call then keeps the bf16 hi / lo scheme. The RoPE kernel that writes the operands and the
+// tile kernel that reads them take the exponents from the same bounds, so they agree.
+__device__ __forceinline__ int ceil_log2_ratio(float x, float y)  // ceil(log2(x / y)) for x, y > 0
+{
+    int e;
+    const float m = frexpf(x / y, &e);  // x / y = m 2^e, m in [0.5, 1)
+    return m == 0.5f ? e - 1 : e;
+}
+__device__ __forceinline__ bool fp8_score_scales(float mq, float mk, int &ea, int &eb)
+{
+    if (!(mq > 0.f) || !(mk > 0.f) || !(mq < 1e30f) || !(mk < 1e30f)) return false;
+    ea = ceil_log2_ratio(mq, 448.f);
+    eb = ceil_log2_ratio(mk, 448.f);
+    if (ea < -40 || ea > 40 || eb < -40 || eb > 40) return false;
+    return ldexpf(mk, 1 + ea) <= 448.f && ldexpf(mq, 1 + eb) <= 448.f;
+}
+
 __device__ __forceinline__ float warp_max(float x)
 {
 #pragma unroll

@@ -213,6 +213,29 @@ __device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint
         : "memory");
 }
 
+// kind::f8f6f4 (e4m3 x e4m3 with the instruction descriptor's format fields 0), A from TMEM
+// (four 8-bit values per column), B from shared memory.
+__device__ __forceinline__ void tc_mma_ts_f8(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+
+// kind::f16 accumulating onto D scaled by 2^-12 on entry: D = A B + 2^-12 D.
+__device__ __forceinline__ void tc_mma_ts_scaled12(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, 1, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p, 12;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc)
+        : "memory");
+}
+
 __device__ __forceinline__ void tc_commit(uint32_t bar)
 {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
@@ -496,6 +519,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             // O[128 x DT] += P V, V MN-major (fp16 P against fp16 values, or bf16 P hi / lo
             // against bf16 values)
             constexpr uint32_t ID_O = kP16 ? idesc_f16(BM, DT, true) : idesc_bf16(BM, DT, true);
+            // fp8-correction scores (rotated q / k at head dim 128, operands written by
+            // launch_rope_tile8 when the bounds allow): the same bytes in the same places as the
+            // bf16 pair, read as fp16 hi parts (query columns 0-63, key bytes 0-255 of a row) and
+            // e4m3 corrections (query columns 64-95 / 96-127, key boxes at KV_ARR / KV_ARR + KV_BLK)
+            int ea = 0, eb = 0;
+            const bool use8 = DT == 128 && SPLIT && a.qk_bound != nullptr &&
+                              fp8_score_scales(a.qk_bound[0], a.qk_bound[1], ea, eb);
+            constexpr uint32_t ID_SH = idesc_f16(BM, BN, false);  // fp16 x fp16 (and e4m3 x e4m3 for kind::f8f6f4)
             ok = mbar_wait(smem_u32(&bars[B_Q]), 0, wl);
             tc_fence_after();
             auto issue_s = [&](int j) {
@@ -503,6 +534,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t kv = sbase + OFF_K + (j % kStages) * K_STAGE;
                 const uint32_t dt = (j & 1) ? t_s1 : t_s0;
                 uint32_t acc = 0;
+                if (use8) {
+                    // 2^12 (q_h8 k_l8 + q_l8 k_h8): two e4m3 products of 4 k-steps of 32
+                    for (int prod = 0; prod < 2; ++prod) {
+                        const uint32_t qa = t_q + DT / 2 + (prod == 0 ? 0 : DT / 4);
+                        const uint32_t kb = kv + KV_ARR + (prod == 0 ? KV_BLK : 0);
+                        for (int ks = 0; ks < DT / 32; ++ks) {
+                            tc_mma_ts_f8(dt, qa + 8 * ks, sdesc(kb + ks * 32, 16, 1024), ID_SH, acc);
+                            acc = 1;
+                        }
+                    }
+                    // + q_h k_h in fp16, the corrections brought back by 2^-12 on the first k-step
+                    for (int ks = 0; ks < DT / 16; ++ks) {
+                        const uint64_t bd = sdesc(kv + (ks >> 2) * KV_BLK + (uint32_t)((ks & 3) * 32), 16, 1024);
+                        if (ks == 0)
+                            tc_mma_ts_scaled12(dt, t_q, bd, ID_SH);
+                        else
+                            tc_mma_ts(dt, t_q + 8 * ks, bd, ID_SH, 1u);
+                    }
+                    tc_commit(smem_u32(&bars[B_S_FULL + st]));
+                    if (j + kStages < n_kt) tc_commit(smem_u32(&bars[B_K_EMPTY + j % kStages]));  // keys free
+                    return;
+                }
                 // (A, B) pairs: (Q hi, K hi), (Q lo, K hi), (Q hi, K lo); 8 k-steps of 16 over D
                 // the query tile lives in TMEM (16-bit values packed two per column): A from TMEM
                 for (int prod = 0; prod < (SPLIT ? 3 : 1); ++prod) {

@@ -651,9 +651,12 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     const int design = design_of(m, dtype, head_dim, heads / kv_heads);
     const bool tile = design == 2, suffix = design == 4;
     const bool q_pair = tile || suffix;  // queries as a bf16 hi + lo pair
-    Scratch qt, qtl, kt, ktl, po, pl, v16, vmax;
+    Scratch qt, qtl, kt, ktl, po, pl, v16, vmax, bound;
     const void *qu = q, *ku = k, *kl = nullptr, *q_lo = nullptr;
     bool q_split = false;
+    // the tiles alone (not the dense-suffix split, whose gather reads the bf16 pairs), bf16
+    // inputs rotated here, head dim 128: fp8-correction scores when the bounds allow
+    const bool tile8 = tile && dtype == RIS_BF16 && head_dim == 128 && rope != nullptr && rope->kind != RIS_ROPE_NONE;
     if (rope != nullptr && rope->kind != RIS_ROPE_NONE) {
         RopeArgs ra{};
         double ms = 1.0;
@@ -673,20 +676,32 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         }
         RIS_CUDA(kt.alloc(nk * (dtype == RIS_BF16 ? 2 : 4), s));
         if (dtype == RIS_BF16) RIS_CUDA(ktl.alloc(nk * 2, s));
+        if (tile8) {
+            RIS_CUDA(bound.alloc(2 * sizeof(float), s));
+            RIS_CUDA(cudaMemsetAsync(bound.p, 0, 2 * sizeof(float), s));
+            RIS_CUDA(launch_rotation_bound(q, q_rows, heads, head_dim, ra.mscale, (float *)bound.p, s));
+            RIS_CUDA(launch_rotation_bound(k, N, kv_heads, head_dim, ra.mscale, (float *)bound.p + 1, s));
+        }
         ra.x_in = q;
         ra.x_out = qt.p;
         ra.x_out_lo = q_pair ? qtl.p : nullptr;
         ra.H = heads;
         ra.N = q_rows;
         ra.pos0 = q_first;
-        RIS_CUDA(launch_rope(ra, dtype, q_pair ? RIS_BF16 : RIS_F32, s));
+        if (tile8)
+            RIS_CUDA(launch_rope_tile8(ra, 0, (const float *)bound.p, s));
+        else
+            RIS_CUDA(launch_rope(ra, dtype, q_pair ? RIS_BF16 : RIS_F32, s));
         ra.N = N;
         ra.pos0 = 0;
         ra.x_in = k;
         ra.x_out = kt.p;
         ra.x_out_lo = ktl.p;
         ra.H = kv_heads;
-        RIS_CUDA(launch_rope(ra, dtype, dtype, s));
+        if (tile8)
+            RIS_CUDA(launch_rope_tile8(ra, 1, (const float *)bound.p, s));
+        else
+            RIS_CUDA(launch_rope(ra, dtype, dtype, s));
         qu = back(qt.p, (size_t)heads * head_dim * (q_pair ? 2 : 4));
         q_lo = back(qtl.p, (size_t)heads * head_dim * 2);
         ku = kt.p;
@@ -727,6 +742,7 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         RIS_CUDA(launch_values_f16(v, (int64_t)nv, v16.p, (float *)vmax.p, s));
         a.v16 = v16.p;
         a.v_absmax = (const float *)vmax.p;
+        a.qk_bound = tile8 ? (const float *)bound.p : nullptr;
     }
     if (suffix) {
         RIS_CUDA(po.alloc((size_t)N * heads * head_dim * sizeof(float), s));

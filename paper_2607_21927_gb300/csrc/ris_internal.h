@@ -103,6 +103,9 @@ struct AttnArgs {
     int64_t n_tasks;       // n_sets * (row1 - row0) * Hkv
     const void *v16;       // tile kernel: the values as fp16, scaled by 2^-E (launch_values_f16)
     const float *v_absmax; // tile kernel: max |v| over the values (device), from which E follows
+    const float *qk_bound; // tile kernel, head dim 128 with rotated q / k: bounds of |q~| and |k~|
+                           // (device, two floats) when the RoPE kernels wrote the fp8-correction
+                           // operands (launch_rope_tile8), else null
     int64_t wait_limit;    // tile kernel: cycles a device-side wait may take (0: about 2^31)
     int32_t debug_no_loads;  // tile kernel, tests only: the loader issues no copies, so the
                              // first wait on them gives up (ris_debug_tile_stall)
@@ -170,6 +173,17 @@ unsigned int read_decode_error();
 
 // dtype_in / dtype_out are ris_dtype values.
 cudaError_t launch_rope(const RopeArgs &a, int dtype_in, int dtype_out, cudaStream_t s);
+
+// Bounds of the rotated values of x [N][H][D] (bf16): mscale times the largest pair norm
+// |(x_c, x_{c+D/2})|, with a margin for the fp32 rotation, atomically maxed into *bound (a
+// float, >= 0 bit patterns; zero it first).
+cudaError_t launch_rotation_bound(const void *x, int64_t N, int H, int D, float mscale, float *bound,
+                                  cudaStream_t s);
+// RoPE (bf16 in) for the tile kernel's fp8-correction scores: role 0 queries, 1 keys; x_out gets
+// fp16 hi parts and x_out_lo, per (token, head), D bytes of e4m3 hi-part corrections then D bytes
+// of e4m3 lo-part corrections (see fp8_score_scales), or, when the bounds at qk_bound rule the
+// scheme out, the bf16 hi / lo pair of launch_rope.
+cudaError_t launch_rope_tile8(const RopeArgs &a, int role, const float *qk_bound, cudaStream_t s);
 
 // bf16 values v[n] (n a multiple of 8, 16-byte aligned) -> *vmax = max |v| (vmax zeroed by
 // this call) and v16[i] = fp16(v[i] / 2^E), E = v_scale_exp(max |v|): the fp16 operand of the

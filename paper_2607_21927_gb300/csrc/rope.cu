@@ -8,6 +8,7 @@
 // and one write of the tensor.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
+#include <cuda_fp8.h>
 
 #include <cstdint>
 
@@ -65,6 +66,72 @@ __global__ void k_rope(const RopeArgs a)
     }
 }
 
+// The largest pair norm of x [rows][D] (bf16), times mscale with a margin of 2^-20 for the
+// rotation's fp32 rounding: a bound of every rotated value (a rotation keeps the pair norm).
+__global__ void k_rotation_bound(const __nv_bfloat16 *x, int64_t rows, int D, float mscale, unsigned int *bound)
+{
+    const int half = D >> 1;
+    float m = 0.f;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < rows * half; t += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = t / half;
+        const int c = (int)(t - r * half);
+        const float x0 = __bfloat162float(x[r * D + c]), x1 = __bfloat162float(x[r * D + c + half]);
+        m = fmaxf(m, sqrtf(fmaf(x0, x0, x1 * x1)));
+    }
+    m = warp_max(m) * mscale * (1.f + 0x1p-20f);
+    if ((threadIdx.x & 31) == 0) atomicMax(bound, __float_as_uint(m));
+}
+
+__device__ __forceinline__ unsigned char to_e4m3(float x)
+{
+    return (unsigned char)__nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3);
+}
+
+// RoPE for the tile kernel's fp8-correction scores (see fp8_score_scales): the same rotation
+// as k_rope, then fp16 hi parts into x_out and the two e4m3 correction operands into x_out_lo,
+// or the bf16 hi / lo pair when the bounds rule the scheme out. ROLE 0: queries (hi part
+// scaled by 2^-ea, lo part by 2^(12+eb)); ROLE 1: keys (hi part by 2^-eb, lo part by 2^(12+ea)).
+template <int ROLE>
+__global__ void k_rope_tile8(const RopeArgs a, const float *qk_bound)
+{
+    const int half = a.D >> 1;
+    const int c = threadIdx.x;  // blockDim.x == D/2
+    const int64_t p = (int64_t)blockIdx.x * kRopeTokens + threadIdx.y;
+    if (p >= a.N || c >= half) return;
+    int ea = 0, eb = 0;
+    const bool f8 = fp8_score_scales(qk_bound[0], qk_bound[1], ea, eb);
+    const float s_hi = f8 ? pow2i(ROLE == 0 ? -ea : -eb) : 1.f;
+    const float s_lo = f8 ? pow2i(12 + (ROLE == 0 ? eb : ea)) : 1.f;
+    const double ang = (double)(p + a.pos0) * a.f[c];
+    const double n = rint(ang * 0.15915494309189533577);
+    double red = fma(-n, 6.28318530717958623200, ang);
+    red = fma(-n, 2.4492935982947064e-16, red);
+    float sn, cs;
+    sincosf((float)red, &sn, &cs);
+    const __nv_bfloat16 *xi = reinterpret_cast<const __nv_bfloat16 *>(a.x_in) + p * (int64_t)a.H * a.D;
+    for (int h = 0; h < a.H; ++h) {
+        const float x0 = __bfloat162float(xi[h * a.D + c]);
+        const float x1 = __bfloat162float(xi[h * a.D + c + half]);
+        const float y[2] = {fmaf(x0, cs, -x1 * sn) * a.mscale, fmaf(x1, cs, x0 * sn) * a.mscale};
+        const int64_t e0 = (p * (int64_t)a.H + h) * a.D;
+        for (int u = 0; u < 2; ++u) {
+            const int cc = c + u * half;
+            if (f8) {
+                const __half hh = __float2half_rn(y[u]);
+                const float hv = __half2float(hh);
+                reinterpret_cast<__half *>(a.x_out)[e0 + cc] = hh;
+                unsigned char *lo = reinterpret_cast<unsigned char *>(a.x_out_lo) + 2 * e0;
+                lo[cc] = to_e4m3(hv * s_hi);
+                lo[a.D + cc] = to_e4m3((y[u] - hv) * s_lo);
+            } else {
+                const __nv_bfloat16 hb = __float2bfloat16_rn(y[u]);
+                reinterpret_cast<__nv_bfloat16 *>(a.x_out)[e0 + cc] = hb;
+                reinterpret_cast<__nv_bfloat16 *>(a.x_out_lo)[e0 + cc] = __float2bfloat16_rn(y[u] - __bfloat162float(hb));
+            }
+        }
+    }
+}
+
 // max |v| over 8 bf16 values per thread and step (grid-stride), one atomic per warp; |v| >= 0,
 // so the order of the float bit patterns is the order of the values
 __global__ void k_absmax_bf16(const uint4 *v, int64_t n8, unsigned int *vmax)
@@ -101,6 +168,30 @@ __global__ void k_values_f16(const uint4 *v, int64_t n8, const float *vmax, uint
 }
 
 }  // namespace
+
+cudaError_t launch_rotation_bound(const void *x, int64_t N, int H, int D, float mscale, float *bound, cudaStream_t s)
+{
+    const int64_t work = N * H * (D / 2);
+    const int threads = 256;
+    const int64_t need = (work + threads - 1) / threads;
+    const unsigned grid = (unsigned)(need < 152 * 8 ? (need > 0 ? need : 1) : 152 * 8);
+    k_rotation_bound<<<grid, threads, 0, s>>>(reinterpret_cast<const __nv_bfloat16 *>(x), N * H, D, mscale,
+                                              reinterpret_cast<unsigned int *>(bound));
+    note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_rope_tile8(const RopeArgs &a, int role, const float *qk_bound, cudaStream_t s)
+{
+    const dim3 block(a.D / 2, kRopeTokens);
+    const dim3 grid((unsigned)((a.N + kRopeTokens - 1) / kRopeTokens));
+    if (role == 0)
+        k_rope_tile8<0><<<grid, block, 0, s>>>(a, qk_bound);
+    else
+        k_rope_tile8<1><<<grid, block, 0, s>>>(a, qk_bound);
+    note_launch();
+    return cudaGetLastError();
+}
 
 cudaError_t launch_values_f16(const void *v, int64_t n, void *v16, float *vmax, cudaStream_t s)
 {

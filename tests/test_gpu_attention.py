@@ -567,3 +567,32 @@ def test_tile_values_beyond_fp16_range(scale_exp):
         check_bf16_path(to_np(scaled_back), ref)
         # the same operands up to a power of two: within fp32 rounding of the unscaled output
         assert torch.allclose(scaled_back, base, rtol=1e-5, atol=1e-5)
+
+
+def test_tile_scores_fall_back_when_q_and_k_are_too_large_for_fp8():
+    """Tile scores use fp16 products with e4m3 correction products when bounds of |q~| and
+    |k~| allow (their product below about 1e5); beyond that the call keeps the bf16 hi / lo
+    scheme. Queries and keys with one channel of 900 each, in channel pairs where the other
+    tensor is zero (so the scores stay moderate), take the fallback and must still match the
+    oracle; the same inputs with those channels at 9 take the fp8 path."""
+    N, Hq, Hkv, D = 1200, 6, 2, 128
+    for big in (900.0, 9.0):
+        (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=67, outliers=True)
+        for t in (q, qn):
+            t[:, :, 3] = big
+            t[:, :, 5] = 0
+            t[:, :, 5 + D // 2] = 0
+        for t in (k, kn):
+            t[:, :, 5] = big
+            t[:, :, 3] = 0
+            t[:, :, 3 + D // 2] = 0
+        m = ris.ris_mask_generate(N, Hkv, 0, 0.5, [1, 2])
+        assert ris.ris_attention_design(m, torch.bfloat16, D) == 2
+        out, lse = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e6, 256), out_dtype=torch.float32,
+                                            return_lse=True)
+        torch.cuda.synchronize()
+        ris.ris_device_status()
+        m.free()
+        ref, ref_lse = run_oracle(qn, kn, vn, 0, 0.5, [1, 2], 3, 1e6, 256)
+        check_bf16_path(to_np(out), ref)
+        np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
