@@ -193,13 +193,13 @@ const char *forced_design()
 
 
 // Union density at and above which masked dense tiles beat gathering pair by pair (bf16,
-// head dim 128): a tile costs the dense causal products (three score products for the hi/lo
-// splits and one value product) whatever the mask, a gathered pair 1.5 KB of K/V rows.
-// Measured crossover on Qwen2-shaped layers (head dim 128): 7.0% of the causal pairs at
-// N = 32768 and 6.9% at N = 65536 (tiles 4.11 / 16.2 ms per launch, the gather 4.00 / 16.0 ms
-// at 6.8%); on TinyLlama-shaped layers (head dim 64, 32 query and 4 KV heads, N = 16384)
-// 13.6%, where the tiles are half the products but the same softmax work.
-constexpr double kTileDensity = 0.069;
+// head dim 128): a tile costs the dense causal products (an fp16 score product, two e4m3 score
+// corrections and one value product) whatever the mask, a gathered pair 1.5 KB of K/V rows.
+// Measured crossover on Qwen2-shaped layers (head dim 128): 6.3% of the causal pairs at
+// N = 32768 and 6.1% at N = 65536 (tiles 3.69 / 14.4 ms per launch, the gather 3.46 / 13.8 ms
+// at 5.9%); on TinyLlama-shaped layers (head dim 64, 32 query and 4 KV heads, N = 16384, three
+// bf16 score products) 13.6%, where the tiles are half the products but the same softmax work.
+constexpr double kTileDensity = 0.062;
 constexpr double kTileDensity64 = 0.136;
 
 // Shortest dense span (Structural block or local window) for which the split pays: two
