@@ -68,17 +68,25 @@ __global__ void k_rope(const RopeArgs a)
 
 // The largest pair norm of x [rows][D] (bf16), times mscale with a margin of 2^-20 for the
 // rotation's fp32 rounding: a bound of every rotated value (a rotation keeps the pair norm).
+// Each thread takes 8 consecutive pairs (16-byte loads of both halves of a row).
 __global__ void k_rotation_bound(const __nv_bfloat16 *x, int64_t rows, int D, float mscale, unsigned int *bound)
 {
-    const int half = D >> 1;
+    const int half = D >> 1, per_row = half / 8;
     float m = 0.f;
-    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < rows * half; t += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t r = t / half;
-        const int c = (int)(t - r * half);
-        const float x0 = __bfloat162float(x[r * D + c]), x1 = __bfloat162float(x[r * D + c + half]);
-        m = fmaxf(m, sqrtf(fmaf(x0, x0, x1 * x1)));
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < rows * per_row; t += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = t / per_row;
+        const int c = 8 * (int)(t - r * per_row);
+        const uint4 a = *reinterpret_cast<const uint4 *>(x + r * D + c);
+        const uint4 b = *reinterpret_cast<const uint4 *>(x + r * D + c + half);
+        const uint32_t wa[4] = {a.x, a.y, a.z, a.w}, wb[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float a0 = __uint_as_float(wa[k] << 16), a1 = __uint_as_float(wa[k] & 0xFFFF0000u);
+            const float b0 = __uint_as_float(wb[k] << 16), b1 = __uint_as_float(wb[k] & 0xFFFF0000u);
+            m = fmaxf(m, fmaxf(fmaf(a0, a0, b0 * b0), fmaf(a1, a1, b1 * b1)));
+        }
     }
-    m = warp_max(m) * mscale * (1.f + 0x1p-20f);
+    m = sqrtf(warp_max(m)) * mscale * (1.f + 0x1p-20f);
     if ((threadIdx.x & 31) == 0) atomicMax(bound, __float_as_uint(m));
 }
 
@@ -171,7 +179,8 @@ __global__ void k_values_f16(const uint4 *v, int64_t n8, const float *vmax, uint
 
 cudaError_t launch_rotation_bound(const void *x, int64_t N, int H, int D, float mscale, float *bound, cudaStream_t s)
 {
-    const int64_t work = N * H * (D / 2);
+    if ((D % 16) != 0) return cudaErrorInvalidValue;
+    const int64_t work = N * H * (D / 16);
     const int threads = 256;
     const int64_t need = (work + threads - 1) / threads;
     const unsigned grid = (unsigned)(need < 152 * 8 ? (need > 0 ? need : 1) : 152 * 8);
