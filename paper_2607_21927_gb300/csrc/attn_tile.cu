@@ -104,8 +104,8 @@ constexpr int SMEM_BYTES = OFF_K + kStages * (Smem<128>::K_STAGE + Smem<128>::V_
 // B_X: per group of kRowThreads softmax warps sharing rows (one per column quarter) and tile
 // parity, the exchange of their partial row maxima (and at the end their partial sums).
 enum Bar {
-    B_Q = 0, B_K_FULL = 1, B_K_EMPTY = 3, B_V_FULL = 5, B_V_EMPTY = 7, B_S_FULL = 9, B_S_EMPTY = 11, B_P_FULL = 13,
-    B_PV_DONE = 15, B_X = 17, B_END = 25, NBAR = 26
+    B_Q = 0, B_K_FULL = 1, B_V_FULL = 3, B_S_FULL = 5, B_S_EMPTY = 7, B_P_FULL = 9, B_PV_DONE = 11, B_X = 13,
+    B_END = 21, NBAR = 22
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -482,12 +482,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0 && a.debug_no_loads == 0) {
             // tile j: keys once the score products of tile j - 2 are done, then values once the
             // value product of tile j - 2 is (it was issued after the score products of tile
-            // j - 1, whose keys are already in flight: no wait here depends on a later load)
+            // j - 1, whose keys are already in flight: no wait here depends on a later load).
+            // The ring stages and the score / P buffers are both indexed by tile parity, so a
+            // stage is free exactly when the barrier that announces those products completes
+            // (S_FULL, PV_DONE): the loader waits on them instead of on barriers of its own,
+            // which saves the tensor pipe two commits per tile.
+            static_assert(kStages == 2, "ring stages share the parity of the score buffers");
             int nk = 0, nv = 0;  // tiles whose keys / values were requested
             for (int j = 0; j < n_kt && ok; ++j) {
                 const int st = j % kStages;
                 const uint32_t par = ((j / kStages) - 1) & 1;
-                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_K_EMPTY + st]), par, wl);
+                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_S_FULL + st]), par, wl);
                 if (!ok) break;
                 const uint32_t bk = smem_u32(&bars[B_K_FULL + st]);
                 const uint32_t dk = sbase + OFF_K + st * K_STAGE;
@@ -497,7 +502,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (SPLIT) tma_load_3d(dk + KV_ARR + blk * KV_BLK, &maps.kl, 64 * blk, g, (kt0 + j) * BN, bk);
                 }
                 nk = j + 1;
-                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_V_EMPTY + st]), par, wl);
+                if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_PV_DONE + st]), par, wl);
                 if (!ok) break;
                 const uint32_t bv = smem_u32(&bars[B_V_FULL + st]);
                 const uint32_t dv = sbase + OFF_V + st * V_STAGE;
@@ -553,7 +558,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc_mma_ts(dt, t_q + 8 * ks, bd, ID_SH, 1u);
                     }
                     tc_commit(smem_u32(&bars[B_S_FULL + st]));
-                    if (j + kStages < n_kt) tc_commit(smem_u32(&bars[B_K_EMPTY + j % kStages]));  // keys free
                     return;
                 }
                 // (A, B) pairs: (Q hi, K hi), (Q lo, K hi), (Q hi, K lo); 8 k-steps of 16 over D
@@ -569,7 +573,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 tc_commit(smem_u32(&bars[B_S_FULL + st]));
-                if (j + kStages < n_kt) tc_commit(smem_u32(&bars[B_K_EMPTY + j % kStages]));  // keys free
             };
             auto issue_o = [&](int j) {
                 const int st = j % kStages;
@@ -586,7 +589,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tc_mma_ts(t_o, pt + (BN / 2) * prod + 8 * ks, bd, ID_O, (j > 0 || prod > 0 || ks > 0) ? 1u : 0u);
                     }
                 }
-                if (j + kStages < n_kt) tc_commit(smem_u32(&bars[B_V_EMPTY + st]));  // values free
                 tc_commit(smem_u32(&bars[B_PV_DONE + (j & 1)]));
             };
             for (int j = 0; j < n_kt && ok; ++j) {
