@@ -33,6 +33,8 @@
 //   - P is split into bf16 hi + lo and O^T += V^T P_hi + V^T P_lo.
 // V is an exact bf16 input. Unrotated bf16 q/k are exact and take one product each.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
 
 #include <cstdint>
 
@@ -49,6 +51,39 @@ __device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1
         "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void mma16816_f16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                             uint32_t a3, uint32_t b0, uint32_t b1)
+{
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+        "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// e4m3 x e4m3 -> fp32, m16n8k32: four e4m3 values per 32-bit register, lowest byte first. A:
+// a0 / a2 row lane/4 at columns 4(lane%4) + [0, 4) / 16 + 4(lane%4) + [0, 4), a1 / a3 the same
+// of row lane/4 + 8; B: b0 / b1 rows 4(lane%4) + [0, 4) / 16 + 4(lane%4) + [0, 4) of column
+// lane/4; C as for m16n8k16.
+__device__ __forceinline__ void mma16832_e4m3(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                              uint32_t a3, uint32_t b0, uint32_t b1)
+{
+    asm volatile(
+        "mma.sync.aligned.m16n8k32.row.col.f32.e4m3.e4m3.f32 "
+        "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// two e4m3 values (lowest byte first) times s, as an fp16 pair
+__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two, float s)
+{
+    const __half2_raw hr = __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)(two & 0xFFFFu), __NV_E4M3);
+    const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&hr));
+    const __half2 h = __floats2half2_rn(f.x * s, f.y * s);
+    return *reinterpret_cast<const uint32_t *>(&h);
 }
 
 __device__ __forceinline__ uint32_t transpose8x8(uint32_t x)
@@ -143,9 +178,22 @@ constexpr float kLazyLog2 = 8.f;  // rescale O only when the row maximum grows b
 // after the other, requesting the next set's key range and first keys while the current set
 // runs and its first K/V rows during the current set's last group, so the load pipeline
 // never drains between sets; a.n_tasks counts (row, KV head) pairs.
-template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut, bool SEEDS>
-__global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
+// E8 (head dim 128, rotated bf16 inputs, 32-byte loads): the operands of the tile kernel's
+// fp8-correction scheme, written by launch_rope_tile8 (see fp8_score_scales): keys as fp16 hi
+// parts (a.k) and, in each (token, head)'s 2D-byte record of a.k_lo, e4m3(k_h 2^-eb) at bytes
+// [0, D) and e4m3(k_l 2^(12+ea)) at [D, 2D); queries likewise (a.q, a.q_lo; 2^-ea and
+// 2^(12+eb)). The gather fetches only the fp16 hi part and the e4m3 lo part of a key row (384
+// bytes instead of 512) and forms
+//   S^T = K_h Q_h + K_h Q_l + 2^-12 e4m3(K_l) e4m3(Q_h)
+// with Q_l taken back to fp16 from its e4m3 operand: two fp16 products and one e4m3 product of
+// half the k-steps (m16n8k32) instead of three bf16 products. Each of the two approximated
+// terms is within about 2^-15 of |q||k| per channel, as in the tile kernel's scheme. (Widening
+// the e4m3 lo part to fp16 in registers for a third fp16 product instead measured slower than
+// the bf16 pairs: the conversions cost more than the bytes saved.)
+template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut, bool SEEDS, bool E8>
+__device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
 {
+    static_assert(!E8 || (D == 128 && QSPLIT && KSPLIT && WIDE), "the fp8 operands: head dim 128, 32-byte loads");
     constexpr int KSTEPS = D / 16;  // k-steps of the score product
     constexpr int KW = D / 8;       // 32-bit words of one K row per lane (D/4 elements)
     constexpr int VW = D / 16;      // 32-bit words of one V row per lane (D/8 elements)
@@ -180,13 +228,32 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
 
     // ---- query fragments (B operand of the score product), head p of this KV group
     uint32_t qh[KSTEPS][2], ql[KSTEPS][2];
+    uint32_t q8[E8 ? 8 : 1];  // E8: e4m3(q_h 2^-ea), elements 32q .. 32q + 31 (natural order)
     {
         const bool hv = p < a.G;
         const int64_t qrow = (t.i * a.Hq + (int64_t)t.g * a.G + (hv ? p : 0)) * D;
+        if constexpr (E8) {
+            const unsigned char *rec = reinterpret_cast<const unsigned char *>(a.q_lo) + 2 * qrow;
+            const uint4 x0 = hv ? *reinterpret_cast<const uint4 *>(rec + 32 * q) : make_uint4(0u, 0u, 0u, 0u);
+            const uint4 x1 = hv ? *reinterpret_cast<const uint4 *>(rec + 32 * q + 16) : make_uint4(0u, 0u, 0u, 0u);
+            q8[0] = x0.x; q8[1] = x0.y; q8[2] = x0.z; q8[3] = x0.w;
+            q8[4] = x1.x; q8[5] = x1.y; q8[6] = x1.z; q8[7] = x1.w;
+        }
+        const float ql_scale = E8 ? pow2i(-12 - eb) : 1.f;
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
             const int d0 = kelem<D, WIDE>(ks, q);
-            if (QSPLIT && a.q_lo != nullptr) {  // the split given as a bf16 pair
+            if constexpr (E8) {  // fp16 hi part; lo part from its e4m3 operand
+                const uint2 wh = hv ? *reinterpret_cast<const uint2 *>(reinterpret_cast<const __half *>(a.q) + qrow + d0)
+                                    : make_uint2(0u, 0u);
+                const uint32_t w8 = hv ? *reinterpret_cast<const uint32_t *>(
+                                             reinterpret_cast<const unsigned char *>(a.q_lo) + 2 * qrow + D + d0)
+                                       : 0u;
+                qh[ks][0] = wh.x;
+                qh[ks][1] = wh.y;
+                ql[ks][0] = e4m3x2_to_f16x2(w8, ql_scale);
+                ql[ks][1] = e4m3x2_to_f16x2(w8 >> 16, ql_scale);
+            } else if (QSPLIT && a.q_lo != nullptr) {  // the split given as a bf16 pair
                 const uint2 wh = hv ? *reinterpret_cast<const uint2 *>(reinterpret_cast<const __nv_bfloat16 *>(a.q) + qrow + d0)
                                     : make_uint2(0u, 0u);
                 const uint2 wl = hv ? *reinterpret_cast<const uint2 *>(reinterpret_cast<const __nv_bfloat16 *>(a.q_lo) + qrow + d0)
@@ -219,7 +286,11 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     const size_t row_bytes = (size_t)a.Hkv * D * sizeof(__nv_bfloat16);
     const size_t head_off = (size_t)t.g * D * sizeof(__nv_bfloat16);
     const char *kb = reinterpret_cast<const char *>(a.k) + head_off + 2 * kelem<D, WIDE>(0, q);
-    const char *kbl = KSPLIT ? reinterpret_cast<const char *>(a.k_lo) + head_off + 2 * kelem<D, WIDE>(0, q) : nullptr;
+    // E8: the e4m3 lo part of a key row, bytes D .. 2D - 1 of its record (the record stride is the
+    // hi part's row stride), elements 32q .. 32q + 31 to lane q
+    const char *kbl = !KSPLIT ? nullptr
+                      : E8    ? reinterpret_cast<const char *>(a.k_lo) + head_off + D + 32 * q
+                              : reinterpret_cast<const char *>(a.k_lo) + head_off + 2 * kelem<D, WIDE>(0, q);
     const char *vb = reinterpret_cast<const char *>(a.v) + head_off + 2 * velem<D, WIDE>(0, p);
 
     float o[MT][4];
@@ -287,7 +358,10 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         const int ik0 = slot(c0, c1, gs, p), ik1 = slot(c0, c1, gs, p + 8);
         load_row(kb + (size_t)ik0 * row_bytes, k0, KW, WIDE ? 128 : 64, WIDE);
         load_row(kb + (size_t)ik1 * row_bytes, k1, KW, WIDE ? 128 : 64, WIDE);
-        if (KSPLIT) {
+        if (E8) {
+            ldg32(kbl + (size_t)ik0 * row_bytes, kl0);
+            ldg32(kbl + (size_t)ik1 * row_bytes, kl1);
+        } else if (KSPLIT) {
             load_row(kbl + (size_t)ik0 * row_bytes, kl0, KW, WIDE ? 128 : 64, WIDE);
             load_row(kbl + (size_t)ik1 * row_bytes, kl1, KW, WIDE ? 128 : 64, WIDE);
         }
@@ -337,6 +411,17 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
         for (int c = 0; c < 2; ++c)
 #pragma unroll
             for (int e = 0; e < 4; ++e) sa[c][e] = sb[c][e] = sl[c][e] = 0.f;
+        if constexpr (E8) {
+#pragma unroll
+            for (int ks = 0; ks < KSTEPS; ++ks) {
+                mma16816_f16(sa[ks & 1], k0[2 * ks], k1[2 * ks], k0[2 * ks + 1], k1[2 * ks + 1], qh[ks][0], qh[ks][1]);
+                mma16816_f16(sb[ks & 1], k0[2 * ks], k1[2 * ks], k0[2 * ks + 1], k1[2 * ks + 1], ql[ks][0], ql[ks][1]);
+            }
+#pragma unroll
+            for (int ks = 0; ks < D / 32; ++ks)
+                mma16832_e4m3(sl[ks & 1], kl0[2 * ks], kl1[2 * ks], kl0[2 * ks + 1], kl1[2 * ks + 1], q8[2 * ks],
+                              q8[2 * ks + 1]);
+        } else {
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
             mma16816(sa[ks & 1], k0[2 * ks], k1[2 * ks], k0[2 * ks + 1], k1[2 * ks + 1], qh[ks][0], qh[ks][1]);
@@ -348,9 +433,12 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
                          kl1[(2 * ks + 1) % LW], qh[ks][0], qh[ks][1]);
             }
         }
+        }
         float s[4];
+        constexpr float kLoScale = E8 ? 0x1p-12f : 1.f;  // E8: the e4m3 product carries 2^12
 #pragma unroll
-        for (int e = 0; e < 4; ++e) s[e] = ((sa[0][e] + sa[1][e]) + (sb[0][e] + sb[1][e])) + (sl[0][e] + sl[1][e]);
+        for (int e = 0; e < 4; ++e)
+            s[e] = ((sa[0][e] + sa[1][e]) + (sb[0][e] + sb[1][e])) + kLoScale * (sl[0][e] + sl[1][e]);
         if (more)
             issue_k(n0, n1, gs1);
         else if (cross)
@@ -472,8 +560,24 @@ __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_b
     }  // sets
 }
 
-template <int D, bool QSPLIT, bool WIDE, typename TOut>
-cudaError_t launch_w(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t s)
+// F8: the queries and keys came from launch_rope_tile8; which of its two schemes it wrote
+// follows from the bounds at a.qk_bound, read here on the device as it did.
+template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut, bool SEEDS, bool F8>
+__global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
+{
+    if constexpr (F8) {
+        int ea = 0, eb = 0;
+        if (fp8_score_scales(a.qk_bound[0], a.qk_bound[1], ea, eb))
+            gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, true>(a, eb);
+        else
+            gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, false>(a, 0);
+    } else {
+        gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, false>(a, 0);
+    }
+}
+
+template <int D, bool QSPLIT, bool WIDE, typename TOut, bool F8>
+cudaError_t launch_f(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t s)
 {
     // rotated inputs: fp32 queries and hi + lo keys; as given: bf16 queries and keys
     constexpr bool KSPLIT = QSPLIT;
@@ -483,21 +587,34 @@ cudaError_t launch_w(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t 
         b.n_tasks = (a.row1 - a.row0) * a.Hkv;
         const unsigned grid = (unsigned)((b.n_tasks + kAttnWarps - 1) / kAttnWarps);
         if (col_bytes == 2)
-            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, true><<<grid, block, 0, s>>>(b);
+            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, true, F8><<<grid, block, 0, s>>>(b);
         else
-            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, true><<<grid, block, 0, s>>>(b);
+            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, true, F8><<<grid, block, 0, s>>>(b);
         note_launch();
         return cudaGetLastError();
     }
     const unsigned grid = (unsigned)((a.n_tasks + kAttnWarps - 1) / kAttnWarps);
     if (dense)
-        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, true, TOut, false><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, true, TOut, false, F8><<<grid, block, 0, s>>>(a);
     else if (col_bytes == 2)
-        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, false><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, false, F8><<<grid, block, 0, s>>>(a);
     else
-        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, false><<<grid, block, 0, s>>>(a);
+        k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, false, F8><<<grid, block, 0, s>>>(a);
     note_launch();
     return cudaGetLastError();
+}
+
+template <int D, bool QSPLIT, bool WIDE, typename TOut>
+cudaError_t launch_w(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t s)
+{
+    // operands in launch_rope_tile8's form (a.qk_bound set) are read only by the F8 kernel, which
+    // needs head dim 128 and 32-byte aligned inputs (the caller checks both)
+    if constexpr (D == 128 && QSPLIT && WIDE) {
+        if (a.qk_bound != nullptr) return launch_f<D, QSPLIT, WIDE, TOut, true>(a, col_bytes, dense, s);
+    } else {
+        if (a.qk_bound != nullptr) return cudaErrorInvalidValue;
+    }
+    return launch_f<D, QSPLIT, WIDE, TOut, false>(a, col_bytes, dense, s);
 }
 
 bool aligned32(const void *p) { return p == nullptr || (reinterpret_cast<uintptr_t>(p) & 31u) == 0; }

@@ -80,8 +80,9 @@ __device__ __forceinline__ float pow2i(int e) { return __uint_as_float((uint32_t
 //   q.k ~ q_h.k_h + 2^-12 (e4m3(q_h 2^-ea) . e4m3(k_l 2^(12+ea)) + e4m3(q_l 2^(12+eb)) . e4m3(k_h 2^-eb)),
 // the dropped q_l.k_l being below 2^-22 of q.k. The exponents keep every e4m3 operand within
 // its range of 448 given bounds mq >= |q~| and mk >= |k~| (|k_l| <= 2^-11 |k|, so
-// |k_l 2^(12+ea)| <= 2^(1+ea) mk); false when no pair exists (very large q and k together), and
-// the call then keeps the bf16 hi / lo scheme. The RoPE kernel that writes the operands and the
+// |k_l 2^(12+ea)| <= 2^(1+ea) mk), and the fp16 hi parts finite (bounds below 2^15); false
+// when no pair exists (very large q and k together, or either beyond fp16), and the call then
+// keeps the bf16 hi / lo scheme. The RoPE kernel that writes the operands and the
 // tile kernel that reads them take the exponents from the same bounds, so they agree.
 __device__ __forceinline__ int ceil_log2_ratio(float x, float y)  // ceil(log2(x / y)) for x, y > 0
 {
@@ -91,7 +92,7 @@ __device__ __forceinline__ int ceil_log2_ratio(float x, float y)  // ceil(log2(x
 }
 __device__ __forceinline__ bool fp8_score_scales(float mq, float mk, int &ea, int &eb)
 {
-    if (!(mq > 0.f) || !(mk > 0.f) || !(mq < 1e30f) || !(mk < 1e30f)) return false;
+    if (!(mq > 0.f) || !(mk > 0.f) || !(mq < 32768.f) || !(mk < 32768.f)) return false;
     ea = ceil_log2_ratio(mq, 448.f);
     eb = ceil_log2_ratio(mk, 448.f);
     if (ea < -40 || ea > 40 || eb < -40 || eb > 40) return false;

@@ -263,6 +263,7 @@ int design_of(const ris_mask_s *m, int32_t dtype, int32_t head_dim, int32_t grou
 }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned32(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 31u) == 0; }
 
 int64_t row_word_offset(int64_t i)
 {
@@ -650,14 +651,18 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     prepare_pool_once();
     const int design = design_of(m, dtype, head_dim, heads / kv_heads);
     const bool tile = design == 2, suffix = design == 4;
-    const bool q_pair = tile || suffix;  // queries as a bf16 hi + lo pair
+    const bool rotated = rope != nullptr && rope->kind != RIS_ROPE_NONE;
+    // bf16 inputs rotated here at head dim 128, on the tiles, the dense-suffix split or the bf16
+    // gather: fp16 + e4m3 score operands when the bounds allow (else the bf16 pairs), written
+    // by launch_rope_tile8 and read alike by the tile kernel and the gather (whose fp8 form
+    // needs its 32-byte loads: values 32-byte aligned)
+    const bool tile8 = dtype == RIS_BF16 && head_dim == 128 && rotated &&
+                       (tile || ((suffix || design == 0) && aligned32(v)));
+    const bool q_pair = tile || suffix || tile8;  // queries as a 16-bit pair (else fp32)
     Scratch qt, qtl, kt, ktl, po, pl, v16, vmax, bound;
     const void *qu = q, *ku = k, *kl = nullptr, *q_lo = nullptr;
     bool q_split = false;
-    // the tiles alone (not the dense-suffix split, whose gather reads the bf16 pairs), bf16
-    // inputs rotated here, head dim 128: fp8-correction scores when the bounds allow
-    const bool tile8 = tile && dtype == RIS_BF16 && head_dim == 128 && rope != nullptr && rope->kind != RIS_ROPE_NONE;
-    if (rope != nullptr && rope->kind != RIS_ROPE_NONE) {
+    if (rotated) {
         RopeArgs ra{};
         double ms = 1.0;
         RIS_TRY(ris_rope_freqs(rope, N, head_dim, ra.f, &ms));
@@ -665,9 +670,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         ra.D = head_dim;
         ra.mscale = (float)ms;
         const size_t nq = (size_t)q_rows * heads * head_dim, nk = (size_t)N * kv_heads * head_dim;
-        // rotated queries: fp32 (split into bf16 hi + lo by the gather kernels) or, when the
-        // tile kernel runs, a bf16 hi + lo pair; rotated keys in fp32, or for bf16 inputs a
-        // bf16 hi + lo pair
+        // rotated queries: fp32 (split into bf16 hi + lo by the gather kernels) or a 16-bit pair
+        // (the fp8 scheme's operands, or a bf16 hi + lo pair); rotated keys in fp32, or for bf16
+        // inputs a 16-bit pair
         if (q_pair) {
             RIS_CUDA(qt.alloc(nq * 2, s));
             RIS_CUDA(qtl.alloc(nq * 2, s));
@@ -734,7 +739,8 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.row0 = row0;
     a.row1 = row1;
     a.n_tasks = (int64_t)a.n_sets * (row1 - row0) * kv_heads;
-    if (q_pair) {
+    a.qk_bound = tile8 ? (const float *)bound.p : nullptr;
+    if (tile || suffix) {
         // the tile kernel's value product takes the values as fp16 (scaled into range)
         const size_t nv = (size_t)N * kv_heads * head_dim;
         RIS_CUDA(v16.alloc(nv * 2, s));
@@ -742,7 +748,6 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         RIS_CUDA(launch_values_f16(v, (int64_t)nv, v16.p, (float *)vmax.p, s));
         a.v16 = v16.p;
         a.v_absmax = (const float *)vmax.p;
-        a.qk_bound = tile8 ? (const float *)bound.p : nullptr;
     }
     if (suffix) {
         RIS_CUDA(po.alloc((size_t)N * heads * head_dim * sizeof(float), s));

@@ -569,30 +569,40 @@ def test_tile_values_beyond_fp16_range(scale_exp):
         assert torch.allclose(scaled_back, base, rtol=1e-5, atol=1e-5)
 
 
-def test_tile_scores_fall_back_when_q_and_k_are_too_large_for_fp8():
-    """Tile scores use fp16 products with e4m3 correction products when bounds of |q~| and
-    |k~| allow (their product below about 1e5); beyond that the call keeps the bf16 hi / lo
-    scheme. Queries and keys with one channel of 900 each, in channel pairs where the other
-    tensor is zero (so the scores stay moderate), take the fallback and must still match the
-    oracle; the same inputs with those channels at 9 take the fp8 path."""
-    N, Hq, Hkv, D = 1200, 6, 2, 128
-    for big in (900.0, 9.0):
-        (q, k, v), (qn, kn, vn) = make_inputs(N, Hq, Hkv, D, seed=67, outliers=True)
-        for t in (q, qn):
-            t[:, :, 3] = big
-            t[:, :, 5] = 0
-            t[:, :, 5 + D // 2] = 0
-        for t in (k, kn):
-            t[:, :, 5] = big
-            t[:, :, 3] = 0
-            t[:, :, 3 + D // 2] = 0
-        m = ris.ris_mask_generate(N, Hkv, 0, 0.5, [1, 2])
-        assert ris.ris_attention_design(m, torch.bfloat16, D) == 2
-        out, lse = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e6, 256), out_dtype=torch.float32,
-                                            return_lse=True)
-        torch.cuda.synchronize()
-        ris.ris_device_status()
-        m.free()
-        ref, ref_lse = run_oracle(qn, kn, vn, 0, 0.5, [1, 2], 3, 1e6, 256)
-        check_bf16_path(to_np(out), ref)
-        np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
+# (N, mode, density, seeds, design): the tiles, the register gather, the dense-suffix split
+FP8_SCHEME_CASES = [(1200, 0, 0.5, [1, 2], 2), (1200, 0, 0.02, [1], 0), (3000, 1, 0.1, [1], 4)]
+
+
+@pytest.mark.parametrize("case", ["fp8", "both_large", "q_beyond_fp16"])
+@pytest.mark.parametrize("N,mode,d,seeds,design", FP8_SCHEME_CASES)
+def test_fp8_score_scheme_and_its_fallback(N, mode, d, seeds, design, case):
+    """At head dim 128 with rotated bf16 inputs the tiles, the gather and the dense-suffix split
+    take fp16 score products with e4m3 corrections when bounds of |q~| and |k~| allow (their
+    product below about 1e5, each below 2^15 so that the fp16 hi parts stay finite); otherwise
+    the call keeps the bf16 hi / lo scheme, chosen on the device. Queries and keys get one large
+    channel each, in channel pairs where the other tensor is zero (so the scores stay moderate):
+    at 9 they take the fp8 path; at 900 each the product rules it out; a query channel of 69632
+    with keys scaled by 2^-7 passes the product rule but not fp16's range. Every case must match
+    the oracle."""
+    Hq, Hkv, D = 6, 2, 128
+    big_q, big_k, k_scale = {"fp8": (9.0, 9.0, 1.0), "both_large": (900.0, 900.0, 1.0),
+                             "q_beyond_fp16": (69632.0, 1.0, 2.0 ** -7)}[case]
+    (q, k, v), _ = make_inputs(N, Hq, Hkv, D, seed=67, outliers=True)
+    q[:, :, 3] = big_q
+    q[:, :, 5] = 0
+    q[:, :, 5 + D // 2] = 0
+    k.mul_(k_scale)
+    k[:, :, 5] = big_k
+    k[:, :, 3] = 0
+    k[:, :, 3 + D // 2] = 0
+    qn, kn, vn = to_np(q.cpu()), to_np(k.cpu()), to_np(v.cpu())
+    m = ris.ris_mask_generate(N, Hkv, mode, d, seeds)
+    assert ris.ris_attention_design(m, torch.bfloat16, D) == design
+    out, lse = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e6, 256), out_dtype=torch.float32,
+                                        return_lse=True)
+    torch.cuda.synchronize()
+    ris.ris_device_status()
+    m.free()
+    ref, ref_lse = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e6, 256)
+    check_bf16_path(to_np(out), ref)
+    np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
