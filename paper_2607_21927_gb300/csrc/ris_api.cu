@@ -654,7 +654,7 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     const bool rotated = rope != nullptr && rope->kind != RIS_ROPE_NONE;
     // bf16 inputs rotated here at head dim 128, on the tiles, the dense-suffix split or the bf16
     // gather: fp16 + e4m3 score operands when the bounds allow (else the bf16 pairs), written
-    // by launch_rope_tile8 and read alike by the tile kernel and the gather (whose fp8 form
+    // by launch_fp8_prep and read alike by the tile kernel and the gather (whose fp8 form
     // needs its 32-byte loads: values 32-byte aligned)
     const bool tile8 = dtype == RIS_BF16 && head_dim == 128 && rotated &&
                        (tile || ((suffix || design == 0) && aligned32(v)));
@@ -682,31 +682,44 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         RIS_CUDA(kt.alloc(nk * (dtype == RIS_BF16 ? 2 : 4), s));
         if (dtype == RIS_BF16) RIS_CUDA(ktl.alloc(nk * 2, s));
         if (tile8) {
-            RIS_CUDA(bound.alloc(2 * sizeof(float), s));
-            RIS_CUDA(cudaMemsetAsync(bound.p, 0, 2 * sizeof(float), s));
-            RIS_CUDA(launch_rotation_bound(q, q_rows, heads, head_dim, ra.mscale, (float *)bound.p, s));
-            RIS_CUDA(launch_rotation_bound(k, N, kv_heads, head_dim, ra.mscale, (float *)bound.p + 1, s));
-        }
-        ra.x_in = q;
-        ra.x_out = qt.p;
-        ra.x_out_lo = q_pair ? qtl.p : nullptr;
-        ra.H = heads;
-        ra.N = q_rows;
-        ra.pos0 = q_first;
-        if (tile8)
-            RIS_CUDA(launch_rope_tile8(ra, 0, (const float *)bound.p, s));
-        else
+            // bounds (and the values as fp16 for the tile kernels), then the operands: two launches
+            RIS_CUDA(bound.alloc(3 * sizeof(float), s));
+            if (tile || suffix) RIS_CUDA(v16.alloc(nk * 2, s));
+            Fp8PrepArgs pa{};
+            pa.q = q;
+            pa.k = k;
+            pa.v = v;
+            pa.q_hi = qt.p;
+            pa.q_lo = qtl.p;
+            pa.k_hi = kt.p;
+            pa.k_lo = ktl.p;
+            pa.v16 = (tile || suffix) ? v16.p : nullptr;
+            pa.bounds = (float *)bound.p;
+            pa.N = N;
+            pa.q_rows = q_rows;
+            pa.q_first = q_first;
+            pa.Hq = heads;
+            pa.Hkv = kv_heads;
+            pa.D = head_dim;
+            std::memcpy(pa.f, ra.f, sizeof(pa.f));
+            pa.mscale = ra.mscale;
+            RIS_CUDA(launch_fp8_prep(pa, s));
+        } else {
+            ra.x_in = q;
+            ra.x_out = qt.p;
+            ra.x_out_lo = q_pair ? qtl.p : nullptr;
+            ra.H = heads;
+            ra.N = q_rows;
+            ra.pos0 = q_first;
             RIS_CUDA(launch_rope(ra, dtype, q_pair ? RIS_BF16 : RIS_F32, s));
-        ra.N = N;
-        ra.pos0 = 0;
-        ra.x_in = k;
-        ra.x_out = kt.p;
-        ra.x_out_lo = ktl.p;
-        ra.H = kv_heads;
-        if (tile8)
-            RIS_CUDA(launch_rope_tile8(ra, 1, (const float *)bound.p, s));
-        else
+            ra.N = N;
+            ra.pos0 = 0;
+            ra.x_in = k;
+            ra.x_out = kt.p;
+            ra.x_out_lo = ktl.p;
+            ra.H = kv_heads;
             RIS_CUDA(launch_rope(ra, dtype, dtype, s));
+        }
         qu = back(qt.p, (size_t)heads * head_dim * (q_pair ? 2 : 4));
         q_lo = back(qtl.p, (size_t)heads * head_dim * 2);
         ku = kt.p;
@@ -741,13 +754,16 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.n_tasks = (int64_t)a.n_sets * (row1 - row0) * kv_heads;
     a.qk_bound = tile8 ? (const float *)bound.p : nullptr;
     if (tile || suffix) {
-        // the tile kernel's value product takes the values as fp16 (scaled into range)
-        const size_t nv = (size_t)N * kv_heads * head_dim;
-        RIS_CUDA(v16.alloc(nv * 2, s));
-        RIS_CUDA(vmax.alloc(sizeof(float), s));
-        RIS_CUDA(launch_values_f16(v, (int64_t)nv, v16.p, (float *)vmax.p, s));
+        // the tile kernel's value product takes the values as fp16 (scaled into range), written
+        // above with the fp8 operands or here
+        if (!tile8) {
+            const size_t nv = (size_t)N * kv_heads * head_dim;
+            RIS_CUDA(v16.alloc(nv * 2, s));
+            RIS_CUDA(vmax.alloc(sizeof(float), s));
+            RIS_CUDA(launch_values_f16(v, (int64_t)nv, v16.p, (float *)vmax.p, s));
+        }
         a.v16 = v16.p;
-        a.v_absmax = (const float *)vmax.p;
+        a.v_absmax = tile8 ? (const float *)bound.p + 2 : (const float *)vmax.p;
     }
     if (suffix) {
         RIS_CUDA(po.alloc((size_t)N * heads * head_dim * sizeof(float), s));

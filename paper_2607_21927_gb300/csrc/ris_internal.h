@@ -174,16 +174,25 @@ unsigned int read_decode_error();
 // dtype_in / dtype_out are ris_dtype values.
 cudaError_t launch_rope(const RopeArgs &a, int dtype_in, int dtype_out, cudaStream_t s);
 
-// Bounds of the rotated values of x [N][H][D] (bf16): mscale times the largest pair norm
-// |(x_c, x_{c+D/2})|, with a margin for the fp32 rotation, atomically maxed into *bound (a
-// float, >= 0 bit patterns; zero it first).
-cudaError_t launch_rotation_bound(const void *x, int64_t N, int H, int D, float mscale, float *bound,
-                                  cudaStream_t s);
-// RoPE (bf16 in) for the tile kernel's fp8-correction scores: role 0 queries, 1 keys; x_out gets
-// fp16 hi parts and x_out_lo, per (token, head), D bytes of e4m3 hi-part corrections then D bytes
-// of e4m3 lo-part corrections (see fp8_score_scales), or, when the bounds at qk_bound rule the
-// scheme out, the bf16 hi / lo pair of launch_rope.
-cudaError_t launch_rope_tile8(const RopeArgs &a, int role, const float *qk_bound, cudaStream_t s);
+// The pre-passes of a layer call whose scores take the fp8-correction operands (see
+// fp8_score_scales in attn_common.cuh), bf16 inputs, head dim a multiple of 16, every pointer
+// 16-byte aligned. Two launches: bounds of |q~|, |k~| (and max |v| when v16 is set) into
+// bounds[0..2] (zeroed by this call), then RoPE of q (positions q_first .. q_first + q_rows - 1)
+// and k (positions 0 .. N-1) into q_hi / q_lo and k_hi / k_lo: fp16 hi parts, and per (token,
+// head) D bytes of e4m3 corrections of the hi part then D bytes of e4m3 corrections of the lo
+// part; or, when the bounds rule the scheme out, the bf16 hi / lo pair. With v16 set, the values
+// as fp16 scaled by 2^-E, E = v_scale_exp(bounds[2]), as launch_values_f16 writes them.
+struct Fp8PrepArgs {
+    const void *q, *k, *v;  // bf16 [q_rows][Hq][D], [N][Hkv][D], [N][Hkv][D]
+    void *q_hi, *q_lo, *k_hi, *k_lo;
+    void *v16;              // or null
+    float *bounds;          // [3]
+    int64_t N, q_rows, q_first;
+    int32_t Hq, Hkv, D;
+    double f[kMaxHeadDimHalf];  // rotation frequencies (fp64)
+    float mscale;
+};
+cudaError_t launch_fp8_prep(const Fp8PrepArgs &a, cudaStream_t s);
 
 // bf16 values v[n] (n a multiple of 8, 16-byte aligned) -> *vmax = max |v| (vmax zeroed by
 // this call) and v16[i] = fp16(v[i] / 2^E), E = v_scale_exp(max |v|): the fp16 operand of the
