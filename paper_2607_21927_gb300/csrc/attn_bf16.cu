@@ -583,15 +583,19 @@ cudaError_t launch_f(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t 
     constexpr bool KSPLIT = QSPLIT;
     const dim3 block(kAttnWarps * 32);
     if (!dense && a.n_sets > 1) {  // per-seed sets: one warp per (row, KV head) walks them all
-        AttnArgs b = a;
-        b.n_tasks = (a.row1 - a.row0) * a.Hkv;
-        const unsigned grid = (unsigned)((b.n_tasks + kAttnWarps - 1) / kAttnWarps);
-        if (col_bytes == 2)
-            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, true, F8><<<grid, block, 0, s>>>(b);
-        else
-            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, true, F8><<<grid, block, 0, s>>>(b);
-        note_launch();
-        return cudaGetLastError();
+        if constexpr (F8) {
+            return cudaErrorInvalidValue;  // per-seed sets take the bf16 pairs (the caller's choice)
+        } else {
+            AttnArgs b = a;
+            b.n_tasks = (a.row1 - a.row0) * a.Hkv;
+            const unsigned grid = (unsigned)((b.n_tasks + kAttnWarps - 1) / kAttnWarps);
+            if (col_bytes == 2)
+                k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, true, false><<<grid, block, 0, s>>>(b);
+            else
+                k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, true, false><<<grid, block, 0, s>>>(b);
+            note_launch();
+            return cudaGetLastError();
+        }
     }
     const unsigned grid = (unsigned)((a.n_tasks + kAttnWarps - 1) / kAttnWarps);
     if (dense)
