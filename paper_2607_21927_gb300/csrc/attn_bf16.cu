@@ -179,7 +179,7 @@ constexpr float kLazyLog2 = 8.f;  // rescale O only when the row maximum grows b
 // runs and its first K/V rows during the current set's last group, so the load pipeline
 // never drains between sets; a.n_tasks counts (row, KV head) pairs.
 // E8 (head dim 128, rotated bf16 inputs, 32-byte loads): the operands of the tile kernel's
-// fp8-correction scheme, written by launch_rope_tile8 (see fp8_score_scales): keys as fp16 hi
+// fp8-correction scheme, written by launch_fp8_prep (see fp8_score_scales): keys as fp16 hi
 // parts (a.k) and, in each (token, head)'s 2D-byte record of a.k_lo, e4m3(k_h 2^-eb) at bytes
 // [0, D) and e4m3(k_l 2^(12+ea)) at [D, 2D); queries likewise (a.q, a.q_lo; 2^-ea and
 // 2^(12+eb)). The gather fetches only the fp16 hi part and the e4m3 lo part of a key row (384
@@ -560,7 +560,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
     }  // sets
 }
 
-// F8: the queries and keys came from launch_rope_tile8; which of its two schemes it wrote
+// F8: the queries and keys came from launch_fp8_prep; which of its two schemes it wrote
 // follows from the bounds at a.qk_bound, read here on the device as it did.
 template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut, bool SEEDS, bool F8>
 __global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
@@ -611,7 +611,7 @@ cudaError_t launch_f(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t 
 template <int D, bool QSPLIT, bool WIDE, typename TOut>
 cudaError_t launch_w(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t s)
 {
-    // operands in launch_rope_tile8's form (a.qk_bound set) are read only by the F8 kernel, which
+    // operands in launch_fp8_prep's form (a.qk_bound set) are read only by the F8 kernel, which
     // needs head dim 128 and 32-byte aligned inputs (the caller checks both)
     if constexpr (D == 128 && QSPLIT && WIDE) {
         if (a.qk_bound != nullptr) return launch_f<D, QSPLIT, WIDE, TOut, true>(a, col_bytes, dense, s);

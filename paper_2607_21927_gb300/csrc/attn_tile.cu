@@ -525,7 +525,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // against bf16 values)
             constexpr uint32_t ID_O = kP16 ? idesc_f16(BM, DT, true) : idesc_bf16(BM, DT, true);
             // fp8-correction scores (rotated q / k at head dim 128, operands written by
-            // launch_rope_tile8 when the bounds allow): the same bytes in the same places as the
+            // launch_fp8_prep when the bounds allow): the same bytes in the same places as the
             // bf16 pair, read as fp16 hi parts (query columns 0-63, key bytes 0-255 of a row) and
             // e4m3 corrections (query columns 64-95 / 96-127, key boxes at KV_ARR / KV_ARR + KV_BLK)
             int ea = 0, eb = 0;

@@ -103,9 +103,9 @@ struct AttnArgs {
     int64_t n_tasks;       // n_sets * (row1 - row0) * Hkv
     const void *v16;       // tile kernel: the values as fp16, scaled by 2^-E (launch_values_f16)
     const float *v_absmax; // tile kernel: max |v| over the values (device), from which E follows
-    const float *qk_bound; // head dim 128 with rotated q / k in launch_rope_tile8's form: bounds of |q~| and |k~|
+    const float *qk_bound; // head dim 128 with rotated q / k in launch_fp8_prep's form: bounds of |q~| and |k~|
                            // (device, two floats) when the RoPE kernels wrote the fp8-correction
-                           // operands (launch_rope_tile8), else null
+                           // operands (launch_fp8_prep), else null
     int64_t wait_limit;    // tile kernel: cycles a device-side wait may take (0: about 2^31)
     int32_t debug_no_loads;  // tile kernel, tests only: the loader issues no copies, so the
                              // first wait on them gives up (ris_debug_tile_stall)
