@@ -27,9 +27,12 @@
 //
 // Precision. With activation outlier channels (|v| up to ~30) a max-abs error of 1e-2 needs
 // ~12+ significant bits in the scores and in P, more than bf16 (8) or fp16 (11) carry. So:
-//   - rotated queries arrive in fp32 and are split into bf16 hi + lo in registers;
+//   - rotated queries arrive in fp32 and are split into bf16 hi + lo in registers, or as a
+//     bf16 hi + lo pair;
 //   - rotated keys arrive as a bf16 hi + lo pair (written by the RoPE kernel);
 //   - S^T = K_hi Q_hi + K_hi Q_lo + K_lo Q_hi (the lo*lo term is below 2^-16);
+//   - or, at head dim 128 with rotated bf16 inputs, fp16 hi parts with e4m3 lo parts (E8
+//     below);
 //   - P is split into bf16 hi + lo and O^T += V^T P_hi + V^T P_lo.
 // V is an exact bf16 input. Unrotated bf16 q/k are exact and take one product each.
 #include <cuda_bf16.h>
@@ -236,8 +239,9 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
             const unsigned char *rec = reinterpret_cast<const unsigned char *>(a.q_lo) + 2 * qrow;
             const uint4 x0 = hv ? *reinterpret_cast<const uint4 *>(rec + 32 * q) : make_uint4(0u, 0u, 0u, 0u);
             const uint4 x1 = hv ? *reinterpret_cast<const uint4 *>(rec + 32 * q + 16) : make_uint4(0u, 0u, 0u, 0u);
-            q8[0] = x0.x; q8[1] = x0.y; q8[2] = x0.z; q8[3] = x0.w;
-            q8[4] = x1.x; q8[5] = x1.y; q8[6] = x1.z; q8[7] = x1.w;
+            const uint32_t w[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) q8[e] = w[e];
         }
         const float ql_scale = E8 ? pow2i(-12 - eb) : 1.f;
 #pragma unroll

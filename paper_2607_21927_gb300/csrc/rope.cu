@@ -5,7 +5,10 @@
 // token: the angle p * f_c is formed in fp64 and reduced to [-pi, pi] in fp64 (an fp32
 // product loses ~4e-3 rad at p = 65535), then sin/cos of the reduced angle come from the
 // CUDA math library in fp32 and the rotation runs in fp32. The work is HBM-bound: one read
-// and one write of the tensor.
+// and one write of the tensor. For the fp16 + e4m3 score operands (head dim 128, bf16 inputs)
+// two launches serve a whole layer call: k_fp8_bounds bounds q, k (and v) in one pass, then
+// k_fp8_rotate rotates q and k (one thread per token and 8 frequencies, 16-byte accesses) into
+// those operands and writes the fp16 values.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_fp8.h>
