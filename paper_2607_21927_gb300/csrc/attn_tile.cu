@@ -6,44 +6,51 @@
 // percent, and the dense mode) a dense 128 x 128 score tile with the mask applied as -inf
 // beats gathering rows pair by pair. One CTA owns one (128-query tile, query head, set):
 //
-//   warp 8 (TMA)   streams 128-key tiles of K~ hi + K~ lo (64 KB) and of the values (fp16,
-//                  32 KB) in 128-byte swizzled boxes into two two-stage shared-memory rings:
-//                  a key stage is refilled as soon as its score products are done, a value
-//                  stage once its value product is, so the next keys load while P and the
-//                  value product of the current tile are still pending;
-//   warp 9 (MMA)   one elected lane issues tcgen05.mma: S = Q_hi K_hi^T + Q_lo K_hi^T +
-//                  Q_hi K_lo^T (A = the query tile, kept in TMEM) into a double-buffered TMEM
-//                  score tile, and O += P V (A = P as fp16, written into TMEM over the consumed
-//                  scores) into the TMEM output tile, committing each step to an mbarrier;
-//                  TMEM holds S/P twice (2 x 128 columns), O (128) and Q hi / lo (2 x 64), all
-//                  512 columns;
+//   warp 8 (TMA)   streams 128-key tiles of the keys (64 KB: hi parts and corrections) and of
+//                  the values (fp16, 32 KB) in 128-byte swizzled boxes into two two-stage
+//                  shared-memory rings: a key stage is refilled as soon as its score products
+//                  are done, a value stage once its value product is; it also waits for each
+//                  tile's values to land and then arrives on that tile's P_FULL barrier, so
+//                  that the MMA warp waits once per value product;
+//   warp 9 (MMA)   one elected lane issues tcgen05.mma: the score tile S (A = the query tile,
+//                  kept in TMEM) into a double-buffered TMEM score tile, and O += P V (A = P
+//                  as fp16, written into TMEM over the consumed scores) into the TMEM output
+//                  tile, committing each step to an mbarrier; TMEM holds S/P twice (2 x 128
+//                  columns), O (128) and the query operands (128), all 512 columns;
 //   warps 0-7      two threads per query row (score and output columns 0-63 / 64-127): write
-//                  the row's query half into TMEM, then per tile tcgen05.ld the scores, apply
-//                  the bitmap (or the causal cut), exchange the partial row max with the
-//                  partner thread, fp32 online softmax with lazy rescaling of O in TMEM (only
-//                  when the row max grows by more than 2^8), write P into TMEM, and at the end
-//                  normalise O (and undo the values' power-of-two scale) and store the row.
+//                  the row's query part into TMEM, then per tile tcgen05.ld the scores, apply
+//                  the bitmap (words fetched three tiles ahead) or the causal cut, exchange the
+//                  partial row max with the partner thread, fp32 online softmax with lazy
+//                  rescaling of O in TMEM (only when the row max grows by more than 2^8),
+//                  write P into TMEM, and at the end normalise O (and undo the values'
+//                  power-of-two scale) and store the row.
 //
 // Precision. With activation outlier channels the scores reach tens of units while the
 // output moves by p (v_j - o) per unit of score error, so the scores need about 17
-// significant bits: the three products keep q and k to about 16 bits each (bf16 hi + lo).
-// One product of fp16 keys moves outputs by up to 0.1; fp16 main products with fp8 (e4m3 /
-// e5m2) correction products by up to 4e-3 to 7e-3 (CPU emulation on inputs with outlier
-// channels), so neither is taken. P enters the value product as one fp16 (11 significant
-// bits; max-abs 6.5e-3 in the same emulation against 1.7e-3 for a bf16 hi + lo pair), and the
-// row sum adds P as rounded, so that each weight's rounding moves the output by at most 2^-11
-// of that weight times |v_j - o|. The values are exact in fp16 after a power-of-two scale
-// (none unless some |v| reaches 2^14), undone in the epilogue.
+// significant bits. At head dim 128 with rotated inputs (the operands written by
+// launch_fp8_prep) S = q_h k_h + 2^-12 (e4m3(q_h) e4m3(k_l) + e4m3(q_l) e4m3(k_h)) with fp16
+// hi parts and power-of-two scales taken from bounds of |q~| and |k~| (fp8_score_scales): the
+// two e4m3 products (kind::f8f6f4, twice the rate) go first and the fp16 product folds them in
+// with scale-input-d; max-abs about 7e-3 in CPU emulation. Where the bounds rule that out, at
+// head dim 64, and for inputs not rotated here, S = Q_hi K_hi^T + Q_lo K_hi^T + Q_hi K_lo^T
+// with bf16 hi + lo pairs. One fp16 key product alone moves outputs by up to 0.1. P enters the
+// value product as one fp16 (11 significant bits; max-abs 6.5e-3 in the same emulation
+// against 1.7e-3 for a bf16 hi + lo pair), and the row sum adds P as rounded, so that each
+// weight's rounding moves the output by at most 2^-11 of that weight times |v_j - o|. The
+// values are exact in fp16 after a power-of-two scale (none unless some |v| reaches 2^14),
+// undone in the epilogue.
 //
-// Measured: the kernel issues its products at the measured sustained bf16 rate (about 95
-// cycles per 128 x 128 x 16 product at the power-capped clock): 32 products per tile pair
-// take ~3,090 cycles (C5's Stochastic layer at 64k: 16.4 ms per launch; with a bf16 P pair
-// and 40 products, 19.6 ms). Dropping score products (timing experiments, wrong results)
-// runs into the softmax's own per-tile latency (~3,000 cycles), so fewer products would need
-// a shorter softmax chain as well. Four threads per row (16 softmax warps) measured the same
-// as two. With one ring of combined K/V stages, released only after the value product, the
-// next tile's keys started loading only then and the tensor pipe waited for them; 128-key
-// tiles with the query in TMEM beat 64-key tiles with the query in shared memory.
+// Measured: a tile pair takes 24 slots of 16-bit product time (8 fp16 score products, 2 x 4
+// e4m3 corrections at twice the rate, 8 fp16 value products); C5's Stochastic layer at 64k
+// runs in 13.3-13.5 ms per launch (16.4 ms with three bf16 score products, 19.6 with a bf16 P
+// pair as well). What holds the pipe below its rate is the MMA warp's own time between issues
+// (each mbarrier wait costs its thread about 100 cycles even on a completed phase, and the
+// issue blocks until the pipe takes each product) and, with a bitmap, the softmax's wait for
+// the bitmap words: so the MMA warp waits on one barrier before a tile's score products (the
+// keys; the score buffer's reuse is implied by the P_FULL it waited on two tiles before) and
+// one before its value product, and the bitmap words come three tiles ahead. Four threads per
+// row (16 softmax warps) measured the same as two. 128-key tiles with the query in TMEM beat
+// 64-key tiles with the query in shared memory.
 //
 // The suffix pass of the dense-suffix split (SUFFIX) runs the same pipeline over the key
 // tiles of each row's dense suffix only (its Structural block and / or local window: every key
@@ -104,8 +111,7 @@ constexpr int SMEM_BYTES = OFF_K + kStages * (Smem<128>::K_STAGE + Smem<128>::V_
 // B_X: per group of kRowThreads softmax warps sharing rows (one per column quarter) and tile
 // parity, the exchange of their partial row maxima (and at the end their partial sums).
 enum Bar {
-    B_Q = 0, B_K_FULL = 1, B_V_FULL = 3, B_S_FULL = 5, B_S_EMPTY = 7, B_P_FULL = 9, B_PV_DONE = 11, B_X = 13,
-    B_END = 21, NBAR = 22
+    B_Q = 0, B_K_FULL = 1, B_V_FULL = 3, B_S_FULL = 5, B_P_FULL = 7, B_PV_DONE = 9, B_X = 11, B_END = 19, NBAR = 20
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -455,8 +461,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < NBAR; ++i) {
             uint32_t cnt = 1;
-            if (i == B_Q || i == B_S_EMPTY || i == B_S_EMPTY + 1 || i == B_P_FULL || i == B_P_FULL + 1)
-                cnt = kSoftmaxThreads;
+            if (i == B_Q) cnt = kSoftmaxThreads;
+            if (i == B_P_FULL || i == B_P_FULL + 1) cnt = kSoftmaxThreads + 1;  // + the loader's relay
             if (i >= B_X && i < B_END) cnt = 32 * kRowThreads;
             mbar_init(smem_u32(&bars[i]), cnt);
         }
@@ -487,8 +493,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             // stage is free exactly when the barrier that announces those products completes
             // (S_FULL, PV_DONE): the loader waits on them instead of on barriers of its own,
             // which saves the tensor pipe two commits per tile.
+            // The loader also waits for each tile's values to land and then arrives on that tile's
+            // P_FULL (which counts the softmax threads and this one), so that the MMA warp waits
+            // once before a value product instead of twice: each wait costs its issuing thread
+            // about 100 cycles even on a completed phase, and the tensor pipe idles meanwhile.
             static_assert(kStages == 2, "ring stages share the parity of the score buffers");
-            int nk = 0, nv = 0;  // tiles whose keys / values were requested
+            int nk = 0, nv = 0, nr = 0;  // tiles whose keys / values were requested; values relayed
+            auto relay = [&](int jv) -> bool {
+                if (!mbar_wait(smem_u32(&bars[B_V_FULL + jv % kStages]), (jv / kStages) & 1, wl)) return false;
+                mbar_arrive(smem_u32(&bars[B_P_FULL + (jv & 1)]));
+                nr = jv + 1;
+                return true;
+            };
             for (int j = 0; j < n_kt && ok; ++j) {
                 const int st = j % kStages;
                 const uint32_t par = ((j / kStages) - 1) & 1;
@@ -502,6 +518,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (SPLIT) tma_load_3d(dk + KV_ARR + blk * KV_BLK, &maps.kl, 64 * blk, g, (kt0 + j) * BN, bk);
                 }
                 nk = j + 1;
+                if (j >= 1) ok = relay(j - 1);
+                if (!ok) break;
                 if (j >= kStages) ok = mbar_wait(smem_u32(&bars[B_PV_DONE + st]), par, wl);
                 if (!ok) break;
                 const uint32_t bv = smem_u32(&bars[B_V_FULL + st]);
@@ -510,6 +528,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int blk = 0; blk < NB; ++blk) tma_load_3d(dv + blk * KV_BLK, &maps.v, 64 * blk, g, (kt0 + j) * BN, bv);
                 nv = j + 1;
             }
+            if (ok && nv == n_kt && nr < nv) ok = relay(nv - 1);
             // let the copies requested last into each stage land before the CTA can leave
             // (earlier ones were consumed before their stage was refilled)
             for (int j = nk - kStages; j < nk; ++j)
@@ -592,15 +611,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_commit(smem_u32(&bars[B_PV_DONE + (j & 1)]));
             };
             for (int j = 0; j < n_kt && ok; ++j) {
-                const int st = j & 1;
+                // the score buffer j & 1 held P of tile j - 2, and P_FULL of that tile (waited for
+                // before its value product) came after the softmax threads had read its scores:
+                // so only the keys are waited for here
                 ok = mbar_wait(smem_u32(&bars[B_K_FULL + j % kStages]), (j / kStages) & 1, wl);
-                if (ok && j >= 2) ok = mbar_wait(smem_u32(&bars[B_S_EMPTY + st]), ((j >> 1) - 1) & 1, wl);
                 if (!ok) break;
                 tc_fence_after();
                 issue_s(j);
                 if (j >= 1) {
+                    // P of tile j - 1 written and its values landed (relayed by the loader)
                     ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((j - 1) & 1)]), ((j - 1) >> 1) & 1, wl);
-                    if (ok) ok = mbar_wait(smem_u32(&bars[B_V_FULL + (j - 1) % kStages]), ((j - 1) / kStages) & 1, wl);
                     if (!ok) break;
                     tc_fence_after();
                     issue_o(j - 1);
@@ -608,7 +628,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (ok) {
                 ok = mbar_wait(smem_u32(&bars[B_P_FULL + ((n_kt - 1) & 1)]), ((n_kt - 1) >> 1) & 1, wl);
-                if (ok) ok = mbar_wait(smem_u32(&bars[B_V_FULL + (n_kt - 1) % kStages]), ((n_kt - 1) / kStages) & 1, wl);
                 if (ok) {
                     tc_fence_after();
                     issue_o(n_kt - 1);
@@ -690,14 +709,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             mbar_arrive(smem_u32(&bars[B_Q]));
         }
-        uint32_t cw[SC / 32];
+        // bitmap words fetched three tiles ahead (one tile ahead left part of a DRAM miss exposed:
+        // two ahead gained 3.5% at 64k, three 1-2% more)
+        uint32_t cw[SC / 32], nw[SC / 32], n2w[SC / 32];
 #pragma unroll
-        for (int e = 0; e < SC / 32; ++e) cw[e] = mask_word(0, e);
+        for (int e = 0; e < SC / 32; ++e) {
+            cw[e] = mask_word(0, e);
+            nw[e] = (1 < n_kt) ? mask_word(1, e) : 0u;
+            n2w[e] = (2 < n_kt) ? mask_word(2, e) : 0u;
+        }
         for (int j = 0; j < n_kt; ++j) {
             const int st = j & 1;
-            uint32_t nw[SC / 32];
+            uint32_t nnw[SC / 32];
 #pragma unroll
-            for (int e = 0; e < SC / 32; ++e) nw[e] = (j + 1 < n_kt) ? mask_word(j + 1, e) : 0u;
+            for (int e = 0; e < SC / 32; ++e) nnw[e] = (j + 3 < n_kt) ? mask_word(j + 3, e) : 0u;
             ok = __all_sync(0xFFFFFFFFu, mbar_wait(smem_u32(&bars[B_S_FULL + st]), (j >> 1) & 1, wl));
             if (!ok) break;
             tc_fence_after();
@@ -705,7 +730,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t sb = ((j & 1) ? t_s1 : t_s0) + lane_off + SC * cq;
             tmem_ld_cols<SC>(sb, sv);
             tc_fence_before();
-            mbar_arrive(smem_u32(&bars[B_S_EMPTY + st]));
 
             // mask, partial row max as a tree (the scale is positive: it is applied to the max
             // and folded into the exponent of P), then the full row max from the other threads
@@ -714,6 +738,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int c = 0; c < 32; ++c) sv[32 * e + c] = ((cw[e] >> c) & 1u) ? sv[32 * e + c] : -INFINITY;
                 cw[e] = nw[e];
+                nw[e] = n2w[e];
+                n2w[e] = nnw[e];
             }
             float mx9[9];
 #pragma unroll
