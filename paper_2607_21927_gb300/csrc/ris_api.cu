@@ -194,13 +194,14 @@ const char *forced_design()
 
 // Union density at and above which masked dense tiles beat gathering pair by pair (bf16,
 // head dim 128): a tile costs the dense causal products (an fp16 score product, two e4m3 score
-// corrections and one value product) whatever the mask, a gathered pair 1.5 KB of K/V rows.
-// Measured crossover on Qwen2-shaped layers (head dim 128): 6.3% of the causal pairs at
-// N = 32768 and 6.1% at N = 65536 (tiles 3.69 / 14.4 ms per launch, the gather 3.46 / 13.8 ms
-// at 5.9%); on TinyLlama-shaped layers (head dim 64, 32 query and 4 KV heads, N = 16384, three
-// bf16 score products) 13.6%, where the tiles are half the products but the same softmax work.
-constexpr double kTileDensity = 0.062;
-constexpr double kTileDensity64 = 0.136;
+// corrections and one value product) whatever the mask, a gathered pair 1.25 KB of K/V rows.
+// Measured crossover on Qwen2-shaped layers (head dim 128): 5.8% of the causal pairs at
+// N = 32768 and N = 65536 (tiles 3.34 / 13.2-13.5 ms per launch, the gather on the fp8
+// operands 3.39 / 13.5 ms at 5.9%); on TinyLlama-shaped layers (head dim 64, 32 query and 4 KV
+// heads, N = 16384, three bf16 score products) 11.1% (tiles 1.94 ms, the gather 1.69 / 1.99 ms
+// at 9.6% / 11.4%), where the tiles are half the products but the same softmax work.
+constexpr double kTileDensity = 0.058;
+constexpr double kTileDensity64 = 0.111;
 
 // Shortest dense span (Structural block or local window) for which the split pays: two
 // 128-key tiles.
