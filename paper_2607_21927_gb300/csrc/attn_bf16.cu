@@ -35,6 +35,11 @@
 //     below);
 //   - P is split into bf16 hi + lo and O^T += V^T P_hi + V^T P_lo.
 // V is an exact bf16 input. Unrotated bf16 q/k are exact and take one product each.
+//
+// Residency. The gather is bound by the gathered rows it keeps in flight, hence by how many
+// warps fit on an SM. In the fp8 form (one set per task) each thread parks its query fragments
+// and output accumulators in its own lane of tensor memory (128 columns per CTA) and reloads
+// them around the products that use them: 168 registers, three CTAs per SM instead of two.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_fp8.h>
@@ -87,6 +92,70 @@ __device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two, float s)
     const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&hr));
     const __half2 h = __floats2half2_rn(f.x * s, f.y * s);
     return *reinterpret_cast<const uint32_t *>(&h);
+}
+
+// Per-thread private storage in tensor memory: thread l of warp w owns TMEM lane 32 (w % 4) + l,
+// and a 32x32b access moves N consecutive 32-bit columns of that lane (warp-collective).
+template <int N>
+__device__ __forceinline__ void tm_st(uint32_t taddr, const uint32_t *v);
+template <>
+__device__ __forceinline__ void tm_st<8>(uint32_t taddr, const uint32_t *v)
+{
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(v[0]),
+                 "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+                 : "memory");
+}
+template <>
+__device__ __forceinline__ void tm_st<16>(uint32_t taddr, const uint32_t *v)
+{
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+                 ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+                 "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+                 : "memory");
+}
+template <int N>
+__device__ __forceinline__ void tm_ld(uint32_t taddr, uint32_t *v);
+template <>
+__device__ __forceinline__ void tm_ld<8>(uint32_t taddr, uint32_t *v)
+{
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n\t"
+                 "tcgen05.wait::ld.sync.aligned;"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7])
+                 : "r"(taddr)
+                 : "memory");
+}
+template <>
+__device__ __forceinline__ void tm_ld<16>(uint32_t taddr, uint32_t *v)
+{
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+                 "tcgen05.wait::ld.sync.aligned;"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+                   "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+                 : "r"(taddr)
+                 : "memory");
+}
+__device__ __forceinline__ void tm_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// the output accumulators o[8][4] <-> 32 columns
+__device__ __forceinline__ void tm_st_o(uint32_t taddr, float (&o)[8][4])
+{
+    uint32_t w[16];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) w[i] = __float_as_uint(o[4 * h + i / 4][i % 4]);
+        tm_st<16>(taddr + 16 * h, w);
+    }
+    tm_wait_st();
+}
+__device__ __forceinline__ void tm_ld_o(uint32_t taddr, float (&o)[8][4])
+{
+    uint32_t w[16];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        tm_ld<16>(taddr + 16 * h, w);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) o[4 * h + i / 4][i % 4] = __uint_as_float(w[i]);
+    }
 }
 
 __device__ __forceinline__ uint32_t transpose8x8(uint32_t x)
@@ -193,10 +262,12 @@ constexpr float kLazyLog2 = 8.f;  // rescale O only when the row maximum grows b
 // terms is within about 2^-15 of |q||k| per channel, as in the tile kernel's scheme. (Widening
 // the e4m3 lo part to fp16 in registers for a third fp16 product instead measured slower than
 // the bf16 pairs: the conversions cost more than the bytes saved.)
-template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut, bool SEEDS, bool E8>
-__device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
+template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut, bool SEEDS, bool E8,
+          bool TQ>
+__device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t tbase)
 {
     static_assert(!E8 || (D == 128 && QSPLIT && KSPLIT && WIDE), "the fp8 operands: head dim 128, 32-byte loads");
+    static_assert(!TQ || (E8 && !SEEDS), "query fragments and accumulators in TMEM: the fp8 form, one set");
     constexpr int KSTEPS = D / 16;  // k-steps of the score product
     constexpr int KW = D / 8;       // 32-bit words of one K row per lane (D/4 elements)
     constexpr int VW = D / 16;      // 32-bit words of one V row per lane (D/8 elements)
@@ -287,6 +358,25 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
         }
     }
 
+    // TQ: this thread's TMEM lane; the query fragments in columns 0-39 (k-step ks: hi, hi, lo,
+    // lo at 4 ks .. 4 ks + 3; the e4m3 words at 32-39), the output accumulators in 64-95
+    const uint32_t tl = tbase + ((uint32_t)(32 * ((threadIdx.x >> 5) & 3)) << 16);
+    if constexpr (TQ) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            uint32_t w[16];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                w[4 * k] = qh[4 * h + k][0];
+                w[4 * k + 1] = qh[4 * h + k][1];
+                w[4 * k + 2] = ql[4 * h + k][0];
+                w[4 * k + 3] = ql[4 * h + k][1];
+            }
+            tm_st<16>(tl + 16 * h, w);
+        }
+        tm_st<8>(tl + 32, q8);
+        tm_wait_st();
+    }
     const size_t row_bytes = (size_t)a.Hkv * D * sizeof(__nv_bfloat16);
     const size_t head_off = (size_t)t.g * D * sizeof(__nv_bfloat16);
     const char *kb = reinterpret_cast<const char *>(a.k) + head_off + 2 * kelem<D, WIDE>(0, q);
@@ -328,6 +418,8 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
             }
         }
     }
+
+    if constexpr (TQ) tm_st_o(tl + 64, o);
 
     // ---- key indices, prefetched 64 keys (4 groups) ahead: lane holds positions
     //      64c + lane and 64c + 32 + lane of chunk c; slots past the row read the row itself
@@ -415,7 +507,26 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
         for (int c = 0; c < 2; ++c)
 #pragma unroll
             for (int e = 0; e < 4; ++e) sa[c][e] = sb[c][e] = sl[c][e] = 0.f;
-        if constexpr (E8) {
+        if constexpr (TQ) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                uint32_t w[16];
+                tm_ld<16>(tl + 16 * h, w);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int ks = 4 * h + k;
+                    mma16816_f16(sa[ks & 1], k0[2 * ks], k1[2 * ks], k0[2 * ks + 1], k1[2 * ks + 1], w[4 * k], w[4 * k + 1]);
+                    mma16816_f16(sb[ks & 1], k0[2 * ks], k1[2 * ks], k0[2 * ks + 1], k1[2 * ks + 1], w[4 * k + 2],
+                                 w[4 * k + 3]);
+                }
+            }
+            uint32_t w8[8];
+            tm_ld<8>(tl + 32, w8);
+#pragma unroll
+            for (int ks = 0; ks < D / 32; ++ks)
+                mma16832_e4m3(sl[ks & 1], kl0[2 * ks], kl1[2 * ks], kl0[2 * ks + 1], kl1[2 * ks + 1], w8[2 * ks],
+                              w8[2 * ks + 1]);
+        } else if constexpr (E8) {
 #pragma unroll
             for (int ks = 0; ks < KSTEPS; ++ks) {
                 mma16816_f16(sa[ks & 1], k0[2 * ks], k1[2 * ks], k0[2 * ks + 1], k1[2 * ks + 1], qh[ks][0], qh[ks][1]);
@@ -468,6 +579,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
             m1 = mn1;
             l0 *= al0;
             l1 *= al1;
+            if constexpr (TQ) tm_ld_o(tl + 64, o);
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt) {
                 o[mt][0] *= al0;
@@ -475,6 +587,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
                 o[mt][2] *= al0;
                 o[mt][3] *= al1;
             }
+            if constexpr (TQ) tm_st_o(tl + 64, o);
         }
         const float mu0 = (m0 == -INFINITY) ? 0.f : m0, mu1 = (m1 == -INFINITY) ? 0.f : m1;
         const float p0 = exp2f(s0 - mu0), p1 = exp2f(s1 - mu1);
@@ -490,6 +603,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
         const uint32_t pl1 = transpose8x8(pack_bf16(p2 - h2, p3 - h3));
 
         // ---- O^T += V^T P^T
+        if constexpr (TQ) tm_ld_o(tl + 64, o);
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
             const uint32_t a0 = __byte_perm(v0[mt], v1[mt], 0x5410);
@@ -499,6 +613,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
             mma16816(o[mt], a0, a1, a2, a3, pb0, pb1);
             mma16816(o[mt], a0, a1, a2, a3, pl0, pl1);
         }
+        if constexpr (TQ) tm_st_o(tl + 64, o);
         if (more)
             issue_v(n0, n1, gs1);
         else if (cross)
@@ -511,6 +626,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
     }
 
     // ---- epilogue: full row sums, normalise, undo the head-dim permutation
+    if constexpr (TQ) tm_ld_o(tl + 64, o);
 #pragma unroll
     for (int off = 4; off < 32; off <<= 1) {
         l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, off);
@@ -566,17 +682,39 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb)
 
 // F8: the queries and keys came from launch_fp8_prep; which of its two schemes it wrote
 // follows from the bounds at a.qk_bound, read here on the device as it did.
+// F8 (one set per task): the query fragments and output accumulators live in tensor memory
+// (each thread's own TMEM lane, 128 columns per CTA), which leaves room for three CTAs of four
+// warps per SM instead of two, and so more gathered rows in flight.
+constexpr int kGatherTmemCols = 128;
 template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE, typename TOut, bool SEEDS, bool F8>
-__global__ void __launch_bounds__(kAttnWarps * 32, RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
+__global__ void __launch_bounds__(kAttnWarps * 32, F8 ? 3 : RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
 {
     if constexpr (F8) {
+        static_assert(!SEEDS, "per-seed sets take the bf16 pairs");
+        __shared__ uint32_t tbase_sh;
+        const int warp = threadIdx.x >> 5;
+        if (warp == 0) {
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                         ::"r"((uint32_t)__cvta_generic_to_shared(&tbase_sh)), "r"(kGatherTmemCols) : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t tb = tbase_sh;
         int ea = 0, eb = 0;
         if (fp8_score_scales(a.qk_bound[0], a.qk_bound[1], ea, eb))
-            gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, true>(a, eb);
+            gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, true, true>(a, eb, tb);
         else
-            gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, false>(a, 0);
+            gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, false, false>(a, 0, 0u);
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        if (warp == 0)
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tb), "r"(kGatherTmemCols)
+                         : "memory");
     } else {
-        gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, false>(a, 0);
+        gather_task<D, QSPLIT, KSPLIT, WIDE, TIdx, DENSE, TOut, SEEDS, false, false>(a, 0, 0u);
     }
 }
 

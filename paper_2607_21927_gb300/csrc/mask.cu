@@ -32,11 +32,9 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1
 {
 #pragma unroll
     for (int r = 0; r < 10; ++r) {
-        const uint32_t lo0 = 0xD2511F53u * c.x;
-        const uint32_t hi0 = __umulhi(0xD2511F53u, c.x);
-        const uint32_t lo1 = 0xCD9E8D57u * c.z;
-        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z);
-        c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+        const uint64_t p0 = (uint64_t)0xD2511F53u * c.x;
+        const uint64_t p1 = (uint64_t)0xCD9E8D57u * c.z;
+        c = make_uint4((uint32_t)(p1 >> 32) ^ c.y ^ k0, (uint32_t)p1, (uint32_t)(p0 >> 32) ^ c.w ^ k1, (uint32_t)p0);
         k0 += 0x9E3779B9u;
         k1 += 0xBB67AE85u;
     }
@@ -88,6 +86,8 @@ __global__ void __launch_bounds__(kBitsThreads) k_mask_bits(const MaskBitsArgs a
         bits |= range_bits(j0, blk0, i);
         const uint32_t causal = range_bits(j0, 0, i - 1);  // drawn pairs are j < i
         if (a.thr > 0) {
+            // u < thr for thr in [1, 2^32] is u <= thr - 1 in 32 bits
+            const uint32_t tm1 = a.thr > 0xFFFFFFFFull ? 0xFFFFFFFFu : (uint32_t)(a.thr - 1);
 #pragma unroll 1
             for (int32_t s = s0; s < s1; ++s) {
                 const uint32_t seed = a.seeds.v[s];
@@ -99,10 +99,10 @@ __global__ void __launch_bounds__(kBitsThreads) k_mask_bits(const MaskBitsArgs a
                         make_uint4((uint32_t)((j0 >> 2) + c), (uint32_t)i, a.stream, a.layer_key),
                         seed, head_key);
                     uint32_t keep = 0;
-                    keep |= ((uint64_t)u.x < a.thr) ? 1u : 0u;
-                    keep |= ((uint64_t)u.y < a.thr) ? 2u : 0u;
-                    keep |= ((uint64_t)u.z < a.thr) ? 4u : 0u;
-                    keep |= ((uint64_t)u.w < a.thr) ? 8u : 0u;
+                    keep |= (u.x <= tm1) ? 1u : 0u;
+                    keep |= (u.y <= tm1) ? 2u : 0u;
+                    keep |= (u.z <= tm1) ? 4u : 0u;
+                    keep |= (u.w <= tm1) ? 8u : 0u;
                     bits |= (keep & need) << (4 * c);
                 }
             }
