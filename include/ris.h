@@ -296,7 +296,7 @@ ris_status ris_kernel_timer_samples(double *total_ms, int64_t *launches, double 
 /* Attention kernel design a layer call on `mask` uses for this input dtype and head_dim
  * (host-only, no device work): 0 register gather, 2 tcgen05 masked dense tiles,
  * 3 fp32 gather, 4 dense-suffix split; -1 for invalid arguments. bf16 calls use tiles when
- * the mask is dense or keeps at least 6.1% (head_dim 128) or 11.1% (head_dim 64) of the
+ * the mask is dense or keeps at least 6.8% (head_dim 128) or 11.1% (head_dim 64) of the
  * causal pairs in what a gather would fetch (and always when heads/kv_heads > 8, which this
  * call does not see). The dense-suffix split applies to masks (not per seed) with Structural
  * blocks of at least 256 tokens or a local window of at least 256 keys: every key of row i

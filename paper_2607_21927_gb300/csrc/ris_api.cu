@@ -195,12 +195,12 @@ const char *forced_design()
 // Union density at and above which masked dense tiles beat gathering pair by pair (bf16,
 // head dim 128): a tile costs the dense causal products (an fp16 score product, two e4m3 score
 // corrections and one value product) whatever the mask, a gathered pair 1.25 KB of K/V rows.
-// Measured crossover on Qwen2-shaped layers (head dim 128): 6.1% of the causal pairs at
-// N = 65536, 6.35% at N = 32768 (tiles 13.0 / 3.34 ms per launch; the gather on the fp8
-// operands 12.59 / 3.10 ms at 5.85%, 14.55 / 3.58 ms at 6.8%); on TinyLlama-shaped layers (head dim 64, 32 query and 4 KV
+// Measured crossover on Qwen2-shaped layers (head dim 128): 6.8% of the causal pairs at
+// N = 65536 and N = 32768 (tiles 13.25 / 3.34 ms per launch; the gather on the fp8 operands
+// 11.38 / 2.89 ms at 5.85%, 13.15 / 3.33 ms at 6.8%); on TinyLlama-shaped layers (head dim 64, 32 query and 4 KV
 // heads, N = 16384, three bf16 score products) 11.1% (tiles 1.94 ms, the gather 1.69 / 1.99 ms
 // at 9.6% / 11.4%), where the tiles are half the products but the same softmax work.
-constexpr double kTileDensity = 0.061;
+constexpr double kTileDensity = 0.068;
 constexpr double kTileDensity64 = 0.111;
 
 // Shortest dense span (Structural block or local window) for which the split pays: two
