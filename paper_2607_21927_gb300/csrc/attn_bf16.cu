@@ -40,6 +40,8 @@
 // warps fit on an SM. In the fp8 form (one set per task) each thread parks its query fragments
 // and output accumulators in its own lane of tensor memory (128 columns per CTA) and reloads
 // them around the products that use them: 168 registers, three CTAs per SM instead of two.
+// The loads that feed one product share one wait, and a store of the accumulators is waited
+// for only before their next load.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_fp8.h>
@@ -135,6 +137,37 @@ __device__ __forceinline__ void tm_ld<16>(uint32_t taddr, uint32_t *v)
                  : "memory");
 }
 __device__ __forceinline__ void tm_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// loads that share one wait: issue them with tm_issue<N>, then tm_wait_ld, then tm_pin<N> on
+// each destination (an empty asm that redefines the registers, so that no use of them is
+// scheduled before the wait)
+template <int N>
+__device__ __forceinline__ void tm_issue(uint32_t taddr, uint32_t *v);
+template <>
+__device__ __forceinline__ void tm_issue<8>(uint32_t taddr, uint32_t *v)
+{
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7])
+                 : "r"(taddr)
+                 : "memory");
+}
+template <>
+__device__ __forceinline__ void tm_issue<16>(uint32_t taddr, uint32_t *v)
+{
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+                   "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+                 : "r"(taddr)
+                 : "memory");
+}
+__device__ __forceinline__ void tm_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void tm_pin(uint32_t *v)
+{
+#pragma unroll
+    for (int i = 0; i < N; i += 8)
+        asm volatile("" : "+r"(v[i]), "+r"(v[i + 1]), "+r"(v[i + 2]), "+r"(v[i + 3]), "+r"(v[i + 4]), "+r"(v[i + 5]),
+                     "+r"(v[i + 6]), "+r"(v[i + 7]));
+}
 // the output accumulators o[8][4] <-> 32 columns
 __device__ __forceinline__ void tm_st_o(uint32_t taddr, float (&o)[8][4])
 {
@@ -145,17 +178,20 @@ __device__ __forceinline__ void tm_st_o(uint32_t taddr, float (&o)[8][4])
         for (int i = 0; i < 16; ++i) w[i] = __float_as_uint(o[4 * h + i / 4][i % 4]);
         tm_st<16>(taddr + 16 * h, w);
     }
-    tm_wait_st();
 }
 __device__ __forceinline__ void tm_ld_o(uint32_t taddr, float (&o)[8][4])
 {
-    uint32_t w[16];
+    uint32_t w[2][16];
+    tm_wait_st();  // the previous store of these columns
+    tm_issue<16>(taddr, w[0]);
+    tm_issue<16>(taddr + 16, w[1]);
+    tm_wait_ld();
+    tm_pin<16>(w[0]);
+    tm_pin<16>(w[1]);
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        tm_ld<16>(taddr + 16 * h, w);
+    for (int h = 0; h < 2; ++h)
 #pragma unroll
-        for (int i = 0; i < 16; ++i) o[4 * h + i / 4][i % 4] = __uint_as_float(w[i]);
-    }
+        for (int i = 0; i < 16; ++i) o[4 * h + i / 4][i % 4] = __uint_as_float(w[h][i]);
 }
 
 __device__ __forceinline__ uint32_t transpose8x8(uint32_t x)
@@ -511,10 +547,17 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
 #pragma unroll
             for (int e = 0; e < 4; ++e) sa[c][e] = sb[c][e] = sl[c][e] = 0.f;
         if constexpr (TQ) {
+            uint32_t wq[2][16], w8[8];
+            tm_issue<16>(tl, wq[0]);
+            tm_issue<16>(tl + 16, wq[1]);
+            tm_issue<8>(tl + 32, w8);
+            tm_wait_ld();
+            tm_pin<16>(wq[0]);
+            tm_pin<16>(wq[1]);
+            tm_pin<8>(w8);
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                uint32_t w[16];
-                tm_ld<16>(tl + 16 * h, w);
+                const uint32_t *w = wq[h];
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     const int ks = 4 * h + k;
@@ -523,8 +566,6 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
                                  w[4 * k + 3]);
                 }
             }
-            uint32_t w8[8];
-            tm_ld<8>(tl + 32, w8);
 #pragma unroll
             for (int ks = 0; ks < D / 32; ++ks)
                 mma16832_e4m3(sl[ks & 1], kl0[2 * ks], kl1[2 * ks], kl0[2 * ks + 1], kl1[2 * ks + 1], w8[2 * ks],
