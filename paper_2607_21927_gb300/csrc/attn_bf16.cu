@@ -37,7 +37,7 @@
 // V is an exact bf16 input. Unrotated bf16 q/k are exact and take one product each.
 //
 // Residency. The gather is bound by the gathered rows it keeps in flight, hence by how many
-// warps fit on an SM. In the fp8 form (one set per task) each thread parks its query fragments
+// warps fit on an SM. In the fp8 form each thread parks its query fragments
 // and output accumulators in its own lane of tensor memory (128 columns per CTA) and reloads
 // them around the products that use them: 168 registers, three CTAs per SM instead of two.
 // The loads that feed one product share one wait, and a store of the accumulators is waited
@@ -303,7 +303,7 @@ template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE,
 __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t tbase)
 {
     static_assert(!E8 || (D == 128 && QSPLIT && KSPLIT && WIDE), "the fp8 operands: head dim 128, 32-byte loads");
-    static_assert(!TQ || (E8 && !SEEDS), "query fragments and accumulators in TMEM: the fp8 form, one set");
+    static_assert(!TQ || E8, "query fragments and accumulators in TMEM: the fp8 form");
     constexpr int KSTEPS = D / 16;  // k-steps of the score product
     constexpr int KW = D / 8;       // 32-bit words of one K row per lane (D/4 elements)
     constexpr int VW = D / 16;      // 32-bit words of one V row per lane (D/8 elements)
@@ -718,6 +718,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
         load_chunk(64, nxt);
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+        if constexpr (TQ) tm_st_o(tl + 64, o);
         m0 = m1 = -INFINITY;
         l0 = l1 = 0.f;
     }
@@ -726,7 +727,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
 
 // F8: the queries and keys came from launch_fp8_prep; which of its two schemes it wrote
 // follows from the bounds at a.qk_bound, read here on the device as it did.
-// F8 (one set per task): the query fragments and output accumulators live in tensor memory
+// F8: the query fragments and output accumulators live in tensor memory
 // (each thread's own TMEM lane, 128 columns per CTA), which leaves room for three CTAs of four
 // warps per SM instead of two, and so more gathered rows in flight.
 constexpr int kGatherTmemCols = 128;
@@ -734,7 +735,6 @@ template <int D, bool QSPLIT, bool KSPLIT, bool WIDE, typename TIdx, bool DENSE,
 __global__ void __launch_bounds__(kAttnWarps * 32, F8 ? 3 : RIS_ATTN_MIN_BLOCKS) k_attn_bf16(const AttnArgs a)
 {
     if constexpr (F8) {
-        static_assert(!SEEDS, "per-seed sets take the bf16 pairs");
         __shared__ uint32_t tbase_sh;
         const int warp = threadIdx.x >> 5;
         if (warp == 0) {
@@ -769,19 +769,15 @@ cudaError_t launch_f(const AttnArgs &a, int col_bytes, bool dense, cudaStream_t 
     constexpr bool KSPLIT = QSPLIT;
     const dim3 block(kAttnWarps * 32);
     if (!dense && a.n_sets > 1) {  // per-seed sets: one warp per (row, KV head) walks them all
-        if constexpr (F8) {
-            return cudaErrorInvalidValue;  // per-seed sets take the bf16 pairs (the caller's choice)
-        } else {
-            AttnArgs b = a;
-            b.n_tasks = (a.row1 - a.row0) * a.Hkv;
-            const unsigned grid = (unsigned)((b.n_tasks + kAttnWarps - 1) / kAttnWarps);
-            if (col_bytes == 2)
-                k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, true, false><<<grid, block, 0, s>>>(b);
-            else
-                k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, true, false><<<grid, block, 0, s>>>(b);
-            note_launch();
-            return cudaGetLastError();
-        }
+        AttnArgs b = a;
+        b.n_tasks = (a.row1 - a.row0) * a.Hkv;
+        const unsigned grid = (unsigned)((b.n_tasks + kAttnWarps - 1) / kAttnWarps);
+        if (col_bytes == 2)
+            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint16_t, false, TOut, true, F8><<<grid, block, 0, s>>>(b);
+        else
+            k_attn_bf16<D, QSPLIT, KSPLIT, WIDE, uint32_t, false, TOut, true, F8><<<grid, block, 0, s>>>(b);
+        note_launch();
+        return cudaGetLastError();
     }
     const unsigned grid = (unsigned)((a.n_tasks + kAttnWarps - 1) / kAttnWarps);
     if (dense)

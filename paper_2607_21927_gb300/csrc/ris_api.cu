@@ -656,10 +656,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     // bf16 inputs rotated here at head dim 128, on the tiles, the dense-suffix split or the bf16
     // gather: fp16 + e4m3 score operands when the bounds allow (else the bf16 pairs), written
     // by launch_fp8_prep and read alike by the tile kernel and the gather (whose fp8 form
-    // needs its 32-byte loads: values 32-byte aligned; per-seed sets keep the bf16 pairs, on
-    // which their short rows measured 1-4% faster)
+    // needs its 32-byte loads: values 32-byte aligned), per-seed sets included
     const bool tile8 = dtype == RIS_BF16 && head_dim == 128 && rotated &&
-                       (tile || ((suffix || (design == 0 && !m->per_seed)) && aligned32(v)));
+                       (tile || ((suffix || design == 0) && aligned32(v)));
     const bool q_pair = tile || suffix || tile8;  // queries as a 16-bit pair (else fp32)
     Scratch qt, qtl, kt, ktl, po, pl, v16, vmax, bound;
     const void *qu = q, *ku = k, *kl = nullptr, *q_lo = nullptr;

@@ -569,13 +569,15 @@ def test_tile_values_beyond_fp16_range(scale_exp):
         assert torch.allclose(scaled_back, base, rtol=1e-5, atol=1e-5)
 
 
-# (N, mode, density, seeds, design): the tiles, the register gather, the dense-suffix split
-FP8_SCHEME_CASES = [(1200, 0, 0.5, [1, 2], 2), (1200, 0, 0.02, [1], 0), (3000, 1, 0.1, [1], 4)]
+# (N, mode, density, seeds, design, per_seed): the tiles, the register gather, the dense-suffix
+# split, and the register gather's per-seed set loop
+FP8_SCHEME_CASES = [(1200, 0, 0.5, [1, 2], 2, False), (1200, 0, 0.02, [1], 0, False), (3000, 1, 0.1, [1], 4, False),
+                    (1300, 0, 0.03, [1, 2, 3], 0, True)]
 
 
 @pytest.mark.parametrize("case", ["fp8", "both_large", "q_beyond_fp16"])
-@pytest.mark.parametrize("N,mode,d,seeds,design", FP8_SCHEME_CASES)
-def test_fp8_score_scheme_and_its_fallback(N, mode, d, seeds, design, case):
+@pytest.mark.parametrize("N,mode,d,seeds,design,per_seed", FP8_SCHEME_CASES)
+def test_fp8_score_scheme_and_its_fallback(N, mode, d, seeds, design, per_seed, case):
     """At head dim 128 with rotated bf16 inputs the tiles, the gather and the dense-suffix split
     take fp16 score products with e4m3 corrections when bounds of |q~| and |k~| allow (their
     product below about 1e5, each below 2^15 so that the fp16 hi parts stay finite); otherwise
@@ -583,7 +585,7 @@ def test_fp8_score_scheme_and_its_fallback(N, mode, d, seeds, design, case):
     channel each, in channel pairs where the other tensor is zero (so the scores stay moderate):
     at 9 they take the fp8 path; at 900 each the product rules it out; a query channel of 69632
     with keys scaled by 2^-7 passes the product rule but not fp16's range. Every case must match
-    the oracle."""
+    the oracle, every seed's output of a per-seed mask too."""
     Hq, Hkv, D = 6, 2, 128
     big_q, big_k, k_scale = {"fp8": (9.0, 9.0, 1.0), "both_large": (900.0, 900.0, 1.0),
                              "q_beyond_fp16": (69632.0, 1.0, 2.0 ** -7)}[case]
@@ -596,13 +598,14 @@ def test_fp8_score_scheme_and_its_fallback(N, mode, d, seeds, design, case):
     k[:, :, 3] = 0
     k[:, :, 3 + D // 2] = 0
     qn, kn, vn = to_np(q.cpu()), to_np(k.cpu()), to_np(v.cpu())
-    m = ris.ris_mask_generate(N, Hkv, mode, d, seeds)
+    m = ris.ris_mask_generate(N, Hkv, mode, d, seeds, per_seed=per_seed)
     assert ris.ris_attention_design(m, torch.bfloat16, D) == design
     out, lse = ris.ris_attention_masked(m, q, k, v, rope=ris.rope_cfg(3, 1e6, 256), out_dtype=torch.float32,
                                         return_lse=True)
     torch.cuda.synchronize()
     ris.ris_device_status()
     m.free()
-    ref, ref_lse = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e6, 256)
-    check_bf16_path(to_np(out), ref)
-    np.testing.assert_allclose(to_np(lse).T, ref_lse, rtol=0, atol=2e-3)
+    for s in range(len(seeds) if per_seed else 1):
+        ref, ref_lse = run_oracle(qn, kn, vn, mode, d, seeds, 3, 1e6, 256, seed_index=s if per_seed else -1)
+        check_bf16_path(to_np(out[s] if per_seed else out), ref)
+        np.testing.assert_allclose(to_np(lse[s] if per_seed else lse).T, ref_lse, rtol=0, atol=2e-3)
