@@ -908,7 +908,10 @@ def main():
 
         # Host transfers overlap the compute: one stream brings the layers' q/k/v in, another
         # takes the outputs out, both ordered against the compute stream with per-layer events.
-        h2d_s, d2h_s = torch.cuda.Stream(), torch.cuda.Stream()
+        # Masks are built on their own stream: the mask call waits for its own kernels (to size
+        # the key lists), which on the compute stream would also drain every queued layer at
+        # each run boundary and leave the device idle while the host resumes.
+        h2d_s, d2h_s, mask_s = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
         in_ready = [torch.cuda.Event() for _ in range(L)]
         layer_free = [torch.cuda.Event() for _ in range(L)]
         out_ready = [[torch.cuda.Event() for _ in range(L)] for _ in runs]
@@ -925,7 +928,9 @@ def main():
                     vs[layer].copy_(hv[layer], non_blocking=True)
                     in_ready[layer].record(h2d_s)
             for ri, (name, mode, dens, ns) in enumerate(runs):
-                m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom, per_seed=per_seed)
+                m = ris.ris_mask_generate(N, Hkv, mode, dens, list(range(ns)), opts=geom, per_seed=per_seed,
+                                          stream=mask_s)
+                stream.wait_stream(mask_s)
                 b = ris.ris_mask_row_split(m, world) if strong else None
                 for layer in range(L):
                     stream.wait_event(in_ready[layer])
@@ -944,6 +949,7 @@ def main():
                         d2h_s.wait_event(out_ready[ri][layer])
                         ho[ri][layer].copy_(outs[ri][layer], non_blocking=True)
                         out_free[ri][layer].record(d2h_s)
+                mask_s.wait_stream(stream)  # the mask is released after its layers
                 m.free()
             first[0] = False
 

@@ -76,6 +76,11 @@ SMALL = [
     (129, 12, 2, 128, torch.bfloat16, 0, 0.3, 3, 3, 64),
     (257, 6, 2, 128, torch.bfloat16, 2, 1.0, 1, 3, 64),
     (130, 6, 2, 128, torch.bfloat16, 0, 0.01, 1, 1, 4096),
+    # the register gather's fp8 form (rotated bf16, head dim 128) at 1, 5 and 8 query heads per
+    # KV head: every head of the tensor-core tile's N dimension used, or some left empty
+    (700, 2, 2, 128, torch.bfloat16, 1, 0.01, 2, 1, 4096),
+    (901, 5, 1, 128, torch.bfloat16, 0, 0.03, 1, 3, 256),
+    (700, 8, 1, 128, torch.bfloat16, 0, 0.02, 1, 3, 256),
 ]
 
 
