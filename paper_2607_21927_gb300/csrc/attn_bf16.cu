@@ -33,8 +33,10 @@
 //   - S^T = K_hi Q_hi + K_hi Q_lo + K_lo Q_hi (the lo*lo term is below 2^-16);
 //   - or, at head dim 128 with rotated bf16 inputs, fp16 hi parts with e4m3 lo parts (E8
 //     below);
-//   - P is split into bf16 hi + lo and O^T += V^T P_hi + V^T P_lo.
-// V is an exact bf16 input. Unrotated bf16 q/k are exact and take one product each.
+//   - P is split into bf16 hi + lo and O^T += V^T P_hi + V^T P_lo against the exact bf16 V;
+//   - E8: P as one fp16 against the values' fp16 copy (exact after a power-of-two scale), the
+//     row sums adding P as rounded, as the tile kernel does.
+// Unrotated bf16 q/k are exact and take one product each.
 //
 // Residency. The gather is bound by the gathered rows it keeps in flight, hence by how many
 // warps fit on an SM. In the fp8 form each thread parks its query fragments
@@ -421,7 +423,10 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
     const char *kbl = !KSPLIT ? nullptr
                       : E8    ? reinterpret_cast<const char *>(a.k_lo) + head_off + D + 32 * q
                               : reinterpret_cast<const char *>(a.k_lo) + head_off + 2 * kelem<D, WIDE>(0, q);
-    const char *vb = reinterpret_cast<const char *>(a.v) + head_off + 2 * velem<D, WIDE>(0, p);
+    // E8: the values are read as their fp16 copy (scaled into range by 2^-E, E from the largest
+    // |v|), and P enters the value product as one fp16 with the row sums adding P as rounded
+    const char *vb = reinterpret_cast<const char *>(E8 ? a.v16 : a.v) + head_off + 2 * velem<D, WIDE>(0, p);
+    const float vsc = E8 ? pow2i(v_scale_exp(*a.v_absmax)) : 1.f;  // 2^E, undone in the epilogue
 
     float o[MT][4];
 #pragma unroll
@@ -447,9 +452,9 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
                 const float4 x0 = src[0], x1 = src[1];
                 const float run[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    o[4 * r + j][hs] = run[2 * j];
-                    o[4 * r + j][2 + hs] = run[2 * j + 1];
+                for (int j = 0; j < 4; ++j) {  // into the values' scale (E8: 2^-E, exact)
+                    o[4 * r + j][hs] = run[2 * j] / vsc;
+                    o[4 * r + j][2 + hs] = run[2 * j + 1] / vsc;
                 }
             }
         }
@@ -636,15 +641,27 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
         const float mu0 = (m0 == -INFINITY) ? 0.f : m0, mu1 = (m1 == -INFINITY) ? 0.f : m1;
         const float p0 = exp2f(s0 - mu0), p1 = exp2f(s1 - mu1);
         const float p2 = exp2f(s2 - mu0), p3 = exp2f(s3 - mu1);
-        l0 += p0 + p2;
-        l1 += p1 + p3;
-        // P = P_hi + P_lo in bf16; transposed into the B operand P[head p][keys 2q.., 2q+8..]
-        const float h0 = __bfloat162float(__float2bfloat16_rn(p0)), h1 = __bfloat162float(__float2bfloat16_rn(p1));
-        const float h2 = __bfloat162float(__float2bfloat16_rn(p2)), h3 = __bfloat162float(__float2bfloat16_rn(p3));
-        const uint32_t pb0 = transpose8x8(pack_bf16(h0, h1));
-        const uint32_t pb1 = transpose8x8(pack_bf16(h2, h3));
-        const uint32_t pl0 = transpose8x8(pack_bf16(p0 - h0, p1 - h1));
-        const uint32_t pl1 = transpose8x8(pack_bf16(p2 - h2, p3 - h3));
+        // P transposed into the B operand P[head p][keys 2q.., 2q+8..]: E8 one fp16 (the row sums
+        // add it as rounded, so each weight's rounding moves the output by at most 2^-11 of that
+        // weight times |v_j - o|), else P_hi + P_lo in bf16
+        uint32_t pb0, pb1, pl0 = 0u, pl1 = 0u;
+        if constexpr (E8) {
+            const __half2 f01 = __floats2half2_rn(p0, p1), f23 = __floats2half2_rn(p2, p3);
+            const float2 r01 = __half22float2(f01), r23 = __half22float2(f23);
+            l0 += r01.x + r23.x;
+            l1 += r01.y + r23.y;
+            pb0 = transpose8x8(*reinterpret_cast<const uint32_t *>(&f01));
+            pb1 = transpose8x8(*reinterpret_cast<const uint32_t *>(&f23));
+        } else {
+            l0 += p0 + p2;
+            l1 += p1 + p3;
+            const float h0 = __bfloat162float(__float2bfloat16_rn(p0)), h1 = __bfloat162float(__float2bfloat16_rn(p1));
+            const float h2 = __bfloat162float(__float2bfloat16_rn(p2)), h3 = __bfloat162float(__float2bfloat16_rn(p3));
+            pb0 = transpose8x8(pack_bf16(h0, h1));
+            pb1 = transpose8x8(pack_bf16(h2, h3));
+            pl0 = transpose8x8(pack_bf16(p0 - h0, p1 - h1));
+            pl1 = transpose8x8(pack_bf16(p2 - h2, p3 - h3));
+        }
 
         // ---- O^T += V^T P^T
         if constexpr (TQ) tm_ld_o(tl + 64, o);
@@ -654,8 +671,12 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
             const uint32_t a1 = __byte_perm(v0[mt], v1[mt], 0x7632);
             const uint32_t a2 = __byte_perm(v2[mt], v3[mt], 0x5410);
             const uint32_t a3 = __byte_perm(v2[mt], v3[mt], 0x7632);
-            mma16816(o[mt], a0, a1, a2, a3, pb0, pb1);
-            mma16816(o[mt], a0, a1, a2, a3, pl0, pl1);
+            if constexpr (E8) {
+                mma16816_f16(o[mt], a0, a1, a2, a3, pb0, pb1);
+            } else {
+                mma16816(o[mt], a0, a1, a2, a3, pb0, pb1);
+                mma16816(o[mt], a0, a1, a2, a3, pl0, pl1);
+            }
         }
         if constexpr (TQ) tm_st_o(tl + 64, o);
         if (more)
@@ -676,7 +697,7 @@ __device__ __forceinline__ void gather_task(const AttnArgs &a, int eb, uint32_t 
         l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, off);
         l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, off);
     }
-    const float inv0 = 1.f / l0, inv1 = 1.f / l1;
+    const float inv0 = vsc / l0, inv1 = vsc / l1;
     const int h0 = 2 * q, h1 = 2 * q + 1;
     TOut *out = reinterpret_cast<TOut *>(a.out) + (((int64_t)t.s * a.N + t.i) * a.Hq + (int64_t)t.g * a.G) * D;
     // runs of 8 consecutive head-dim elements: words 4r .. 4r+3 of the lane's V layout

@@ -683,9 +683,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
         RIS_CUDA(kt.alloc(nk * (dtype == RIS_BF16 ? 2 : 4), s));
         if (dtype == RIS_BF16) RIS_CUDA(ktl.alloc(nk * 2, s));
         if (tile8) {
-            // bounds (and the values as fp16 for the tile kernels), then the operands: two launches
+            // bounds, then the operands and the values as fp16: two launches
             RIS_CUDA(bound.alloc(3 * sizeof(float), s));
-            if (tile || suffix) RIS_CUDA(v16.alloc(nk * 2, s));
+            RIS_CUDA(v16.alloc(nk * 2, s));
             Fp8PrepArgs pa{};
             pa.q = q;
             pa.k = k;
@@ -694,7 +694,7 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
             pa.q_lo = qtl.p;
             pa.k_hi = kt.p;
             pa.k_lo = ktl.p;
-            pa.v16 = (tile || suffix) ? v16.p : nullptr;
+            pa.v16 = v16.p;
             pa.bounds = (float *)bound.p;
             pa.N = N;
             pa.q_rows = q_rows;
@@ -754,9 +754,9 @@ ris_status run_attention(const ris_mask_s *m, const void *q, const void *k, cons
     a.row1 = row1;
     a.n_tasks = (int64_t)a.n_sets * (row1 - row0) * kv_heads;
     a.qk_bound = tile8 ? (const float *)bound.p : nullptr;
-    if (tile || suffix) {
-        // the tile kernel's value product takes the values as fp16 (scaled into range), written
-        // above with the fp8 operands or here
+    if (tile || suffix || tile8) {
+        // the value products of the tile kernel and of the gather's fp8 form take the values as
+        // fp16 (scaled into range), written above with the fp8 operands or here
         if (!tile8) {
             const size_t nv = (size_t)N * kv_heads * head_dim;
             RIS_CUDA(v16.alloc(nv * 2, s));
