@@ -117,27 +117,6 @@ __device__ __forceinline__ void tm_st<16>(uint32_t taddr, const uint32_t *v)
                  "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
                  : "memory");
 }
-template <int N>
-__device__ __forceinline__ void tm_ld(uint32_t taddr, uint32_t *v);
-template <>
-__device__ __forceinline__ void tm_ld<8>(uint32_t taddr, uint32_t *v)
-{
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n\t"
-                 "tcgen05.wait::ld.sync.aligned;"
-                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7])
-                 : "r"(taddr)
-                 : "memory");
-}
-template <>
-__device__ __forceinline__ void tm_ld<16>(uint32_t taddr, uint32_t *v)
-{
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
-                 "tcgen05.wait::ld.sync.aligned;"
-                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-                   "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
-                 : "r"(taddr)
-                 : "memory");
-}
 __device__ __forceinline__ void tm_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 // loads that share one wait: issue them with tm_issue<N>, then tm_wait_ld, then tm_pin<N> on
 // each destination (an empty asm that redefines the registers, so that no use of them is
@@ -170,7 +149,8 @@ __device__ __forceinline__ void tm_pin(uint32_t *v)
         asm volatile("" : "+r"(v[i]), "+r"(v[i + 1]), "+r"(v[i + 2]), "+r"(v[i + 3]), "+r"(v[i + 4]), "+r"(v[i + 5]),
                      "+r"(v[i + 6]), "+r"(v[i + 7]));
 }
-// the output accumulators o[8][4] <-> 32 columns
+// the output accumulators o[8][4] <-> 32 columns; a store is not waited for here, the next
+// load of the same columns (tm_ld_o) waits for it
 __device__ __forceinline__ void tm_st_o(uint32_t taddr, float (&o)[8][4])
 {
     uint32_t w[16];
