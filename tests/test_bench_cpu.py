@@ -36,3 +36,29 @@ def test_reference_arm_line():
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["config"]["name"] == "C1" and line["higher_is_better"] is True
+
+
+def test_recorded_traffic_follows_the_source_hashes(monkeypatch, tmp_path):
+    """The DRAM bytes recorded under profiles/traffic.json count only while every kernel source
+    they were captured on is unchanged (sha256 prefix); a changed source gives no traffic."""
+    import hashlib
+
+    sys.path.insert(0, ROOT)
+    import bench
+
+    csrc = tmp_path / "paper_2607_21927_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (tmp_path / "profiles").mkdir()
+    (csrc / "a.cu").write_text("kernel a\n")
+    (csrc / "b.cu").write_text("kernel b\n")
+    h = {n: hashlib.sha256((csrc / n).read_bytes()).hexdigest()[:16] for n in ("a.cu", "b.cu")}
+    rec = {"a.cu": {"W": {"source_sha256_16": h["a.cu"], "dram_bytes_per_launch_full_size": 123}},
+           "a.cu+b.cu": {"W": {"source_sha256_16": [h["a.cu"], h["b.cu"]], "dram_bytes_per_launch_full_size": 456}}}
+    (tmp_path / "profiles" / "traffic.json").write_text(json.dumps(rec))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.recorded_traffic(("a.cu",), "W") == 123
+    assert bench.recorded_traffic(("a.cu", "b.cu"), "W") == 456
+    assert bench.recorded_traffic(("a.cu",), "other") is None
+    (csrc / "b.cu").write_text("kernel b, edited\n")
+    assert bench.recorded_traffic(("a.cu", "b.cu"), "W") is None
+    assert bench.recorded_traffic(("a.cu",), "W") == 123
