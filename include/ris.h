@@ -155,6 +155,9 @@ ris_status ris_rope_freqs(const ris_rope_cfg *rope, int64_t N, int32_t head_dim,
  * keeps its own mask. Output: bitmap + CSR in device memory owned by *out_mask.
  * seeds: HOST array of n_seeds values, 1 <= n_seeds <= 256. kv_heads is used only when
  * opts->per_head = 1. Blocks: the CSR size is read back before the key lists are written.
+ * The wait covers `stream` only: a mask built on a stream of its own (ordered before the
+ * attention calls that read it, and freed after them) leaves work queued on other streams
+ * running while the host waits.
  * Errors: RIS_ERR_INVALID (N < 1 or > 2^31, density outside (0,1], bad opts or seeds),
  * RIS_ERR_OOM, RIS_ERR_CUDA. On error *out_mask is NULL. */
 ris_status ris_mask_generate(int64_t N, int32_t kv_heads, int32_t mode, double density,
